@@ -1,0 +1,375 @@
+"""Benchmark of the DAR attention hot path on GB300.
+
+One step = one decode step of the 160M-like workload (B32 H12 d64, context 4096,
+w128, d_down 16, bf16): ``dar_cache_append`` of one token per sequence (the
+token leaving the window is down-projected into its page) followed by
+``dar_attn_decode``.  ``value`` is algorithmic bytes per step / device time
+(GB/s, whole job).  The caches rotate over enough copies that the bytes
+touched between two uses of one copy exceed 4x L2, so no step reads a warm L2.
+
+Also reported on the same line: the decode kernel's roofline (live CUDA-event
+duration of that kernel inside the timed region), an end-to-end number through
+the public API with host buffers, the CPU oracle on a bounded sample, the SM
+clocks seen during the timed region, and the 410M-like prefill (B8 H16 N8192
+w512 d_down 16, bf16) in TFLOP/s.
+
+``--impl reference`` times the CPU oracle (the reference arm of this build) on
+the same workload and prints the same kind of line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode GB/s & prefill TFLOP/s of DAR attention, % of GB300 roofline (1 GPU)"
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), \
+            "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ----------------------------------------------------------------------------- distributed
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def init_dist(world, backend):
+    import torch.distributed as dist
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend)
+    return dist
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """Largest value of x over all ranks (the job's time is its slowest rank's)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (getattr(self, "out", "") or "").strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- oracle (CPU) timing
+
+def oracle_decode_sample(cfg, budget_s=12.0, nthreads=None):
+    """Time the CPU oracle on whole sequences of the decode workload until about
+    ``budget_s`` seconds are spent; returns (GB/s over the cache bytes of the
+    sample, cores, description)."""
+    import oracle
+    from paper_2606_18587_gb300 import inputs as I
+    from paper_2606_18587_gb300 import workloads as W
+    nthreads = nthreads or os.cpu_count() or 1
+    lens = I.decode_lengths(cfg)
+    Dk, Uk, Dv, Uv = I.projections(cfg.seed, cfg.Hkv, cfg.d, cfg.dd)
+    q = I.decode_query(cfg)
+    spent, nbytes, nseq = 0.0, 0, 0
+    for b in range(cfg.B):
+        kb, vb = I.decode_history(cfg, b, int(lens[b]))
+        t0 = time.perf_counter()
+        oracle.decode(np.ascontiguousarray(q[b:b + 1]), kb[None], vb[None], lens[b:b + 1], Dk, Uk, Dv, Uv, cfg.w,
+                      cfg.dtype, nthreads=nthreads)
+        spent += time.perf_counter() - t0
+        sub = I.Decode(cfg.name, cfg.seed, 1, cfg.Hq, cfg.Hkv, cfg.d, cfg.dd, cfg.w, cfg.dtype, L=int(lens[b]))
+        nbytes += W.decode_step_bytes(sub, lens[b:b + 1])
+        nseq += 1
+        if spent >= budget_s:
+            break
+    return nbytes / spent / 1e9, nthreads, f"{nseq} of {cfg.B} sequences (all {cfg.Hq} heads), one decode step each"
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_ours(args, world, rank, local):
+    import torch
+    from paper_2606_18587_gb300 import dar
+    from paper_2606_18587_gb300 import inputs as I
+    from paper_2606_18587_gb300 import workloads as W
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    init_dist(world, "nccl")
+    hbm_peak, tc_peak, tc_sus, peak_src = load_peaks()
+    cfg = I.DECODE_160M
+    K, Wm = args.steps, args.warmup
+
+    # rotating caches: each step uses the next copy, so between two uses of one copy
+    # the other copies (more than 4x L2 in total) pass through the memory system
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    one = W.decode_step_bytes(cfg, I.decode_lengths(cfg))
+    R = max(2, int(np.ceil(4 * l2 / one)) + 1)
+    wls = [W.DecodeWorkload(cfg, extra_tokens=K + Wm + 8) for _ in range(R)]
+    knew, vnew = [], []
+    for s in range(R):
+        kh, vh = I.decode_new_tokens(cfg, s)
+        knew.append(W.upload(kh, cfg.dtype))
+        vnew.append(W.upload(vh, cfg.dtype))
+    outs = [torch.empty_like(wl.q) for wl in wls]
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        wl = wls[i % R]
+        dar.dar_cache_append(wl.cache, knew[i % R], vnew[i % R], wl.Dk, wl.Dv)
+        dar.dar_attn_decode(wl.cache, wl.q, wl.Uk, wl.Uv, wl.workspace, out=outs[i % R])
+
+    for i in range(Wm):
+        step(i)
+    torch.cuda.synchronize()
+    lens_at = [W.download(wl.cache.seq_lens).astype(np.int64) for wl in wls]
+
+    # expected bytes of the timed steps (lengths grow by one per step of a copy)
+    step_bytes, dec_bytes = [], []
+    for i in range(Wm, Wm + K):
+        c = i % R
+        L_before = lens_at[c] + (i - Wm) // R
+        step_bytes.append(W.append_step_bytes(cfg, L_before) + W.decode_step_bytes(cfg, L_before + 1))
+        dec_bytes.append(W.decode_step_bytes(cfg, L_before + 1))
+
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for j in range(K):
+            i = Wm + j
+            wl = wls[i % R]
+            ev[j][0].record(stream)
+            dar.dar_cache_append(wl.cache, knew[i % R], vnew[i % R], wl.Dk, wl.Dv)
+            ev[j][1].record(stream)
+            dar.dar_attn_decode(wl.cache, wl.q, wl.Uk, wl.Uv, wl.workspace, out=outs[i % R])
+            ev[j][2].record(stream)
+        stop.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+    total_ms = max_over_ranks(start.elapsed_time(stop), world, dev)
+    dec_ms = [ev[j][1].elapsed_time(ev[j][2]) for j in range(K)]
+    app_ms = [ev[j][0].elapsed_time(ev[j][1]) for j in range(K)]
+    status = sum(wl.cache.device_status() for wl in wls)
+    if status:
+        raise RuntimeError(f"device status {status} during the benchmark")
+
+    value = world * sum(step_bytes) / (total_ms * 1e-3) / 1e9
+    dec_gbs = float(np.mean(dec_bytes)) / (float(np.mean(dec_ms)) * 1e-3) / 1e9
+
+    # ---- end to end through the public API: host buffers, copies inside the timed region
+    pin = lambda t: t.cpu().pin_memory()  # noqa: E731
+    hq = [pin(wl.q) for wl in wls]
+    hk = [pin(k) for k in knew]
+    hv = [pin(v) for v in vnew]
+    hout = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    lens_e2e = [W.download(wl.cache.seq_lens).astype(np.int64) for wl in wls]
+    e2e_bytes = []
+    for j in range(K):
+        L_before = lens_e2e[j % R] + j // R
+        e2e_bytes.append(W.append_step_bytes(cfg, L_before) + W.decode_step_bytes(cfg, L_before + 1))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for j in range(K):
+        c = j % R
+        wl = wls[c]
+        knew[c].copy_(hk[c], non_blocking=True)
+        vnew[c].copy_(hv[c], non_blocking=True)
+        wl.q.copy_(hq[c], non_blocking=True)
+        dar.dar_cache_append(wl.cache, knew[c], vnew[c], wl.Dk, wl.Dv)
+        dar.dar_attn_decode(wl.cache, wl.q, wl.Uk, wl.Uv, wl.workspace, out=outs[c])
+        hout[c].copy_(outs[c], non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_val = world * sum(e2e_bytes) / (e2e_ms * 1e-3) / 1e9
+    h2d = (knew[0].numel() + vnew[0].numel() + wls[0].q.numel()) * knew[0].element_size()
+    d2h = outs[0].numel() * outs[0].element_size()
+
+    # ---- prefill (410M-like) on the same GPU
+    pcfg = I.PREFILL_410M
+    pw = W.PrefillWorkload(pcfg)
+    flops = W.prefill_flops(pcfg)
+    for _ in range(max(3, Wm)):
+        pw.run()
+    torch.cuda.synchronize()
+    pk = max(3, min(K, 10))
+    pev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(pk)]
+    for a, b in pev:
+        a.record(stream)
+        pw.run()
+        b.record(stream)
+    torch.cuda.synchronize()
+    p_ms = float(np.mean([a.elapsed_time(b) for a, b in pev]))
+    p_tflops = flops / (p_ms * 1e-3) / 1e12
+    prefill = {"workload": pcfg.name, "tflops": round(p_tflops, 2), "ms": round(p_ms, 4),
+               "flops_per_call": flops, "exps_per_call": W.prefill_exps(pcfg),
+               "roofline": {"bound": "tensor", "achieved": round(p_tflops, 2), "peak": tc_peak, "unit": "TFLOP/s",
+                            "frac": round(p_tflops / tc_peak, 4), "traffic": None,
+                            "peak_source": f"{peak_src} bf16 dense (burst)"}}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        gbs, cores, sample = oracle_decode_sample(cfg, budget_s=args.cpu_budget)
+        cpu = {"value": round(gbs, 4), "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world, "steps": K, "warmup": Wm,
+            "ms_per_step": round(total_ms / K, 5), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,1) keys/values/queries)",
+            "config": {"workload": cfg.name, "B": cfg.B, "Hq": cfg.Hq, "Hkv": cfg.Hkv, "context": cfg.L,
+                       "w": cfg.w, "d": cfg.d, "d_down": cfg.dd, "step": "append 1 token + decode",
+                       "l2": f"{R} rotating cache copies ({R * one / 1e6:.0f} MB > 4x L2 {l2 / 1e6:.0f} MB)",
+                       "parallelism": f"{world} independent replicas" if world > 1 else "single GPU"},
+            "clocks": clk.summary(),
+            "e2e": {"value": round(e2e_val, 2), "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": 2 * K,
+            "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                         "frac": round(dec_gbs / hbm_peak, 4), "traffic": None,
+                         "kernel": "decode_kernel<bf16,16,1>", "bytes_per_launch": int(np.mean(dec_bytes)),
+                         "us_per_launch": round(1e3 * float(np.mean(dec_ms)), 3),
+                         "peak_source": f"{peak_src} HBM copy"},
+            "append_us_per_launch": round(1e3 * float(np.mean(app_ms)), 3),
+            "prefill": prefill,
+        }
+        if cpu:
+            line["cpu_baseline"] = cpu
+        print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+def run_reference(args, world, rank, local):
+    """The CPU oracle on the same decode workload: each step is one whole
+    sequence's decode step (all heads), on all host cores."""
+    if world > 1:
+        init_dist(world, "gloo")
+        if rank != 0:
+            barrier(world)
+            return
+    from paper_2606_18587_gb300 import inputs as I
+    cfg = I.DECODE_160M
+    budget = max(1.0, args.cpu_budget / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        oracle_decode_sample(cfg, budget_s=0.0)
+    vals = []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        gbs, cores, sample = oracle_decode_sample(cfg, budget_s=budget)
+        vals.append(gbs)
+    wall = time.perf_counter() - t0
+    v = float(np.mean(vals))
+    line = {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * wall / args.steps, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded N(0,1) keys/values/queries)",
+            "config": {"workload": cfg.name, "B": cfg.B, "Hq": cfg.Hq, "Hkv": cfg.Hkv, "context": cfg.L,
+                       "w": cfg.w, "d": cfg.d, "d_down": cfg.dd, "step": "one decode step of a sample"},
+            "cpu_baseline": {"value": round(v, 4), "unit": "GB/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(v, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        barrier(world)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for the CPU baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    world, rank, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, world, rank, local)
+    else:
+        run_ours(args, world, rank, local)
+
+
+if __name__ == "__main__":
+    main()

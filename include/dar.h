@@ -1,0 +1,165 @@
+/*
+ * dar.h -- C ABI of the GB300 (sm_103a) kernels for Distance-Adaptive
+ * Representation (DAR) attention: causal attention in which the last w tokens
+ * (the current one included) keep full head-dimension keys and values and
+ * older tokens keep only d_down-dimensional bottleneck vectors that are lifted
+ * back to d ("Dual Dimensionality for Local and Global Attention", Sec. 2,
+ * Eq. 1-4, and the cache scheme of Sec. 5 "Compute and memory efficiency").
+ *
+ * Conventions shared by every entry point
+ *  - All tensor arguments are DEVICE pointers to caller-allocated, caller-owned,
+ *    contiguous row-major memory.  The library allocates nothing, frees nothing
+ *    and never synchronises: every call enqueues work on `stream` (a
+ *    cudaStream_t passed as void*; NULL = the legacy default stream) and returns.
+ *  - Storage type T is fp32 (DAR_F32) or bf16 (DAR_BF16) for queries, keys,
+ *    values, outputs and the cached vectors.  The projection matrices are
+ *    always fp32.  Arithmetic is fp32 on the device.
+ *  - Per KV head g the method uses four matrices (the per-head reading of
+ *    Eq. 1-2): Dk, Dv = W_down for keys / values, shape [Hkv][d][d_down], and
+ *    Uk, Uv = W_up for keys / values, shape [Hkv][d_down][d].  Passing the
+ *    same pointers for K and V gives one shared bottleneck.
+ *  - GQA: query head h reads KV head g = h / (Hq / Hkv).
+ *  - Supported shapes: d = 64; d_down in {8, 16, 32, 64}; Hq a multiple of Hkv.
+ *  - Arguments are checked on the host before any launch; a bad argument
+ *    returns an error code and launches nothing.  Conditions only the device
+ *    can see (a seq_len or block-table entry out of range) are written to the
+ *    caller's status word (first error wins) and the affected work is skipped;
+ *    the kernels never trap.  dar_last_error() describes the last non-OK
+ *    return on the calling thread.
+ *  - `scale` <= 0 selects the default 1/sqrt(d) of Eq. 4.
+ */
+#ifndef DAR_H
+#define DAR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DAR_OK = 0,
+    DAR_ERR_INVALID_ARG = 1, /* null pointer, negative size, inconsistent shape   */
+    DAR_ERR_UNSUPPORTED = 2, /* valid but not built (d != 64, d_down not listed)  */
+    DAR_ERR_CAPACITY = 3,    /* workspace too small / no page for a token         */
+    DAR_ERR_CUDA = 4         /* the CUDA runtime reported an error at launch      */
+} dar_status;
+
+typedef enum { DAR_F32 = 0, DAR_BF16 = 1 } dar_dtype;
+
+/* Tokens per page of the bottleneck pool. */
+#define DAR_PAGE_SIZE 64
+
+/*
+ * Mixed-dimension KV cache (Sec. 5, "Compute and memory efficiency": tokens
+ * beyond the window keep only their d_down vectors, so the cache costs
+ * O(T d_down + w d) instead of O(T d)).  Host struct holding device pointers.
+ *
+ *  win_k, win_v   [B][Hkv][w][d] T.  The token at position p of sequence b
+ *                 sits in ring slot p % w while L_b - 1 - p < w.
+ *  pool_kd,
+ *  pool_vd        [num_pages][Hkv][DAR_PAGE_SIZE][d_down] T.  The bottleneck
+ *                 vectors k^D = k Dk, v^D = v Dv (Eq. 1) of a token at position
+ *                 p that has left the window live in physical page
+ *                 block_table[b][p / 64], row p % 64.
+ *  block_table    [B][max_pages_per_seq] int32, caller-assigned; entries that
+ *                 are needed must lie in [0, num_pages).
+ *  seq_lens       [B] int32: tokens held per sequence.  dar_cache_append adds
+ *                 to it; the caller zero-fills it for an empty cache.
+ *  status         one int32 the kernels set to a dar_status on a device-side
+ *                 error (0 = no error); the caller clears it.
+ *
+ * Requires w >= 1 (the current token is always local, Eq. 3 with i - j = 0).
+ */
+typedef struct dar_cache {
+    dar_dtype dtype;
+    int32_t B, Hkv, d, d_down, w;
+    int32_t max_pages_per_seq;
+    int32_t num_pages;
+    void *win_k, *win_v;
+    void *pool_kd, *pool_vd;
+    int32_t *block_table;
+    int32_t *seq_lens;
+    int32_t *status;
+} dar_cache;
+
+/*
+ * Eq. 1, the bottleneck h^D = h W_down, per KV head:
+ *   out[b][g][j][c] = round_T( sum_t x[b][g][j][t] * W[g][t][c] )
+ * where the sum is ONE fp32 fused-multiply-add chain over t = 0..d-1 starting
+ * from +0.0f and the result is rounded once to T (nearest even).  The same
+ * chain is used by dar_cache_append and inside dar_attn_prefill, so a token's
+ * cached vector is bit-identical whichever call produced it.
+ *   x [B][Hkv][n][d] T, W [Hkv][d][d_down] fp32, out [B][Hkv][n][d_down] T.
+ */
+dar_status dar_down_project(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t n, int32_t d,
+                            int32_t d_down, const void *x, const float *W, void *out,
+                            void *stream);
+
+/*
+ * Append tokens to every sequence of the cache (inference, Sec. 2.3 and the
+ * cache scheme of Sec. 5).  k_new, v_new [B][Hkv][n][d] T; sequence b appends
+ * its first n_b tokens, n_b = n_per_seq[b] (a device int32[B] with
+ * 0 <= n_b <= n) or n_b = n when n_per_seq is NULL.  They take positions
+ * seq_lens[b] .. seq_lens[b]+n_b-1.  Every token that leaves the window (its
+ * distance from the new last token reaches w) is down-projected with Dk / Dv
+ * exactly as dar_down_project and written to its page; the others go to their
+ * ring slot.  seq_lens[b] += n_b.  A needed block-table entry outside
+ * [0, num_pages), or a length beyond max_pages_per_seq*64 + w, sets
+ * *status = DAR_ERR_CAPACITY (an n_b outside [0, n] sets
+ * DAR_ERR_INVALID_ARG) and skips that sequence.
+ */
+dar_status dar_cache_append(const dar_cache *cache, const void *k_new, const void *v_new,
+                            int32_t n, const int32_t *n_per_seq, const float *Dk,
+                            const float *Dv, void *stream);
+
+/*
+ * Bytes of workspace dar_attn_decode needs for this cache shape and Hq query
+ * heads.  The workspace must be zero-filled once before its first use (for
+ * example with cudaMemsetAsync); every completed call leaves it zero-filled
+ * again, so it can be reused without clearing.  Calls that share one
+ * workspace must not overlap on the device.
+ */
+size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq);
+
+/*
+ * One decode step (Eq. 3-4 for the query at position i = L_b - 1 of each
+ * sequence, L_b = seq_lens[b]): scores against the ring (full d) and the
+ * pages (d_down, with W_up absorbed into the query, q~ = q Uk^T), one softmax
+ * over both, values lifted once, o = (sum_local p v + (sum_global p v^D) Uv) / sum p.
+ *   q [B][Hq][d] T; Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][d] T.
+ * A sequence with L_b == 0 gets a zero output.  Split-K over the sequence with
+ * the partial results combined inside the same kernel.
+ */
+dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, const float *Uk,
+                           const float *Uv, float scale, void *out, void *workspace,
+                           size_t workspace_bytes, void *stream);
+
+/* Bytes of workspace dar_attn_prefill needs (the Eq. 1 vectors of all tokens). */
+size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t N,
+                                   int32_t d_down);
+
+/*
+ * Causal forward over positions 0..N-1 with no earlier context (the training
+ * forward of Sec. 2.3: every token keeps both representations and each query
+ * takes the one Eq. 3 selects).
+ *   q [B][Hq][N][d], k, v [B][Hkv][N][d] T; Dk, Dv [Hkv][d][d_down] fp32;
+ *   Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][N][d] T.
+ * w >= 0; w = 0 is the paper's uniform reduction (no token is local).
+ * The workspace (no initialisation needed) receives k^D, v^D.
+ */
+dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
+                            int32_t d, int32_t d_down, int32_t w, const void *q, const void *k,
+                            const void *v, const float *Dk, const float *Uk, const float *Dv,
+                            const float *Uv, float scale, void *out, void *workspace,
+                            size_t workspace_bytes, void *stream);
+
+/* Message for the last non-OK return on this thread ("" if none). */
+const char *dar_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DAR_H */

@@ -1,0 +1,297 @@
+// dar_abi.cu -- the extern "C" entry points declared in dar.h: argument
+// validation (nothing is launched on a bad argument), workspace layout and
+// dispatch to the kernels.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <string>
+
+#include "dar_common.cuh"
+#include "dar_launch.h"
+
+namespace {
+
+thread_local std::string g_err;
+
+dar_status fail(dar_status s, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return s;
+}
+
+dar_status ok()
+{
+    g_err.clear();
+    return DAR_OK;
+}
+
+dar_status from_cuda(cudaError_t e, const char *what)
+{
+    if (e == cudaSuccess)
+        return ok();
+    return fail(DAR_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool dd_supported(int dd) { return dd == 8 || dd == 16 || dd == 32 || dd == 64; }
+bool dtype_valid(int dt) { return dt == DAR_F32 || dt == DAR_BF16; }
+size_t esize(dar_dtype dt) { return dt == DAR_F32 ? 4 : 2; }
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+float default_scale(float scale, int d) { return scale > 0.f ? scale : 1.0f / sqrtf((float)d); }
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Common shape checks: returns DAR_OK or an error (message set).
+dar_status check_dims(int dt, int d, int dd)
+{
+    if (!dtype_valid(dt))
+        return fail(DAR_ERR_INVALID_ARG, "dtype %d is not DAR_F32 or DAR_BF16", dt);
+    if (d != dar::kHeadDim)
+        return fail(DAR_ERR_UNSUPPORTED, "head dimension d=%d (only d=64 is built)", d);
+    if (!dd_supported(dd))
+        return fail(DAR_ERR_UNSUPPORTED, "d_down=%d (built: 8, 16, 32, 64)", dd);
+    return DAR_OK;
+}
+
+dar_status check_cache(const dar_cache *c)
+{
+    if (!c)
+        return fail(DAR_ERR_INVALID_ARG, "cache is NULL");
+    dar_status s = check_dims(c->dtype, c->d, c->d_down);
+    if (s != DAR_OK)
+        return s;
+    if (c->B < 0 || c->Hkv < 1 || c->w < 1 || c->max_pages_per_seq < 0 || c->num_pages < 0)
+        return fail(DAR_ERR_INVALID_ARG,
+                    "cache shape B=%d Hkv=%d w=%d max_pages_per_seq=%d num_pages=%d (need B>=0, "
+                    "Hkv>=1, w>=1, page counts >=0)",
+                    c->B, c->Hkv, c->w, c->max_pages_per_seq, c->num_pages);
+    if (c->B > 4096)
+        return fail(DAR_ERR_UNSUPPORTED, "batch %d > 4096", c->B);
+    if (c->B == 0)
+        return DAR_OK;
+    if (!c->win_k || !c->win_v || !c->seq_lens || !c->status)
+        return fail(DAR_ERR_INVALID_ARG, "cache ring, seq_lens or status pointer is NULL");
+    if (c->max_pages_per_seq > 0 && (!c->block_table || !c->pool_kd || !c->pool_vd))
+        return fail(DAR_ERR_INVALID_ARG, "cache block_table or pool pointer is NULL");
+    if (c->max_pages_per_seq > 0 && c->num_pages < 1)
+        return fail(DAR_ERR_INVALID_ARG, "max_pages_per_seq=%d but num_pages=0", c->max_pages_per_seq);
+    if (!aligned16(c->win_k) || !aligned16(c->win_v) || !aligned16(c->pool_kd) ||
+        !aligned16(c->pool_vd))
+        return fail(DAR_ERR_INVALID_ARG, "cache buffers must be 16-byte aligned");
+    if ((double)c->B * c->Hkv * c->w * c->d > 9.0e18 ||
+        (double)c->num_pages * c->Hkv * DAR_PAGE_SIZE * c->d_down > 9.0e18)
+        return fail(DAR_ERR_INVALID_ARG, "cache too large");
+    return DAR_OK;
+}
+
+struct DecodeLayout {
+    size_t m, l, acc, counters, sched, total;
+};
+
+DecodeLayout decode_layout(const dar_cache *c, int Hq, const dar::DecodeGeometry &gm)
+{
+    DecodeLayout L;
+    const size_t recs = (size_t)c->B * Hq * gm.maxc;
+    L.m = 0;
+    L.l = L.m + align256(recs * sizeof(float));
+    L.acc = L.l + align256(recs * sizeof(float));
+    L.counters = L.acc + align256(recs * dar::kHeadDim * sizeof(float));
+    L.sched = L.counters + align256((size_t)c->B * c->Hkv * gm.HS * sizeof(int32_t));
+    L.total = L.sched + 256;
+    return L;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *dar_last_error(void) { return g_err.c_str(); }
+
+dar_status dar_down_project(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t n, int32_t d,
+                            int32_t d_down, const void *x, const float *W, void *out, void *stream)
+{
+    dar_status s = check_dims(dtype, d, d_down);
+    if (s != DAR_OK)
+        return s;
+    if (B < 0 || Hkv < 1 || n < 0)
+        return fail(DAR_ERR_INVALID_ARG, "B=%d Hkv=%d n=%d", B, Hkv, n);
+    if (B == 0 || n == 0)
+        return ok();
+    if (!x || !W || !out)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(x) || !aligned16(out) || !aligned16(W))
+        return fail(DAR_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
+    if ((long long)B * Hkv > 65535)
+        return fail(DAR_ERR_UNSUPPORTED, "B*Hkv=%lld > 65535", (long long)B * Hkv);
+    return from_cuda(dar::launch_down_project(dtype, d_down, x, W, out, B, Hkv, n,
+                                              static_cast<cudaStream_t>(stream)),
+                     "dar_down_project launch");
+}
+
+dar_status dar_cache_append(const dar_cache *cache, const void *k_new, const void *v_new,
+                            int32_t n, const int32_t *n_per_seq, const float *Dk,
+                            const float *Dv, void *stream)
+{
+    dar_status s = check_cache(cache);
+    if (s != DAR_OK)
+        return s;
+    if (n < 0)
+        return fail(DAR_ERR_INVALID_ARG, "n=%d", n);
+    if (cache->B == 0 || n == 0)
+        return ok();
+    if (!k_new || !v_new || !Dk || !Dv)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    dar::AppendArgs a;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.Dk = Dk;
+    a.Dv = Dv;
+    a.win_k = cache->win_k;
+    a.win_v = cache->win_v;
+    a.pool_kd = cache->pool_kd;
+    a.pool_vd = cache->pool_vd;
+    a.block_table = cache->block_table;
+    a.n_per_seq = n_per_seq;
+    a.seq_lens = cache->seq_lens;
+    a.status = cache->status;
+    a.B = cache->B;
+    a.Hkv = cache->Hkv;
+    a.n = n;
+    a.w = cache->w;
+    a.maxp = cache->max_pages_per_seq;
+    a.num_pages = cache->num_pages;
+    return from_cuda(dar::launch_cache_append(cache->dtype, cache->d_down, a,
+                                              static_cast<cudaStream_t>(stream)),
+                     "dar_cache_append launch");
+}
+
+size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq)
+{
+    if (check_cache(cache) != DAR_OK || Hq < cache->Hkv || Hq % cache->Hkv)
+        return 0;
+    dar::DecodeGeometry gm = dar::decode_geometry(cache->dtype, Hq, cache->Hkv, cache->d_down,
+                                                  cache->w, cache->max_pages_per_seq);
+    return decode_layout(cache, Hq, gm).total;
+}
+
+dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, const float *Uk,
+                           const float *Uv, float scale, void *out, void *workspace,
+                           size_t workspace_bytes, void *stream)
+{
+    dar_status s = check_cache(cache);
+    if (s != DAR_OK)
+        return s;
+    if (Hq < cache->Hkv || Hq % cache->Hkv)
+        return fail(DAR_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", Hq, cache->Hkv);
+    if (cache->B == 0)
+        return ok();
+    if (!q || !Uk || !Uv || !out || !workspace)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(Uk) || !aligned16(Uv) || !aligned16(workspace))
+        return fail(DAR_ERR_INVALID_ARG, "Uk, Uv and workspace must be 16-byte aligned");
+    dar::DecodeGeometry gm = dar::decode_geometry(cache->dtype, Hq, cache->Hkv, cache->d_down,
+                                                  cache->w, cache->max_pages_per_seq);
+    DecodeLayout L = decode_layout(cache, Hq, gm);
+    if (workspace_bytes < L.total)
+        return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
+    char *ws = static_cast<char *>(workspace);
+    dar::DecodeArgs a;
+    a.q = q;
+    a.out = out;
+    a.win_k = cache->win_k;
+    a.win_v = cache->win_v;
+    a.pool_kd = cache->pool_kd;
+    a.pool_vd = cache->pool_vd;
+    a.block_table = cache->block_table;
+    a.seq_lens = cache->seq_lens;
+    a.status = cache->status;
+    a.Uk = Uk;
+    a.Uv = Uv;
+    a.rec_m = reinterpret_cast<float *>(ws + L.m);
+    a.rec_l = reinterpret_cast<float *>(ws + L.l);
+    a.rec_acc = reinterpret_cast<float *>(ws + L.acc);
+    a.counters = reinterpret_cast<int32_t *>(ws + L.counters);
+    a.sched = reinterpret_cast<int32_t *>(ws + L.sched);
+    a.B = cache->B;
+    a.Hq = Hq;
+    a.Hkv = cache->Hkv;
+    a.G = Hq / cache->Hkv;
+    a.GH = gm.GH;
+    a.HS = gm.HS;
+    a.w = cache->w;
+    a.maxp = cache->max_pages_per_seq;
+    a.num_pages = cache->num_pages;
+    a.maxc = gm.maxc;
+    a.cw = gm.cw;
+    a.cd = gm.cd;
+    a.qscale = default_scale(scale, cache->d) * kLog2e;
+    return from_cuda(dar::launch_decode(cache->dtype, cache->d_down, a,
+                                        static_cast<cudaStream_t>(stream)),
+                     "dar_attn_decode launch");
+}
+
+size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t N,
+                                   int32_t d_down)
+{
+    if (!dtype_valid(dtype) || B < 0 || Hkv < 0 || N < 0 || d_down < 1)
+        return 0;
+    return 2 * align256((size_t)B * Hkv * N * d_down * esize(dtype));
+}
+
+dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
+                            int32_t d, int32_t d_down, int32_t w, const void *q, const void *k,
+                            const void *v, const float *Dk, const float *Uk, const float *Dv,
+                            const float *Uv, float scale, void *out, void *workspace,
+                            size_t workspace_bytes, void *stream)
+{
+    dar_status s = check_dims(dtype, d, d_down);
+    if (s != DAR_OK)
+        return s;
+    if (B < 0 || Hkv < 1 || Hq < Hkv || Hq % Hkv || N < 0 || w < 0)
+        return fail(DAR_ERR_INVALID_ARG, "B=%d Hq=%d Hkv=%d N=%d w=%d", B, Hq, Hkv, N, w);
+    if (B == 0 || N == 0)
+        return ok();
+    if ((long long)B * Hq > 65535 || (long long)B * Hkv > 65535)
+        return fail(DAR_ERR_UNSUPPORTED, "B*Hq=%lld > 65535", (long long)B * Hq);
+    if (!q || !k || !v || !Dk || !Uk || !Dv || !Uv || !out || !workspace)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) ||
+        !aligned16(workspace) || !aligned16(Dk) || !aligned16(Dv) || !aligned16(Uk) ||
+        !aligned16(Uv))
+        return fail(DAR_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
+    const size_t need = dar_prefill_workspace_bytes(dtype, B, Hkv, N, d_down);
+    if (workspace_bytes < need)
+        return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, need);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    char *kd = static_cast<char *>(workspace);
+    char *vd = kd + need / 2;
+    cudaError_t e = dar::launch_down_project(dtype, d_down, k, Dk, kd, B, Hkv, N, st);
+    if (e == cudaSuccess)
+        e = dar::launch_down_project(dtype, d_down, v, Dv, vd, B, Hkv, N, st);
+    if (e != cudaSuccess)
+        return from_cuda(e, "dar_attn_prefill down-projection launch");
+    dar::PrefillArgs a;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.kd = kd;
+    a.vd = vd;
+    a.Uk = Uk;
+    a.Uv = Uv;
+    a.out = out;
+    a.B = B;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.N = N;
+    a.w = w;
+    a.qscale = default_scale(scale, d) * kLog2e;
+    return from_cuda(dar::launch_prefill_simt(dtype, d_down, a, st), "dar_attn_prefill launch");
+}
+
+}  // extern "C"

@@ -1,0 +1,62 @@
+// dar_launch.h -- internal launchers behind the C ABI (host side).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "dar.h"
+
+namespace dar {
+
+struct AppendArgs {
+    const void *k_new, *v_new;  // [B][Hkv][n][64]
+    const float *Dk, *Dv;       // [Hkv][64][dd]
+    void *win_k, *win_v;        // [B][Hkv][w][64]
+    void *pool_kd, *pool_vd;    // [num_pages][Hkv][64][dd]
+    const int32_t *block_table; // [B][maxp]
+    const int32_t *n_per_seq;   // [B] or nullptr (every sequence appends n)
+    int32_t *seq_lens;
+    int32_t *status;
+    int B, Hkv, n, w, maxp, num_pages;
+};
+
+struct DecodeArgs {
+    const void *q;  // [B][Hq][64]
+    void *out;      // [B][Hq][64]
+    const void *win_k, *win_v;
+    const void *pool_kd, *pool_vd;
+    const int32_t *block_table;
+    const int32_t *seq_lens;
+    int32_t *status;
+    const float *Uk, *Uv;  // [Hkv][dd][64]
+    float *rec_m, *rec_l, *rec_acc;  // split-K partial results
+    int32_t *counters;               // per (b, g, head slice) arrival counts
+    int32_t *sched;                  // [2] dynamic item counter, exited-warp counter
+    int B, Hq, Hkv, G, GH, HS, w, maxp, num_pages, maxc, cw, cd;
+    float qscale;  // scale * log2(e)
+};
+
+struct PrefillArgs {
+    const void *q, *k, *v;  // [B][Hq|Hkv][N][64]
+    const void *kd, *vd;    // [B][Hkv][N][dd]   (Eq. 1 output)
+    const float *Uk, *Uv;   // [Hkv][dd][64]
+    void *out;              // [B][Hq][N][64]
+    int B, Hq, Hkv, N, w;
+    float qscale;  // scale * log2(e)
+};
+
+// Each launcher returns cudaSuccess or the launch error.
+cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float *W, void *out,
+                                int B, int Hkv, int n, cudaStream_t s);
+cudaError_t launch_cache_append(dar_dtype dt, int dd, const AppendArgs &a, cudaStream_t s);
+cudaError_t launch_decode(dar_dtype dt, int dd, const DecodeArgs &a, cudaStream_t s);
+cudaError_t launch_prefill_simt(dar_dtype dt, int dd, const PrefillArgs &a, cudaStream_t s);
+
+// Split-K geometry of the decode kernel (shared by workspace sizing and launch).
+struct DecodeGeometry {
+    int cw, cd, maxc, GH, HS;
+};
+DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int maxp);
+
+}  // namespace dar

@@ -1,0 +1,242 @@
+"""Python binding of the DAR CUDA library (``include/dar.h``).
+
+Argument marshalling only: every function passes device pointers, sizes and
+the current CUDA stream straight to the C entry point of the same name; all
+arithmetic runs in the sm_103a kernels.  PyTorch supplies device memory and
+streams.  There is no fallback: if ``libdar_gb300.so`` is missing or a call
+fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdar_gb300.so")
+HEADER = os.path.join(os.path.dirname(_HERE), "include", "dar.h")
+
+DAR_OK, DAR_ERR_INVALID_ARG, DAR_ERR_UNSUPPORTED, DAR_ERR_CAPACITY, DAR_ERR_CUDA = range(5)
+DAR_F32, DAR_BF16 = 0, 1
+PAGE_SIZE = 64
+_TORCH_DTYPE = {DAR_F32: torch.float32, DAR_BF16: torch.bfloat16}
+_CODE = {torch.float32: DAR_F32, torch.bfloat16: DAR_BF16}
+
+
+class DarError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"DAR error {code}: {msg}")
+        self.code = code
+
+
+class dar_cache(ctypes.Structure):
+    _fields_ = [
+        ("dtype", ctypes.c_int),
+        ("B", ctypes.c_int32), ("Hkv", ctypes.c_int32), ("d", ctypes.c_int32),
+        ("d_down", ctypes.c_int32), ("w", ctypes.c_int32),
+        ("max_pages_per_seq", ctypes.c_int32), ("num_pages", ctypes.c_int32),
+        ("win_k", ctypes.c_void_p), ("win_v", ctypes.c_void_p),
+        ("pool_kd", ctypes.c_void_p), ("pool_vd", ctypes.c_void_p),
+        ("block_table", ctypes.c_void_p), ("seq_lens", ctypes.c_void_p), ("status", ctypes.c_void_p),
+    ]
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH):
+    """Load the compiled library (raises if it was not built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"DAR CUDA library not found at {path}; build it with "
+                           "`python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(path)
+    P, I32, SZ, F = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t, ctypes.c_float
+    CP = ctypes.POINTER(dar_cache)
+    sig = {
+        "dar_down_project": ([ctypes.c_int, I32, I32, I32, I32, I32, P, P, P, P], ctypes.c_int),
+        "dar_cache_append": ([CP, P, P, I32, P, P, P, P], ctypes.c_int),
+        "dar_decode_workspace_bytes": ([CP, I32], SZ),
+        "dar_attn_decode": ([CP, I32, P, P, P, F, P, P, SZ, P], ctypes.c_int),
+        "dar_prefill_workspace_bytes": ([ctypes.c_int, I32, I32, I32, I32], SZ),
+        "dar_attn_prefill": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, P, P,
+                              SZ, P], ctypes.c_int),
+        "dar_last_error": ([], ctypes.c_char_p),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    _lib = lib
+    return lib
+
+
+def declared_symbols(header: str = HEADER):
+    """Names of the functions include/dar.h declares."""
+    text = open(header).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\s\*]*?\b(dar_\w+)\s*\(", text, re.M)))
+
+
+def dar_last_error() -> str:
+    return load_library().dar_last_error().decode()
+
+
+def _check(code):
+    if code != DAR_OK:
+        raise DarError(code, dar_last_error())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+
+
+def _dev(t, name, dtype=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    return t
+
+
+def _code(t):
+    if t.dtype not in _CODE:
+        raise ValueError(f"unsupported dtype {t.dtype}")
+    return _CODE[t.dtype]
+
+
+# --------------------------------------------------------------------------- Eq. 1
+
+def dar_down_project(x, W, out=None, stream=None):
+    """Eq. 1 per KV head: ``x [B,Hkv,n,d]`` (T) times ``W [Hkv,d,dd]`` (fp32) -> ``[B,Hkv,n,dd]`` (T)."""
+    _dev(x, "x")
+    _dev(W, "W", torch.float32)
+    B, Hkv, n, d = x.shape
+    dd = W.shape[2]
+    if out is None:
+        out = torch.empty((B, Hkv, n, dd), dtype=x.dtype, device=x.device)
+    _dev(out, "out", x.dtype)
+    _check(load_library().dar_down_project(_code(x), B, Hkv, n, d, dd, _ptr(x), _ptr(W), _ptr(out),
+                                           _stream(stream)))
+    return out
+
+
+# --------------------------------------------------------------------------- cache
+
+class DarCache:
+    """Caller-owned mixed-dimension cache (device tensors) and its ``dar_cache`` struct.
+
+    ``block_table`` (int32 ``[B, max_pages_per_seq]``) maps each sequence's
+    logical pages to physical pages of the pools; by default sequence b owns
+    pages ``b*max_pages_per_seq ..`` in order."""
+
+    def __init__(self, B, Hkv, d_down, w, max_pages_per_seq, num_pages=None, dtype=torch.bfloat16,
+                 block_table=None, device="cuda", d=64):
+        self.dtype = dtype
+        self.B, self.Hkv, self.d, self.d_down, self.w = B, Hkv, d, d_down, w
+        self.max_pages_per_seq = max_pages_per_seq
+        if num_pages is None:
+            num_pages = B * max_pages_per_seq
+        self.num_pages = num_pages
+        self.win_k = torch.zeros((B, Hkv, w, d), dtype=dtype, device=device)
+        self.win_v = torch.zeros_like(self.win_k)
+        self.pool_kd = torch.zeros((max(num_pages, 1), Hkv, PAGE_SIZE, d_down), dtype=dtype, device=device)
+        self.pool_vd = torch.zeros_like(self.pool_kd)
+        if block_table is None:
+            block_table = torch.arange(B * max_pages_per_seq, dtype=torch.int32).reshape(B, max_pages_per_seq)
+        self.block_table = torch.as_tensor(block_table, dtype=torch.int32).to(device).contiguous()
+        if self.block_table.numel() == 0:
+            self.block_table = torch.full((max(B, 1), 1), -1, dtype=torch.int32, device=device)
+        self.seq_lens = torch.zeros(B, dtype=torch.int32, device=device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
+        self._struct = dar_cache(
+            _CODE[dtype], B, Hkv, d, d_down, w, max_pages_per_seq, num_pages,
+            self.win_k.data_ptr(), self.win_v.data_ptr(), self.pool_kd.data_ptr(), self.pool_vd.data_ptr(),
+            self.block_table.data_ptr(), self.seq_lens.data_ptr(), self.status.data_ptr())
+
+    @property
+    def struct(self):
+        return ctypes.byref(self._struct)
+
+    def device_status(self) -> int:
+        return int(self.status.item())
+
+
+def dar_cache_append(cache: DarCache, k_new, v_new, Dk, Dv, n_per_seq=None, stream=None):
+    """Append ``k_new, v_new [B,Hkv,n,d]`` (first ``n_per_seq[b]`` rows of sequence b)."""
+    _dev(k_new, "k_new", cache.dtype)
+    _dev(v_new, "v_new", cache.dtype)
+    _dev(Dk, "Dk", torch.float32)
+    _dev(Dv, "Dv", torch.float32)
+    if n_per_seq is not None:
+        _dev(n_per_seq, "n_per_seq", torch.int32)
+    n = k_new.shape[2]
+    _check(load_library().dar_cache_append(cache.struct, _ptr(k_new), _ptr(v_new), n, _ptr(n_per_seq),
+                                           _ptr(Dk), _ptr(Dv), _stream(stream)))
+
+
+def dar_decode_workspace_bytes(cache: DarCache, Hq: int) -> int:
+    return int(load_library().dar_decode_workspace_bytes(cache.struct, Hq))
+
+
+def decode_workspace(cache: DarCache, Hq: int):
+    """A zero-filled workspace of the size dar_attn_decode needs."""
+    nbytes = dar_decode_workspace_bytes(cache, Hq)
+    if nbytes == 0:
+        raise DarError(DAR_ERR_INVALID_ARG, dar_last_error() or "bad cache/Hq")
+    return torch.zeros(nbytes, dtype=torch.uint8, device=cache.win_k.device)
+
+
+def dar_attn_decode(cache: DarCache, q, Uk, Uv, workspace, scale=0.0, out=None, stream=None):
+    """One decode step for queries ``q [B,Hq,d]`` at the last position of each sequence."""
+    _dev(q, "q", cache.dtype)
+    _dev(Uk, "Uk", torch.float32)
+    _dev(Uv, "Uv", torch.float32)
+    _dev(workspace, "workspace")
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", cache.dtype)
+    Hq = q.shape[1]
+    _check(load_library().dar_attn_decode(cache.struct, Hq, _ptr(q), _ptr(Uk), _ptr(Uv), float(scale),
+                                          _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                          _stream(stream)))
+    return out
+
+
+# --------------------------------------------------------------------------- prefill
+
+def dar_prefill_workspace_bytes(dtype, B, Hkv, N, d_down) -> int:
+    return int(load_library().dar_prefill_workspace_bytes(_CODE[dtype], B, Hkv, N, d_down))
+
+
+def dar_attn_prefill(q, k, v, Dk, Uk, Dv, Uv, w, scale=0.0, out=None, workspace=None, stream=None):
+    """Causal forward: ``q [B,Hq,N,d]``, ``k, v [B,Hkv,N,d]`` -> ``[B,Hq,N,d]``."""
+    _dev(q, "q")
+    _dev(k, "k", q.dtype)
+    _dev(v, "v", q.dtype)
+    for name, t in (("Dk", Dk), ("Uk", Uk), ("Dv", Dv), ("Uv", Uv)):
+        _dev(t, name, torch.float32)
+    B, Hq, N, d = q.shape
+    Hkv = k.shape[1]
+    dd = Dk.shape[2]
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", q.dtype)
+    if workspace is None:
+        workspace = torch.empty(max(1, dar_prefill_workspace_bytes(q.dtype, B, Hkv, N, dd)),
+                                dtype=torch.uint8, device=q.device)
+    _dev(workspace, "workspace")
+    _check(load_library().dar_attn_prefill(
+        _code(q), B, Hq, Hkv, N, d, dd, int(w), _ptr(q), _ptr(k), _ptr(v), _ptr(Dk), _ptr(Uk), _ptr(Dv), _ptr(Uv),
+        float(scale), _ptr(out), _ptr(workspace), workspace.numel(), _stream(stream)))
+    return out

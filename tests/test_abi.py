@@ -1,0 +1,94 @@
+"""C-ABI checks that need no GPU: the library builds for sm_103a, loads,
+exports every function include/dar.h declares, and rejects bad arguments on
+the host (error code, message, nothing launched)."""
+import ctypes
+import os
+import shutil
+
+import pytest
+
+pytest.importorskip("torch")
+
+from paper_2606_18587_gb300 import build as lib_build  # noqa: E402
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(lib_build.LIB) and shutil.which("nvcc") is None and \
+            not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("no nvcc to build the library")
+    lib_build.build()
+    from paper_2606_18587_gb300 import dar
+    return dar
+
+
+def test_exports_every_declared_symbol(lib):
+    names = lib.declared_symbols()
+    assert {"dar_attn_prefill", "dar_attn_decode", "dar_cache_append", "dar_down_project",
+            "dar_decode_workspace_bytes", "dar_prefill_workspace_bytes", "dar_last_error"} <= set(names)
+    raw = ctypes.CDLL(lib.LIB_PATH)
+    for n in names:
+        assert hasattr(raw, n), f"{n} declared in dar.h but not exported"
+
+
+def _cache(lib, **kw):
+    c = dict(dtype=lib.DAR_BF16, B=2, Hkv=2, d=64, d_down=16, w=8, max_pages_per_seq=4, num_pages=8,
+             win_k=256, win_v=512, pool_kd=768, pool_vd=1024, block_table=1280, seq_lens=1536, status=1792)
+    c.update(kw)
+    return lib.dar_cache(*[c[f] for f, _ in lib.dar_cache._fields_])
+
+
+def test_workspace_sizes_are_host_only(lib):
+    L = lib.load_library()
+    c = _cache(lib)
+    n = L.dar_decode_workspace_bytes(ctypes.byref(c), 4)
+    assert n > 0 and n % 256 == 0
+    assert L.dar_decode_workspace_bytes(ctypes.byref(c), 3) == 0      # Hq not a multiple of Hkv
+    assert L.dar_decode_workspace_bytes(ctypes.byref(_cache(lib, d=32)), 4) == 0
+    assert L.dar_prefill_workspace_bytes(lib.DAR_BF16, 2, 3, 100, 16) == 2 * 19200  # K and V, 2*3*100*16*2 B each
+    assert L.dar_prefill_workspace_bytes(lib.DAR_BF16, 1, 1, 3, 8) == 2 * 256  # 48 B rounded up to 256
+    assert L.dar_prefill_workspace_bytes(lib.DAR_F32, 0, 3, 100, 16) == 0
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(d=32), 2), (dict(d_down=12), 2), (dict(w=0), 1), (dict(Hkv=0), 1), (dict(dtype=7), 1),
+    (dict(win_k=0), 1), (dict(win_k=258), 1), (dict(B=5000), 2),
+])
+def test_decode_rejects_bad_cache(lib, kw, code):
+    L = lib.load_library()
+    c = _cache(lib, **kw)
+    r = L.dar_attn_decode(ctypes.byref(c), 4, 256, 256, 256, 0.0, 256, 256, 1 << 30, None)
+    assert r == code
+    assert L.dar_last_error().decode()
+
+
+def test_prefill_rejects_bad_arguments(lib):
+    L = lib.load_library()
+    P = 4096
+    args = lambda **kw: dict(dict(dtype=lib.DAR_BF16, B=1, Hq=4, Hkv=2, N=16, d=64, dd=16, w=4, q=P, k=P, v=P,  # noqa
+                                   Dk=P, Uk=P, Dv=P, Uv=P, scale=0.0, out=P, ws=P, wsb=1 << 20, s=None), **kw)
+
+    def call(**kw):
+        a = args(**kw)
+        return L.dar_attn_prefill(a["dtype"], a["B"], a["Hq"], a["Hkv"], a["N"], a["d"], a["dd"], a["w"],
+                                  a["q"], a["k"], a["v"], a["Dk"], a["Uk"], a["Dv"], a["Uv"], a["scale"],
+                                  a["out"], a["ws"], a["wsb"], a["s"])
+    assert call(Hq=3) == 1
+    assert call(w=-1) == 1
+    assert call(d=128) == 2
+    assert call(dd=24) == 2
+    assert call(q=0) == 1
+    assert call(k=P + 2) == 1
+    assert call(wsb=16) == 3
+    assert "workspace" in L.dar_last_error().decode()
+    assert call(N=0) == 0          # empty problem: nothing to do
+    assert L.dar_last_error().decode() == ""
+
+
+def test_append_rejects_bad_arguments(lib):
+    L = lib.load_library()
+    c = _cache(lib)
+    assert L.dar_cache_append(ctypes.byref(c), 256, 256, -1, None, 256, 256, None) == 1
+    assert L.dar_cache_append(ctypes.byref(c), 0, 256, 4, None, 256, 256, None) == 1
+    assert L.dar_cache_append(ctypes.byref(_cache(lib, w=0)), 256, 256, 4, None, 256, 256, None) == 1
+    assert L.dar_cache_append(ctypes.byref(c), 256, 256, 0, None, 256, 256, None) == 0
