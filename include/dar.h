@@ -51,6 +51,10 @@ typedef enum { DAR_F32 = 0, DAR_BF16 = 1 } dar_dtype;
 /* Tokens per page of the bottleneck pool. */
 #define DAR_PAGE_SIZE 64
 
+/* Largest batch dar_attn_decode accepts (its per-sequence tables live in
+ * shared memory). */
+#define DAR_DECODE_MAX_BATCH 1024
+
 /*
  * Mixed-dimension KV cache (Sec. 5, "Compute and memory efficiency": tokens
  * beyond the window keep only their d_down vectors, so the cache costs
@@ -130,7 +134,8 @@ size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq);
  * over both, values lifted once, o = (sum_local p v + (sum_global p v^D) Uv) / sum p.
  *   q [B][Hq][d] T; Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][d] T.
  * A sequence with L_b == 0 gets a zero output.  Split-K over the sequence with
- * the partial results combined inside the same kernel.
+ * the partial results combined inside the same kernel.  B <= DAR_DECODE_MAX_BATCH.
+ * After a call that set *status, zero-fill the workspace again before reuse.
  */
 dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, const float *Uk,
                            const float *Uv, float scale, void *out, void *workspace,
@@ -147,13 +152,16 @@ size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int3
  *   q [B][Hq][N][d], k, v [B][Hkv][N][d] T; Dk, Dv [Hkv][d][d_down] fp32;
  *   Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][N][d] T.
  * w >= 0; w = 0 is the paper's uniform reduction (no token is local).
- * The workspace (no initialisation needed) receives k^D, v^D.
+ * The workspace (no initialisation needed) receives k^D, v^D.  `status` (a
+ * device int32, may be NULL) is set to a dar_status if a kernel gives up on a
+ * bounded internal wait; the caller clears it.  bf16 runs on the tcgen05
+ * tensor cores, fp32 on the CUDA cores (fp32 FMA, no TF32).
  */
 dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
                             int32_t d, int32_t d_down, int32_t w, const void *q, const void *k,
                             const void *v, const float *Dk, const float *Uk, const float *Dv,
                             const float *Uv, float scale, void *out, void *workspace,
-                            size_t workspace_bytes, void *stream);
+                            size_t workspace_bytes, int32_t *status, void *stream);
 
 /* Message for the last non-OK return on this thread ("" if none). */
 const char *dar_last_error(void);

@@ -129,7 +129,7 @@ dar_status dar_down_project(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t n, 
         return fail(DAR_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
     if ((long long)B * Hkv > 65535)
         return fail(DAR_ERR_UNSUPPORTED, "B*Hkv=%lld > 65535", (long long)B * Hkv);
-    return from_cuda(dar::launch_down_project(dtype, d_down, x, W, out, B, Hkv, n,
+    return from_cuda(dar::launch_down_project(dtype, d_down, x, W, out, B, Hkv, n, d_down,
                                               static_cast<cudaStream_t>(stream)),
                      "dar_down_project launch");
 }
@@ -147,6 +147,8 @@ dar_status dar_cache_append(const dar_cache *cache, const void *k_new, const voi
         return ok();
     if (!k_new || !v_new || !Dk || !Dv)
         return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(Dk) || !aligned16(Dv))
+        return fail(DAR_ERR_INVALID_ARG, "k_new, v_new, Dk and Dv must be 16-byte aligned");
     dar::AppendArgs a;
     a.k_new = k_new;
     a.v_new = v_new;
@@ -189,6 +191,8 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
         return s;
     if (Hq < cache->Hkv || Hq % cache->Hkv)
         return fail(DAR_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", Hq, cache->Hkv);
+    if (cache->B > DAR_DECODE_MAX_BATCH)
+        return fail(DAR_ERR_UNSUPPORTED, "decode batch %d > %d", cache->B, DAR_DECODE_MAX_BATCH);
     if (cache->B == 0)
         return ok();
     if (!q || !Uk || !Uv || !out || !workspace)
@@ -241,14 +245,15 @@ size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int3
 {
     if (!dtype_valid(dtype) || B < 0 || Hkv < 0 || N < 0 || d_down < 1)
         return 0;
-    return 2 * align256((size_t)B * Hkv * N * d_down * esize(dtype));
+    const int stride = dar::prefill_kd_stride(dtype, d_down);
+    return 2 * align256((size_t)B * Hkv * N * stride * esize(dtype));
 }
 
 dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
                             int32_t d, int32_t d_down, int32_t w, const void *q, const void *k,
                             const void *v, const float *Dk, const float *Uk, const float *Dv,
                             const float *Uv, float scale, void *out, void *workspace,
-                            size_t workspace_bytes, void *stream)
+                            size_t workspace_bytes, int32_t *status, void *stream)
 {
     dar_status s = check_dims(dtype, d, d_down);
     if (s != DAR_OK)
@@ -271,9 +276,10 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     char *kd = static_cast<char *>(workspace);
     char *vd = kd + need / 2;
-    cudaError_t e = dar::launch_down_project(dtype, d_down, k, Dk, kd, B, Hkv, N, st);
+    const int kstride = dar::prefill_kd_stride(dtype, d_down);
+    cudaError_t e = dar::launch_down_project(dtype, d_down, k, Dk, kd, B, Hkv, N, kstride, st);
     if (e == cudaSuccess)
-        e = dar::launch_down_project(dtype, d_down, v, Dv, vd, B, Hkv, N, st);
+        e = dar::launch_down_project(dtype, d_down, v, Dv, vd, B, Hkv, N, kstride, st);
     if (e != cudaSuccess)
         return from_cuda(e, "dar_attn_prefill down-projection launch");
     dar::PrefillArgs a;
@@ -285,12 +291,17 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
     a.Uk = Uk;
     a.Uv = Uv;
     a.out = out;
+    a.status = status;
     a.B = B;
     a.Hq = Hq;
     a.Hkv = Hkv;
     a.N = N;
     a.w = w;
+    a.dd = d_down;
+    a.kd_stride = kstride;
     a.qscale = default_scale(scale, d) * kLog2e;
+    if (dtype == DAR_BF16)
+        return from_cuda(dar::launch_prefill_tc(d_down, a, st), "dar_attn_prefill (tcgen05) launch");
     return from_cuda(dar::launch_prefill_simt(dtype, d_down, a, st), "dar_attn_prefill launch");
 }
 

@@ -14,7 +14,8 @@ namespace dar {
 template <typename T, int DD>
 __global__ void __launch_bounds__(128) down_project_kernel(const T *__restrict__ x,
                                                            const float *__restrict__ W,
-                                                           T *__restrict__ out, int Hkv, int n)
+                                                           T *__restrict__ out, int Hkv, int n,
+                                                           int ostride)
 {
     __shared__ float Ws[kHeadDim * DD];
     const int bg = blockIdx.y;
@@ -47,38 +48,59 @@ __global__ void __launch_bounds__(128) down_project_kernel(const T *__restrict__
 #pragma unroll
         for (int c = 0; c < DD; ++c)
             acc[c] = __fmaf_rn(xv[t], Ws[t * DD + c], acc[c]);
-    T *o = out + ((size_t)bg * n + j) * DD;
+    T *o = out + ((size_t)bg * n + j) * ostride;
 #pragma unroll
     for (int c = 0; c < DD; ++c)
         o[c] = from_f32<T>(acc[c]);
+    for (int c = DD; c < ostride; ++c)
+        o[c] = from_f32<T>(0.f);
 }
 
 // ------------------------------------------------------------ cache append
 
-// Eq. 1 for one row, computed by a warp: lane c (and c + 32) owns output c.
+// Eq. 1 for one row, computed by a warp: lane j holds x[2j], x[2j+1] and lane
+// c (and c + 32) runs the fixed-order chain for output c, reading x[t] by
+// shuffle and its column of W from registers loaded in one batch.
 template <typename T, int DD>
 __device__ __forceinline__ void project_row_warp(const T *x, const float *W, T *out, int lane)
 {
     constexpr int CPL = (DD + 31) / 32;
+    const float x0 = to_f32(x[2 * lane]), x1 = to_f32(x[2 * lane + 1]);
+    float wcol[CPL][kHeadDim];
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) {
+        const int c = lane + 32 * i;
+#pragma unroll
+        for (int t = 0; t < kHeadDim; ++t)
+            wcol[i][t] = c < DD ? __ldg(W + t * DD + c) : 0.f;
+    }
     float acc[CPL];
 #pragma unroll
     for (int i = 0; i < CPL; ++i)
         acc[i] = 0.0f;
-#pragma unroll 8
-    for (int t = 0; t < kHeadDim; ++t) {
-        const float xv = to_f32(x[t]);
 #pragma unroll
-        for (int i = 0; i < CPL; ++i) {
-            const int c = lane + 32 * i;
-            if (c < DD)
-                acc[i] = __fmaf_rn(xv, W[t * DD + c], acc[i]);
-        }
+    for (int t = 0; t < kHeadDim; ++t) {
+        const float xt = __shfl_sync(0xffffffffu, (t & 1) ? x1 : x0, t >> 1);
+#pragma unroll
+        for (int i = 0; i < CPL; ++i)
+            acc[i] = __fmaf_rn(xt, wcol[i][t], acc[i]);
     }
 #pragma unroll
     for (int i = 0; i < CPL; ++i) {
         const int c = lane + 32 * i;
         if (c < DD)
             out[c] = from_f32<T>(acc[i]);
+    }
+}
+
+// Copy one 64-element row with the warp (2 elements per lane).
+template <typename T>
+__device__ __forceinline__ void copy_row_warp(const T *src, T *dst, int lane)
+{
+    if constexpr (sizeof(T) == 2) {
+        reinterpret_cast<uint32_t *>(dst)[lane] = reinterpret_cast<const uint32_t *>(src)[lane];
+    } else {
+        reinterpret_cast<uint2 *>(dst)[lane] = reinterpret_cast<const uint2 *>(src)[lane];
     }
 }
 
@@ -97,13 +119,13 @@ __device__ __forceinline__ T *pool_row(const AppendArgs &a, T *pool, int b, int 
 }
 
 // grid B (one CTA per sequence, so its length can be updated at the end),
-// 256 threads.  Sequence b appends nb = n_per_seq[b] (or n) tokens; k_new
+// up to 1024 threads.  Sequence b appends nb = n_per_seq[b] (or n) tokens; k_new
 // rows are strided by n.  Work unit = (KV head g, slot touched by this call): the slot's
 // old occupant migrates to its page, then the new positions of that slot are
 // processed in order (all but the last migrate straight from k_new; the last
 // is written into the ring).
 template <typename T, int DD>
-__global__ void __launch_bounds__(256) cache_append_kernel(AppendArgs a)
+__global__ void __launch_bounds__(1024) cache_append_kernel(AppendArgs a)
 {
     const int b = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -163,10 +185,8 @@ __global__ void __launch_bounds__(256) cache_append_kernel(AppendArgs a)
                 if (rv)
                     project_row_warp<T, DD>(vnew + src, Dv, rv, lane);
             } else {
-                wk[ring + lane] = knew[src + lane];
-                wk[ring + lane + 32] = knew[src + lane + 32];
-                wv[ring + lane] = vnew[src + lane];
-                wv[ring + lane + 32] = vnew[src + lane + 32];
+                copy_row_warp(knew + src, wk + ring, lane);
+                copy_row_warp(vnew + src, wv + ring, lane);
             }
             __syncwarp();
         }
@@ -180,38 +200,41 @@ __global__ void __launch_bounds__(256) cache_append_kernel(AppendArgs a)
 
 template <typename T>
 static cudaError_t down_project_t(int dd, const void *x, const float *W, void *out, int B,
-                                  int Hkv, int n, cudaStream_t s)
+                                  int Hkv, int n, int os, cudaStream_t s)
 {
     dim3 grid((n + 127) / 128, B * Hkv);
     const T *xi = static_cast<const T *>(x);
     T *o = static_cast<T *>(out);
     switch (dd) {
-    case 8: down_project_kernel<T, 8><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n); break;
-    case 16: down_project_kernel<T, 16><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n); break;
-    case 32: down_project_kernel<T, 32><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n); break;
-    case 64: down_project_kernel<T, 64><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n); break;
+    case 8: down_project_kernel<T, 8><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
+    case 16: down_project_kernel<T, 16><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
+    case 32: down_project_kernel<T, 32><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
+    case 64: down_project_kernel<T, 64><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
     default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();
 }
 
 cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float *W, void *out,
-                                int B, int Hkv, int n, cudaStream_t s)
+                                int B, int Hkv, int n, int ostride, cudaStream_t s)
 {
     if (n == 0 || B == 0)
         return cudaSuccess;
-    return dt == DAR_F32 ? down_project_t<float>(dd, x, W, out, B, Hkv, n, s)
-                         : down_project_t<bf16>(dd, x, W, out, B, Hkv, n, s);
+    return dt == DAR_F32 ? down_project_t<float>(dd, x, W, out, B, Hkv, n, ostride, s)
+                         : down_project_t<bf16>(dd, x, W, out, B, Hkv, n, ostride, s);
 }
 
 template <typename T>
 static cudaError_t cache_append_t(int dd, const AppendArgs &a, cudaStream_t s)
 {
+    // one warp per (KV head, touched slot) unit, up to 32 warps per sequence
+    const long long units = (long long)a.Hkv * (a.n < a.w ? a.n : a.w);
+    const int threads = 32 * (int)(units < 1 ? 1 : units > 32 ? 32 : units);
     switch (dd) {
-    case 8: cache_append_kernel<T, 8><<<a.B, 256, 0, s>>>(a); break;
-    case 16: cache_append_kernel<T, 16><<<a.B, 256, 0, s>>>(a); break;
-    case 32: cache_append_kernel<T, 32><<<a.B, 256, 0, s>>>(a); break;
-    case 64: cache_append_kernel<T, 64><<<a.B, 256, 0, s>>>(a); break;
+    case 8: cache_append_kernel<T, 8><<<a.B, threads, 0, s>>>(a); break;
+    case 16: cache_append_kernel<T, 16><<<a.B, threads, 0, s>>>(a); break;
+    case 32: cache_append_kernel<T, 32><<<a.B, threads, 0, s>>>(a); break;
+    case 64: cache_append_kernel<T, 64><<<a.B, threads, 0, s>>>(a); break;
     default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();

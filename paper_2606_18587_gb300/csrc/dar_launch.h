@@ -39,19 +39,26 @@ struct DecodeArgs {
 
 struct PrefillArgs {
     const void *q, *k, *v;  // [B][Hq|Hkv][N][64]
-    const void *kd, *vd;    // [B][Hkv][N][dd]   (Eq. 1 output)
+    const void *kd, *vd;    // [B][Hkv][N][kd_stride]   (Eq. 1 output, zero padded)
     const float *Uk, *Uv;   // [Hkv][dd][64]
     void *out;              // [B][Hq][N][64]
-    int B, Hq, Hkv, N, w;
+    int32_t *status;        // device error word or nullptr
+    int B, Hq, Hkv, N, w, dd, kd_stride;
     float qscale;  // scale * log2(e)
 };
 
+// Row stride (elements) of the prefill bottleneck workspace: the tensor-core
+// path needs rows of at least 16 bf16 (one MMA K step).
+inline int prefill_kd_stride(dar_dtype dt, int dd) { return (dt == DAR_BF16 && dd < 16) ? 16 : dd; }
+
 // Each launcher returns cudaSuccess or the launch error.
+// Eq. 1 into rows of `ostride` elements (entries dd..ostride-1 are zeroed).
 cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float *W, void *out,
-                                int B, int Hkv, int n, cudaStream_t s);
+                                int B, int Hkv, int n, int ostride, cudaStream_t s);
 cudaError_t launch_cache_append(dar_dtype dt, int dd, const AppendArgs &a, cudaStream_t s);
 cudaError_t launch_decode(dar_dtype dt, int dd, const DecodeArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_simt(dar_dtype dt, int dd, const PrefillArgs &a, cudaStream_t s);
+cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s);
 
 // Split-K geometry of the decode kernel (shared by workspace sizing and launch).
 struct DecodeGeometry {

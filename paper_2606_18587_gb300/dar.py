@@ -64,7 +64,7 @@ def load_library(path: str = LIB_PATH):
         "dar_attn_decode": ([CP, I32, P, P, P, F, P, P, SZ, P], ctypes.c_int),
         "dar_prefill_workspace_bytes": ([ctypes.c_int, I32, I32, I32, I32], SZ),
         "dar_attn_prefill": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, P, P,
-                              SZ, P], ctypes.c_int),
+                              SZ, P, P], ctypes.c_int),
         "dar_last_error": ([], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -219,8 +219,10 @@ def dar_prefill_workspace_bytes(dtype, B, Hkv, N, d_down) -> int:
     return int(load_library().dar_prefill_workspace_bytes(_CODE[dtype], B, Hkv, N, d_down))
 
 
-def dar_attn_prefill(q, k, v, Dk, Uk, Dv, Uv, w, scale=0.0, out=None, workspace=None, stream=None):
-    """Causal forward: ``q [B,Hq,N,d]``, ``k, v [B,Hkv,N,d]`` -> ``[B,Hq,N,d]``."""
+def dar_attn_prefill(q, k, v, Dk, Uk, Dv, Uv, w, scale=0.0, out=None, workspace=None, status=None,
+                     stream=None):
+    """Causal forward: ``q [B,Hq,N,d]``, ``k, v [B,Hkv,N,d]`` -> ``[B,Hq,N,d]``.
+    ``status`` is an optional device int32 tensor receiving device-side errors."""
     _dev(q, "q")
     _dev(k, "k", q.dtype)
     _dev(v, "v", q.dtype)
@@ -236,7 +238,9 @@ def dar_attn_prefill(q, k, v, Dk, Uk, Dv, Uv, w, scale=0.0, out=None, workspace=
         workspace = torch.empty(max(1, dar_prefill_workspace_bytes(q.dtype, B, Hkv, N, dd)),
                                 dtype=torch.uint8, device=q.device)
     _dev(workspace, "workspace")
+    if status is not None:
+        _dev(status, "status", torch.int32)
     _check(load_library().dar_attn_prefill(
         _code(q), B, Hq, Hkv, N, d, dd, int(w), _ptr(q), _ptr(k), _ptr(v), _ptr(Dk), _ptr(Uk), _ptr(Dv), _ptr(Uv),
-        float(scale), _ptr(out), _ptr(workspace), workspace.numel(), _stream(stream)))
+        float(scale), _ptr(out), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
     return out

@@ -52,7 +52,7 @@ def test_workspace_sizes_are_host_only(lib):
 
 @pytest.mark.parametrize("kw,code", [
     (dict(d=32), 2), (dict(d_down=12), 2), (dict(w=0), 1), (dict(Hkv=0), 1), (dict(dtype=7), 1),
-    (dict(win_k=0), 1), (dict(win_k=258), 1), (dict(B=5000), 2),
+    (dict(win_k=0), 1), (dict(win_k=258), 1), (dict(B=5000), 2), (dict(B=1025), 2),
 ])
 def test_decode_rejects_bad_cache(lib, kw, code):
     L = lib.load_library()
@@ -66,13 +66,14 @@ def test_prefill_rejects_bad_arguments(lib):
     L = lib.load_library()
     P = 4096
     args = lambda **kw: dict(dict(dtype=lib.DAR_BF16, B=1, Hq=4, Hkv=2, N=16, d=64, dd=16, w=4, q=P, k=P, v=P,  # noqa
-                                   Dk=P, Uk=P, Dv=P, Uv=P, scale=0.0, out=P, ws=P, wsb=1 << 20, s=None), **kw)
+                                   Dk=P, Uk=P, Dv=P, Uv=P, scale=0.0, out=P, ws=P, wsb=1 << 20, st=None, s=None),
+                              **kw)
 
     def call(**kw):
         a = args(**kw)
         return L.dar_attn_prefill(a["dtype"], a["B"], a["Hq"], a["Hkv"], a["N"], a["d"], a["dd"], a["w"],
                                   a["q"], a["k"], a["v"], a["Dk"], a["Uk"], a["Dv"], a["Uv"], a["scale"],
-                                  a["out"], a["ws"], a["wsb"], a["s"])
+                                  a["out"], a["ws"], a["wsb"], a["st"], a["s"])
     assert call(Hq=3) == 1
     assert call(w=-1) == 1
     assert call(d=128) == 2
