@@ -141,6 +141,28 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
                            const float *Uv, float scale, void *out, void *workspace,
                            size_t workspace_bytes, void *stream);
 
+/*
+ * dar_attn_decode for callers that cannot allocate device memory (the paper
+ * has no counterpart; this is an interface convenience).  Some callers have
+ * no device allocator to draw a workspace from (code embedded in a host
+ * framework that exposes none), or must not allocate once serving has started.
+ * This entry point allocates nothing: its scratch is one file-scope device
+ * array of DAR_DECODE_NOALLOC_MAX_BYTES that every GPU which loads the library
+ * holds until the process exits.  Arguments and results are those of
+ * dar_attn_decode; the caller still provides q and out.
+ *  - A cache shape whose dar_decode_workspace_bytes() exceeds the maximum is
+ *    rejected with DAR_ERR_CAPACITY and nothing is launched.
+ *  - The first call on a device looks up the array's device address (with
+ *    that device current); make that first call before any stream capture.
+ *  - Every call clears the part of the array it uses (a memset on `stream`)
+ *    before the kernel runs.  All calls share the one array, so calls that
+ *    overlap on the device (other streams, other threads) race: serialise them.
+ */
+#define DAR_DECODE_NOALLOC_MAX_BYTES (8u << 20)
+dar_status dar_attn_decode_noalloc(const dar_cache *cache, int32_t Hq, const void *q,
+                                   const float *Uk, const float *Uv, float scale, void *out,
+                                   void *stream);
+
 /* Bytes of workspace dar_attn_prefill needs (the Eq. 1 vectors of all tokens). */
 size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t N,
                                    int32_t d_down);

@@ -109,6 +109,8 @@ DecodeLayout decode_layout(const dar_cache *c, int Hq, const dar::DecodeGeometry
 
 }  // namespace
 
+void dar::set_last_error(const char *msg) { g_err = msg ? msg : ""; }
+
 extern "C" {
 
 const char *dar_last_error(void) { return g_err.c_str(); }

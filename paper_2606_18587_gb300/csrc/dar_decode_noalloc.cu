@@ -1,0 +1,65 @@
+// dar_decode_noalloc.cu -- dar_attn_decode for callers that cannot allocate
+// device memory.
+//
+// Some callers have no way to obtain a device buffer for the decode
+// workspace: code embedded in a host framework that exposes no device
+// allocator, or serving loops whose policy forbids any allocation after
+// start-up.  For them this entry point takes its scratch from one
+// file-scope __device__ array of DAR_DECODE_NOALLOC_MAX_BYTES that every GPU
+// loading the library holds until the process exits.
+#include <stdio.h>
+
+#include "dar_common.cuh"
+#include "dar_launch.h"
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_decode_scratch[DAR_DECODE_NOALLOC_MAX_BYTES];
+
+constexpr int kMaxDevices = 64;
+void *g_scratch_ptr[kMaxDevices] = {};  // device address of g_decode_scratch, per device
+
+}  // namespace
+
+extern "C" dar_status dar_attn_decode_noalloc(const dar_cache *cache, int32_t Hq, const void *q,
+                                              const float *Uk, const float *Uv, float scale, void *out,
+                                              void *stream)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+        dar::set_last_error("dar_attn_decode_noalloc: no usable current device");
+        return DAR_ERR_CUDA;
+    }
+    // One-time set-up on this device (with it current): the host-side name of
+    // the array is not a device address, so ask the runtime for the address.
+    if (!g_scratch_ptr[dev]) {
+        void *p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_decode_scratch);
+        if (e != cudaSuccess || !p) {
+            dar::set_last_error(cudaGetErrorString(e));
+            return DAR_ERR_CUDA;
+        }
+        g_scratch_ptr[dev] = p;
+    }
+    const size_t need = dar_decode_workspace_bytes(cache, Hq);
+    if (need == 0)  // invalid cache or Hq: the regular entry point reports which, launching nothing
+        return dar_attn_decode(cache, Hq, q, Uk, Uv, scale, out, g_scratch_ptr[dev], 0, stream);
+    if (need > DAR_DECODE_NOALLOC_MAX_BYTES) {
+        char msg[160];
+        snprintf(msg, sizeof msg,
+                 "dar_attn_decode_noalloc: this cache shape needs %zu bytes of scratch, more than the "
+                 "built-in %u (use dar_attn_decode with a workspace)",
+                 need, (unsigned)DAR_DECODE_NOALLOC_MAX_BYTES);
+        dar::set_last_error(msg);
+        return DAR_ERR_CAPACITY;
+    }
+    // The array keeps whatever the previous call left; the decode kernel needs
+    // its counters at zero, so clear the region this call uses.
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const cudaError_t e = cudaMemsetAsync(g_scratch_ptr[dev], 0, need, s);
+    if (e != cudaSuccess) {
+        dar::set_last_error(cudaGetErrorString(e));
+        return DAR_ERR_CUDA;
+    }
+    return dar_attn_decode(cache, Hq, q, Uk, Uv, scale, out, g_scratch_ptr[dev], need, stream);
+}

@@ -66,4 +66,7 @@ struct DecodeGeometry {
 };
 DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int maxp);
 
+// Set the message dar_last_error() returns on this thread.
+void set_last_error(const char *msg);
+
 }  // namespace dar

@@ -62,6 +62,7 @@ def load_library(path: str = LIB_PATH):
         "dar_cache_append": ([CP, P, P, I32, P, P, P, P], ctypes.c_int),
         "dar_decode_workspace_bytes": ([CP, I32], SZ),
         "dar_attn_decode": ([CP, I32, P, P, P, F, P, P, SZ, P], ctypes.c_int),
+        "dar_attn_decode_noalloc": ([CP, I32, P, P, P, F, P, P], ctypes.c_int),
         "dar_prefill_workspace_bytes": ([ctypes.c_int, I32, I32, I32, I32], SZ),
         "dar_attn_prefill": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, P, P,
                               SZ, P, P], ctypes.c_int),
@@ -210,6 +211,21 @@ def dar_attn_decode(cache: DarCache, q, Uk, Uv, workspace, scale=0.0, out=None, 
     _check(load_library().dar_attn_decode(cache.struct, Hq, _ptr(q), _ptr(Uk), _ptr(Uv), float(scale),
                                           _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                           _stream(stream)))
+    return out
+
+
+def dar_attn_decode_noalloc(cache: DarCache, q, Uk, Uv, scale=0.0, out=None, stream=None):
+    """dar_attn_decode without a caller workspace: the library's built-in device
+    scratch array is used instead (for callers that cannot allocate).  Calls
+    that overlap on the device share that array and must be serialised."""
+    _dev(q, "q", cache.dtype)
+    _dev(Uk, "Uk", torch.float32)
+    _dev(Uv, "Uv", torch.float32)
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", cache.dtype)
+    _check(load_library().dar_attn_decode_noalloc(cache.struct, q.shape[1], _ptr(q), _ptr(Uk), _ptr(Uv),
+                                                  float(scale), _ptr(out), _stream(stream)))
     return out
 
 
