@@ -1,6 +1,7 @@
 // dar_launch.h -- internal launchers behind the C ABI (host side).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -32,7 +33,7 @@ struct DecodeArgs {
     const float *Uk, *Uv;  // [Hkv][dd][64]
     float *rec_m, *rec_l, *rec_acc;  // split-K partial results
     int32_t *counters;               // per (b, g, head slice) arrival counts
-    int32_t *sched;                  // [2] dynamic item counter, exited-warp counter
+    int32_t *sched;                  // [2] item counter, exited-warp counter
     int B, Hq, Hkv, G, GH, HS, w, maxp, num_pages, maxc, cw, cd;
     float qscale;  // scale * log2(e)
 };
@@ -65,6 +66,10 @@ struct DecodeGeometry {
     int cw, cd, maxc, GH, HS;
 };
 DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int maxp);
+
+// 2-D tensor map of a bf16 row-major [rows][cols] array (cols * 2 = 16, 32, 64
+// or 128 bytes, swizzled to match) with boxes of [box_rows][cols].
+bool make_tma_2d_bf16(CUtensorMap *map, const void *base, unsigned long long rows, int cols, int box_rows);
 
 // Set the message dar_last_error() returns on this thread.
 void set_last_error(const char *msg);

@@ -2,10 +2,10 @@
 // tensor cores: tcgen05.mma with operands in shared memory (staged by TMA) and
 // fp32 accumulators in tensor memory (TMEM).
 //
-// One CTA = 128 query rows of one head; key tiles of 128, visited from the
-// diagonal tile down to tile 0.  Per key tile (Eq. 3: local iff i - j < w):
-//   local part   S_loc  = Q  K^T       (M128 N128 K64)   O_loc  += P_loc  V    (N64)
-//   global part  S_glob = Q~ (K^D)^T   (M128 N128 Kdd)   O_glob += P_glob V^D  (Ndd)
+// One CTA = 128 query rows of one head; key tiles of 64, visited from the
+// diagonal down to key 0.  Per key tile (Eq. 3: local iff i - j < w):
+//   local part   S_loc  = Q  K^T       (M128 N64 K64)   O_loc  += P_loc  V    (N64)
+//   global part  S_glob = Q~ (K^D)^T   (M128 N64 Kdd)   O_glob += P_glob V^D  (Ndd)
 // with q~ = q Uk^T (W_up absorbed into the query, exact by linearity of
 // Eq. 2).  A tile issues only the parts it needs; a band tile (both kinds)
 // selects per element.  One online softmax over both parts (Eq. 4), with the
@@ -14,8 +14,10 @@
 //
 // Warp roles (192 threads): warp 0 issues TMA loads, warp 1 allocates TMEM and
 // issues the MMAs (one thread), warps 2-5 own one query row per thread
-// (TMEM lane = row) for q~, the softmax and the epilogue.  Every wait is
-// bounded; on a timeout the CTA flags *status, drains and exits.
+// (TMEM lane = row) for q~, the softmax and the epilogue.  256 TMEM columns
+// and ~100 KB of shared memory per CTA let two CTAs share an SM, so one CTA's
+// softmax overlaps the other's MMA and load waits.  Every wait is bounded; on
+// a timeout the CTA flags *status and exits.
 #include <cuda.h>
 
 #include "dar_common.cuh"
@@ -27,10 +29,10 @@ namespace tcp {
 
 using namespace sm100;
 
-constexpr int BM = 128, BN = 128;
+constexpr int BM = 128, BN = 64;
 constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t COL_SL = 0, COL_SG = 128, COL_OL = 256, COL_OG = 320;
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t COL_SL = 0, COL_SG = 64, COL_OL = 128, COL_OG = 192;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p stays below 2^8 between rescales
 
 constexpr uint32_t align_up(uint32_t x, uint32_t a) { return (x + a - 1) / a * a; }
@@ -38,16 +40,16 @@ constexpr uint32_t align_up(uint32_t x, uint32_t a) { return (x + a - 1) / a * a
 // Shared-memory layout (offsets from a 1024-byte aligned base).
 template <int DP>
 struct Layout {
-    static constexpr int NS = DP == 64 ? 1 : 2;          // K/V stages
+    static constexpr int NS = 2;                          // K/V stages
     static constexpr uint32_t Q = 0;                      // [128][64] bf16, 128B swizzle
     static constexpr uint32_t QT = BM * 64 * 2;           // [128][DP] bf16
     static constexpr uint32_t STG = align_up(QT + BM * DP * 2, 1024);
-    static constexpr uint32_t K_OFF = 0;                  // [128][64]
-    static constexpr uint32_t V_OFF = BN * 64 * 2;        // [128][64]
-    static constexpr uint32_t KD_OFF = 2 * BN * 64 * 2;   // [128][DP]
+    static constexpr uint32_t K_OFF = 0;                  // [64][64]
+    static constexpr uint32_t V_OFF = BN * 64 * 2;        // [64][64]
+    static constexpr uint32_t KD_OFF = 2 * BN * 64 * 2;   // [64][DP]
     static constexpr uint32_t VD_OFF = KD_OFF + BN * DP * 2;
-    static constexpr uint32_t STAGE = VD_OFF + BN * DP * 2;
-    static constexpr uint32_t PL = STG + NS * STAGE;      // P_loc  [2 atoms][128][64] bf16
+    static constexpr uint32_t STAGE = align_up(VD_OFF + BN * DP * 2, 1024);
+    static constexpr uint32_t PL = STG + NS * STAGE;      // P_loc  [128][64] bf16 (one 128B-swizzle atom wide)
     static constexpr uint32_t PG = PL + BM * BN * 2;      // P_glob
     static constexpr uint32_t UK = PG + BM * BN * 2;      // fp32 [DP][64]
     static constexpr uint32_t UV = UK + DP * 64 * 4;
@@ -75,6 +77,36 @@ __device__ __forceinline__ TileKind tile_kind(int i0, int i_last, int j0, int w)
     return k;
 }
 
+template <int N>
+__device__ __forceinline__ float tree_max(const float (&v)[N])
+{
+    float t[N / 2];
+#pragma unroll
+    for (int e = 0; e < N / 2; ++e)
+        t[e] = fmaxf(v[2 * e], v[2 * e + 1]);
+#pragma unroll
+    for (int n = N / 4; n >= 1; n /= 2)
+#pragma unroll
+        for (int e = 0; e < n; ++e)
+            t[e] = fmaxf(t[e], t[e + n]);
+    return t[0];
+}
+
+template <int N>
+__device__ __forceinline__ float tree_sum(const float (&v)[N])
+{
+    float t[N / 2];
+#pragma unroll
+    for (int e = 0; e < N / 2; ++e)
+        t[e] = v[2 * e] + v[2 * e + 1];
+#pragma unroll
+    for (int n = N / 4; n >= 1; n /= 2)
+#pragma unroll
+        for (int e = 0; e < n; ++e)
+            t[e] = t[e] + t[e + n];
+    return t[0];
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -100,7 +132,7 @@ __device__ __forceinline__ uint4 ld_swz(const unsigned char *base, int r, int c)
 }
 
 template <int DP>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKD,
                       const __grid_constant__ CUtensorMap tmVD, PrefillArgs a)
@@ -128,7 +160,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int qt = nqt - 1 - (int)blockIdx.y;  // longest rows first
     const int bh = blockIdx.x, b = bh / a.Hq, h = bh % a.Hq, g = h / (a.Hq / a.Hkv);
     const int i0 = qt * BM, i_last = min(i0 + BM, N) - 1;
-    const int T = qt + 1;  // key tiles kt = qt - t, t = 0..T-1
+    const int T = i_last / BN + 1;  // key tiles kt = T-1-t, t = 0..T-1
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; ++s) {
@@ -167,7 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int s = t % NS;
                 if (t >= NS && !mbar_wait(&empty[s], ((t / NS) - 1) & 1, abort_flag))
                     break;
-                const int j0 = (qt - t) * BN;
+                const int j0 = (T - 1 - t) * BN;
                 const TileKind k = tile_kind(i0, i_last, j0, w);
                 const unsigned bytes = (k.loc ? 2 * BN * 64 * 2 : 0) + (k.glob ? 2 * BN * DP * 2 : 0);
                 unsigned char *st = sm + Ly::STG + s * Ly::STAGE;
@@ -200,7 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (t > 0 && !mbar_wait(s_free, (t - 1) & 1, abort_flag))
                     return false;
                 tc_fence_after();
-                const TileKind k = tile_kind(i0, i_last, (qt - t) * BN, w);
+                const TileKind k = tile_kind(i0, i_last, (T - 1 - t) * BN, w);
                 const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
                 if (k.loc)
 #pragma unroll
@@ -221,11 +253,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!mbar_wait(p_full, t & 1, abort_flag))
                     return false;
                 tc_fence_after();
-                const TileKind k = tile_kind(i0, i_last, (qt - t) * BN, w);
+                const TileKind k = tile_kind(i0, i_last, (T - 1 - t) * BN, w);
                 const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
 #pragma unroll
                 for (int kk = 0; kk < BN / 16; ++kk) {
-                    const uint32_t aoff = (kk / 4) * (BM * 128) + (kk % 4) * 32;
+                    const uint32_t aoff = kk * 32;
                     if (k.loc)
                         mma_f16_ss(tmem + COL_OL, smem_desc(sPL + aoff, 16, 1024, kSw128),
                                    smem_desc(st + Ly::V_OFF + kk * 16 * 128, 16, 1024, kSw128), idPV, true);
@@ -239,18 +271,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mma_commit(&empty[s]);
                 return true;
             };
+            // S(t) is issued as soon as the softmax has read S(t-1), so it
+            // overlaps the softmax of tile t-1; PV(t-1) follows once P(t-1) is written
             for (int t = 0; ok && t <= T; ++t) {
-                if (NS >= 2) {  // S(t) overlaps the softmax of tile t-1
-                    if (t < T)
-                        ok = issue_S(t);
-                    if (ok && t > 0)
-                        ok = issue_PV(t - 1);
-                } else {  // one stage: tile t's operands arrive only after PV(t-1)
-                    if (t > 0)
-                        ok = issue_PV(t - 1);
-                    if (ok && t < T)
-                        ok = issue_S(t);
-                }
+                if (t < T)
+                    ok = issue_S(t);
+                if (ok && t > 0)
+                    ok = issue_PV(t - 1);
             }
         }
     } else {
@@ -269,7 +296,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             sUv[idx] = in ? a.Uv[((size_t)g * a.dd + c) * 64 + t] : 0.f;
         }
         asm volatile("bar.sync 1, 128;" ::: "memory");
-        bool ok = mbar_wait(q_full, 0, abort_flag);
+        // tcgen05.ld/st are warp-collective: every branch around them is warp-uniform
+        auto wait_uniform = [&](uint64_t *bar, unsigned parity) {
+            const bool r = mbar_wait(bar, parity, abort_flag);
+            return __all_sync(0xffffffffu, r) != 0;
+        };
+        bool ok = wait_uniform(q_full, 0);
 
         // q~ row = q Uk^T  (fp32, rounded once to bf16 for the MMA)
         {
@@ -286,17 +318,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 q[8 * c + 6] = bf16lo(v.w);
                 q[8 * c + 7] = bf16hi(v.w);
             }
-#pragma unroll
+#pragma unroll 1
             for (int c8 = 0; c8 < DP / 8; ++c8) {
                 float o[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
                     const float *u = sUk + (c8 * 8 + e) * 64;
-                    float acc = 0.f;
+                    float a0 = 0.f, a1 = 0.f;
 #pragma unroll
-                    for (int t = 0; t < 64; ++t)
-                        acc = fmaf(q[t], u[t], acc);
-                    o[e] = acc;
+                    for (int t = 0; t < 64; t += 2) {
+                        a0 = fmaf(q[t], u[t], a0);
+                        a1 = fmaf(q[t + 1], u[t + 1], a1);
+                    }
+                    o[e] = a0 + a1;
                 }
                 st_swz<DP * 2>(sm + Ly::QT, row, c8,
                                make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]),
@@ -320,15 +354,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float c2 = a.qscale;  // softmax scale * log2(e)
         float m_used = -INFINITY, l = 0.f;
         int pv_waited = -1;  // highest tile whose PV completion has been observed
-        // tcgen05.ld/st are warp-collective: every branch around them is warp-uniform
-        auto wait_uniform = [&](uint64_t *bar, unsigned parity) {
-            const bool r = mbar_wait(bar, parity, abort_flag);
-            return __all_sync(0xffffffffu, r) != 0;
-        };
-        ok = __all_sync(0xffffffffu, ok) != 0;
         for (int t = 0; ok && t < T; ++t) {
-            const int j0 = (qt - t) * BN;
+            const int j0 = (T - 1 - t) * BN;
             const TileKind k = tile_kind(i0, i_last, j0, w);
+            const bool band = k.loc && k.glob;
             if (!wait_uniform(s_full, t & 1)) {
                 ok = false;
                 break;
@@ -338,17 +367,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int c = 0; c < BN; c += 32) {
                 uint32_t r[32];
-                if (k.loc && k.glob) {
+                tmem_ld32(tl + (k.loc ? COL_SL : COL_SG) + c, r);
+                if (band) {
                     uint32_t r2[32];
-                    tmem_ld32(tl + COL_SL + c, r);
                     tmem_ld32(tl + COL_SG + c, r2);
-                    tmem_wait_ld();
 #pragma unroll
                     for (int e = 0; e < 32; ++e)
                         s[c + e] = (i - (j0 + c + e) < w) ? __uint_as_float(r[e]) : __uint_as_float(r2[e]);
                 } else {
-                    tmem_ld32(tl + (k.loc ? COL_SL : COL_SG) + c, r);
-                    tmem_wait_ld();
 #pragma unroll
                     for (int e = 0; e < 32; ++e)
                         s[c + e] = __uint_as_float(r[e]);
@@ -356,22 +382,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_before();
             mbar_arrive(s_free);
-            // causal mask (diagonal tile) and rows past the end
-            if (t == 0 || i >= N) {
+            // causal mask (tiles reaching past row i0) and rows past the end
+            if (j0 + BN - 1 > i0 || i >= N) {
 #pragma unroll
                 for (int e = 0; e < BN; ++e)
                     if (j0 + e > i || i >= N)
                         s[e] = -INFINITY;
             }
-            float mx = -INFINITY;
-#pragma unroll
-            for (int e = 0; e < BN; ++e)
-                mx = fmaxf(mx, s[e]);
-            const float mt = mx * c2;
+            const float mt = tree_max(s) * c2;
             // raise the running max only when it grows by more than the threshold
             const bool raise = mt > m_used + kRescaleThreshold;
             const bool scale_o = raise && m_used != -INFINITY;
-            const float alpha = scale_o ? exp2f(m_used - mt) : 1.f;
+            const float alpha = scale_o ? ex2_approx(m_used - mt) : 1.f;
             if (__any_sync(0xffffffffu, scale_o)) {
                 // every earlier PV must have landed before O is rescaled
                 if (pv_waited < t - 1) {
@@ -386,7 +408,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int c = 0; c < 64 + DP; c += 16) {
                     uint32_t r[16];
                     tmem_ld16(tl + COL_OL + c, r);
-                    tmem_wait_ld();
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
                         r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
@@ -397,15 +418,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             l *= alpha;
             if (raise)
                 m_used = mt;
-            // P = exp2(s * c2 - m)
-            float psum = 0.f;
+            // P = 2^(s * c2 - m); masked entries (s = -inf) give 0
+            const float mneg = m_used == -INFINITY ? 0.f : -m_used;
 #pragma unroll
-            for (int e = 0; e < BN; ++e) {
-                const float p = (s[e] == -INFINITY) ? 0.f : exp2f(fmaf(s[e], c2, -m_used));
-                s[e] = p;
-                psum += p;
-            }
-            l += psum;
+            for (int e = 0; e < BN; ++e)
+                s[e] = ex2_approx(fmaf(s[e], c2, mneg));
+            l += tree_sum(s);
             // the PV of the previous tile must be done reading the P buffers
             if (t > 0 && pv_waited < t - 1) {
                 if (!wait_uniform(pv_done, (t - 1) & 1)) {
@@ -415,7 +433,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 pv_waited = t - 1;
                 tc_fence_after();
             }
-            const bool band = k.loc && k.glob;
 #pragma unroll
             for (int c = 0; c < BN / 8; ++c) {
                 float vl[8], vg[8];
@@ -426,14 +443,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     vl[e] = is_loc ? s[8 * c + e] : 0.f;
                     vg[e] = is_loc ? 0.f : s[8 * c + e];
                 }
-                unsigned char *atomL = sm + Ly::PL + (c / 8) * (BM * 128);
-                unsigned char *atomG = sm + Ly::PG + (c / 8) * (BM * 128);
                 if (k.loc)
-                    st_swz<128>(atomL, row, c % 8,
+                    st_swz<128>(sm + Ly::PL, row, c,
                                 make_uint4(pack_bf16(vl[0], vl[1]), pack_bf16(vl[2], vl[3]),
                                            pack_bf16(vl[4], vl[5]), pack_bf16(vl[6], vl[7])));
                 if (k.glob)
-                    st_swz<128>(atomG, row, c % 8,
+                    st_swz<128>(sm + Ly::PG, row, c,
                                 make_uint4(pack_bf16(vg[0], vg[1]), pack_bf16(vg[2], vg[3]),
                                            pack_bf16(vg[4], vg[5]), pack_bf16(vg[6], vg[7])));
             }
@@ -516,15 +531,16 @@ static EncodeTiledFn encode_fn()
     return fn;
 }
 
-// 2-D bf16 tensor [rows][cols] (row pitch = cols), box [128 rows][cols].
-static bool make_map(CUtensorMap *m, const void *base, unsigned long long rows, int cols, CUtensorMapSwizzle sw)
+// 2-D bf16 tensor [rows][cols] (row pitch = cols), box [box_rows][cols].
+static bool make_map(CUtensorMap *m, const void *base, unsigned long long rows, int cols, int box_rows,
+                     CUtensorMapSwizzle sw)
 {
     EncodeTiledFn fn = encode_fn();
     if (!fn)
         return false;
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-    cuuint32_t box[2] = {(cuuint32_t)cols, 128};
+    cuuint32_t box[2] = {(cuuint32_t)cols, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -539,10 +555,10 @@ static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
                                    : DP == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
                                               : CU_TENSOR_MAP_SWIZZLE_128B;
     const unsigned long long rq = (unsigned long long)a.B * a.Hq * a.N, rk = (unsigned long long)a.B * a.Hkv * a.N;
-    if (!make_map(&mq, a.q, rq, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&mk, a.k, rk, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&mv, a.v, rk, 64, CU_TENSOR_MAP_SWIZZLE_128B) || !make_map(&mkd, a.kd, rk, DP, swd) ||
-        !make_map(&mvd, a.vd, rk, DP, swd))
+    if (!make_map(&mq, a.q, rq, 64, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&mk, a.k, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&mv, a.v, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) || !make_map(&mkd, a.kd, rk, DP, BN, swd) ||
+        !make_map(&mvd, a.vd, rk, DP, BN, swd))
         return cudaErrorInvalidValue;
     auto kern = prefill_tc_kernel<DP>;
     const size_t smem = Layout<DP>::TOTAL + 1024;
@@ -559,6 +575,15 @@ static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
 }
 
 }  // namespace tcp
+
+bool make_tma_2d_bf16(CUtensorMap *map, const void *base, unsigned long long rows, int cols, int box_rows)
+{
+    const CUtensorMapSwizzle sw = cols == 8    ? CU_TENSOR_MAP_SWIZZLE_NONE
+                                  : cols == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
+                                  : cols == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                               : CU_TENSOR_MAP_SWIZZLE_128B;
+    return tcp::make_map(map, base, rows, cols, box_rows, sw);
+}
 
 cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s)
 {

@@ -64,6 +64,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, unsigned parity)
     return ok != 0;
 }
 
+// As mbar_try_wait, but the hardware may park the thread for up to `ns`
+// nanoseconds while the phase is incomplete (it wakes early on completion), so
+// a waiting warp does not keep issuing polls.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, unsigned parity, unsigned ns)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Wait for the phase with the given parity.  Gives up after kWaitLimitNs of
 // wall time, or as soon as *abort is set by another thread; returns false
 // then (and sets *abort).
@@ -73,9 +89,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, volati
         return true;
     const unsigned long long t0 = globaltimer_ns();
     for (unsigned i = 1;; ++i) {
-        if (mbar_try_wait(bar, parity))
+        if (mbar_try_wait_sleep(bar, parity, 20000u))
             return true;
-        if ((i & 63u) == 0u) {
+        if ((i & 7u) == 0u) {
             if (abort && *abort)
                 return false;
             if (globaltimer_ns() - t0 > kWaitLimitNs)
@@ -118,6 +134,52 @@ __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map)
 __device__ __forceinline__ void fence_proxy_async_smem()
 {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// 2^x with the MUFU approximation (ex2.approx.ftz.f32; flushes subnormal results to 0).
+__device__ __forceinline__ float ex2_approx(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// ------------------------------------------------------------------ warp-level MMA
+// (mma.sync m16n8k16, bf16 inputs, fp32 accumulators; fragment layouts per the
+// PTX ISA: lane = 4 * group + tig; A rows group / group + 8, B column group.)
+
+__device__ __forceinline__ void ldsm_x4(uint32_t saddr, uint32_t (&r)[4])
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(saddr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t saddr, uint32_t (&r)[4])
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(saddr));
+}
+
+// d += a * b  (A 16x16 row-major, B 16x8 column-major, D 16x8 fp32)
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1)
+{
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// 2-D tiled TMA load of a box whose innermost extent is `x` elements.
+__device__ __forceinline__ void tma_load_2d_u(uint32_t dst, const CUtensorMap *map, int x, int y, uint64_t *bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+        "[%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
 }
 
 // ------------------------------------------------------------------ tcgen05
