@@ -51,8 +51,8 @@ typedef enum { DAR_F32 = 0, DAR_BF16 = 1 } dar_dtype;
 /* Tokens per page of the bottleneck pool. */
 #define DAR_PAGE_SIZE 64
 
-/* Largest batch dar_attn_decode accepts (its per-sequence tables live in
- * shared memory). */
+/* Largest batch dar_attn_decode accepts (its per-sequence tables are built by
+ * one thread block of 1024 threads, one thread per sequence). */
 #define DAR_DECODE_MAX_BATCH 1024
 
 /*
@@ -120,10 +120,8 @@ dar_status dar_cache_append(const dar_cache *cache, const void *k_new, const voi
 
 /*
  * Bytes of workspace dar_attn_decode needs for this cache shape and Hq query
- * heads.  The workspace must be zero-filled once before its first use (for
- * example with cudaMemsetAsync); every completed call leaves it zero-filled
- * again, so it can be reused without clearing.  Calls that share one
- * workspace must not overlap on the device.
+ * heads.  The workspace needs no initialisation: every call rewrites what it
+ * reads.  Calls that share one workspace must not overlap on the device.
  */
 size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq);
 
@@ -132,10 +130,13 @@ size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq);
  * sequence, L_b = seq_lens[b]): scores against the ring (full d) and the
  * pages (d_down, with W_up absorbed into the query, q~ = q Uk^T), one softmax
  * over both, values lifted once, o = (sum_local p v + (sum_global p v^D) Uv) / sum p.
- *   q [B][Hq][d] T; Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][d] T.
- * A sequence with L_b == 0 gets a zero output.  Split-K over the sequence with
- * the partial results combined inside the same kernel.  B <= DAR_DECODE_MAX_BATCH.
- * After a call that set *status, zero-fill the workspace again before reuse.
+ *   q [B][Hq][d] T; Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][d] T; q, out,
+ *   Uk, Uv and the workspace 16-byte aligned.
+ * A sequence with L_b == 0 gets a zero output.  Split-K over the sequence:
+ * three kernels run in order on `stream` (item set-up and q~, streaming,
+ * combine).  B <= DAR_DECODE_MAX_BATCH.  A length beyond the cache's capacity
+ * or a needed block-table entry outside [0, num_pages) sets
+ * *status = DAR_ERR_CAPACITY; out is then undefined for that sequence.
  */
 dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, const float *Uk,
                            const float *Uv, float scale, void *out, void *workspace,
@@ -154,9 +155,9 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
  *    rejected with DAR_ERR_CAPACITY and nothing is launched.
  *  - The first call on a device looks up the array's device address (with
  *    that device current); make that first call before any stream capture.
- *  - Every call clears the part of the array it uses (a memset on `stream`)
- *    before the kernel runs.  All calls share the one array, so calls that
- *    overlap on the device (other streams, other threads) race: serialise them.
+ *  - The array needs no clearing (every call rewrites what it reads).  All
+ *    calls share the one array, so calls that overlap on the device (other
+ *    streams, other threads) race: serialise them.
  */
 #define DAR_DECODE_NOALLOC_MAX_BYTES (8u << 20)
 dar_status dar_attn_decode_noalloc(const dar_cache *cache, int32_t Hq, const void *q,

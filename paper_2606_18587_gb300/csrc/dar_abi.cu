@@ -91,9 +91,12 @@ dar_status check_cache(const dar_cache *c)
 }
 
 struct DecodeLayout {
-    size_t m, l, acc, counters, sched, total;
+    size_t m, l, acc, qt, counters, total;
 };
 
+// Workspace of dar_attn_decode: split-K records for the smallest chunks, the
+// absorbed queries and one counter per (sequence, KV head, head slice) group.
+// Every call rewrites what it reads.
 DecodeLayout decode_layout(const dar_cache *c, int Hq, const dar::DecodeGeometry &gm)
 {
     DecodeLayout L;
@@ -101,9 +104,9 @@ DecodeLayout decode_layout(const dar_cache *c, int Hq, const dar::DecodeGeometry
     L.m = 0;
     L.l = L.m + align256(recs * sizeof(float));
     L.acc = L.l + align256(recs * sizeof(float));
-    L.counters = L.acc + align256(recs * dar::kHeadDim * sizeof(float));
-    L.sched = L.counters + align256((size_t)c->B * c->Hkv * gm.HS * sizeof(int32_t));
-    L.total = L.sched + 256;
+    L.qt = L.acc + align256(recs * dar::kHeadDim * sizeof(float));
+    L.counters = L.qt + align256((size_t)c->B * Hq * c->d_down * sizeof(float));
+    L.total = L.counters + align256((size_t)c->B * c->Hkv * gm.HS * sizeof(int32_t));
     return L;
 }
 
@@ -199,11 +202,14 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
         return ok();
     if (!q || !Uk || !Uv || !out || !workspace)
         return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
-    if (!aligned16(Uk) || !aligned16(Uv) || !aligned16(workspace))
-        return fail(DAR_ERR_INVALID_ARG, "Uk, Uv and workspace must be 16-byte aligned");
+    if (!aligned16(q) || !aligned16(out) || !aligned16(Uk) || !aligned16(Uv) || !aligned16(workspace))
+        return fail(DAR_ERR_INVALID_ARG, "q, out, Uk, Uv and workspace must be 16-byte aligned");
     dar::DecodeGeometry gm = dar::decode_geometry(cache->dtype, Hq, cache->Hkv, cache->d_down,
                                                   cache->w, cache->max_pages_per_seq);
     DecodeLayout L = decode_layout(cache, Hq, gm);
+    if ((double)cache->B * Hq * gm.maxc >= 2147483647.0)
+        return fail(DAR_ERR_UNSUPPORTED, "B * Hq * chunks = %.0f exceeds the int32 record index",
+                    (double)cache->B * Hq * gm.maxc);
     if (workspace_bytes < L.total)
         return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
     char *ws = static_cast<char *>(workspace);
@@ -222,8 +228,8 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
     a.rec_m = reinterpret_cast<float *>(ws + L.m);
     a.rec_l = reinterpret_cast<float *>(ws + L.l);
     a.rec_acc = reinterpret_cast<float *>(ws + L.acc);
+    a.qt = reinterpret_cast<float *>(ws + L.qt);
     a.counters = reinterpret_cast<int32_t *>(ws + L.counters);
-    a.sched = reinterpret_cast<int32_t *>(ws + L.sched);
     a.B = cache->B;
     a.Hq = Hq;
     a.Hkv = cache->Hkv;

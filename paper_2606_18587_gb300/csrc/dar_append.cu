@@ -6,6 +6,7 @@
 // token's cached vector is bit-identical whichever kernel produced it.
 #include "dar_common.cuh"
 #include "dar_launch.h"
+#include "dar_sm100.cuh"
 
 namespace dar {
 
@@ -57,100 +58,46 @@ __global__ void __launch_bounds__(128) down_project_kernel(const T *__restrict__
 }
 
 // ------------------------------------------------------------ cache append
+//
+// One CTA per sequence (so its length can be updated at the end).  Thread ch
+// owns the Eq. 1 chains (kv, g, c) -- output c of KV head g of the keys
+// (kv = 0) or values (kv = 1) -- and keeps that column of W in registers.
+// Positions that leave the window in this call are staged up to kAppRows at a
+// time in shared memory (from the ring for old occupants, from k_new/v_new for
+// new tokens that leave at once); every chain thread runs its fixed-order
+// chains over the staged rows and writes the pages.  After all ring reads, the
+// new tokens that stay in the window are copied into their ring slots, then
+// the length is updated.  Loads that do not depend on the length (W columns,
+// the last new rows) are issued at entry, so a one-token step costs about two
+// round trips to memory.
+constexpr int kAppThreads = 512;
+constexpr int kAppRows = 8;  // rows staged per round (fewer for many heads)
+constexpr int kAppStageBytes = 96 << 10;
 
-// Eq. 1 for one row, computed by a warp: lane j holds x[2j], x[2j+1] and lane
-// c (and c + 32) runs the fixed-order chain for output c, reading x[t] by
-// shuffle and its column of W from registers loaded in one batch.
-template <typename T, int DD>
-__device__ __forceinline__ void project_row_warp(const T *x, const float *W, T *out, int lane)
-{
-    constexpr int CPL = (DD + 31) / 32;
-    const float x0 = to_f32(x[2 * lane]), x1 = to_f32(x[2 * lane + 1]);
-    float wcol[CPL][kHeadDim];
-#pragma unroll
-    for (int i = 0; i < CPL; ++i) {
-        const int c = lane + 32 * i;
-#pragma unroll
-        for (int t = 0; t < kHeadDim; ++t)
-            wcol[i][t] = c < DD ? __ldg(W + t * DD + c) : 0.f;
-    }
-    float acc[CPL];
-#pragma unroll
-    for (int i = 0; i < CPL; ++i)
-        acc[i] = 0.0f;
-#pragma unroll
-    for (int t = 0; t < kHeadDim; ++t) {
-        const float xt = __shfl_sync(0xffffffffu, (t & 1) ? x1 : x0, t >> 1);
-#pragma unroll
-        for (int i = 0; i < CPL; ++i)
-            acc[i] = __fmaf_rn(xt, wcol[i][t], acc[i]);
-    }
-#pragma unroll
-    for (int i = 0; i < CPL; ++i) {
-        const int c = lane + 32 * i;
-        if (c < DD)
-            out[c] = from_f32<T>(acc[i]);
-    }
-}
-
-// Copy one 64-element row with the warp (2 elements per lane).
 template <typename T>
-__device__ __forceinline__ void copy_row_warp(const T *src, T *dst, int lane)
+__host__ __device__ inline int app_rows(int Hkv)
 {
-    if constexpr (sizeof(T) == 2) {
-        reinterpret_cast<uint32_t *>(dst)[lane] = reinterpret_cast<const uint32_t *>(src)[lane];
-    } else {
-        reinterpret_cast<uint2 *>(dst)[lane] = reinterpret_cast<const uint2 *>(src)[lane];
-    }
+    const int per_row = 2 * Hkv * kHeadDim * (int)sizeof(T);
+    const int r = kAppStageBytes / per_row;
+    return r < 1 ? 1 : r > kAppRows ? kAppRows : r;
 }
 
-// Row of the bottleneck pool for position p of sequence b, KV head g, or
-// nullptr (status set) when its block-table entry is not a valid page.
 template <typename T, int DD>
-__device__ __forceinline__ T *pool_row(const AppendArgs &a, T *pool, int b, int g, int p)
+__global__ void __launch_bounds__(kAppThreads) cache_append_kernel(AppendArgs a)
 {
-    const int lp = p / kPage;
-    const int id = lp < a.maxp ? a.block_table[(size_t)b * a.maxp + lp] : -1;
-    if (id < 0 || id >= a.num_pages) {
-        report(a.status, DAR_ERR_CAPACITY);
-        return nullptr;
-    }
-    return pool + (((size_t)id * a.Hkv + g) * kPage + (p % kPage)) * DD;
-}
-
-// grid B (one CTA per sequence, so its length can be updated at the end),
-// up to 1024 threads.  Sequence b appends nb = n_per_seq[b] (or n) tokens; k_new
-// rows are strided by n.  Work unit = (KV head g, slot touched by this call): the slot's
-// old occupant migrates to its page, then the new positions of that slot are
-// processed in order (all but the last migrate straight from k_new; the last
-// is written into the ring).
-template <typename T, int DD>
-__global__ void __launch_bounds__(1024) cache_append_kernel(AppendArgs a)
-{
-    const int b = blockIdx.x;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    constexpr int E = Granule<T>::kElems;
+    constexpr int GPR = kHeadDim / E;  // 16-byte granules per 64-element row
+    extern __shared__ __align__(16) unsigned char app_smem[];
+    T *s_x = reinterpret_cast<T *>(app_smem);  // [rows][kv][Hkv][64]
     __shared__ int s_L, s_nb, s_ok;
-    if (threadIdx.x == 0) {
-        const int L = a.seq_lens[b];
-        const int nb = a.n_per_seq ? a.n_per_seq[b] : a.n;
-        const long long Lnew = (long long)L + nb;
-        int ok = 1;
-        if (L < 0 || nb < 0 || nb > a.n) {
-            report(a.status, DAR_ERR_INVALID_ARG);
-            ok = 0;
-        } else if (Lnew - a.w > (long long)a.maxp * kPage || Lnew > 0x7fffffffLL) {
-            report(a.status, DAR_ERR_CAPACITY);
-            ok = 0;
-        }
-        s_L = L;
-        s_nb = nb;
-        s_ok = ok;
-    }
-    __syncthreads();
-    if (!s_ok || s_nb == 0)
-        return;
-    const int L = s_L, n = a.n, nb = s_nb, w = a.w, Lnew = L + nb;
-    const int touched = min(nb, w);
+    __shared__ int s_pid[kAppRows];  // page of each staged row (-1: invalid)
+
+    // a decode launched after this kernel may start its query-only work now
+    sm100::grid_dep_launch();
+    const int b = blockIdx.x, tid = threadIdx.x;
+    const int Hkv = a.Hkv, n = a.n, w = a.w;
+    const int nchains = 2 * Hkv * DD;
+    const int R = app_rows<T>(Hkv);
     const T *knew = static_cast<const T *>(a.k_new);
     const T *vnew = static_cast<const T *>(a.v_new);
     T *wk = static_cast<T *>(a.win_k);
@@ -158,41 +105,118 @@ __global__ void __launch_bounds__(1024) cache_append_kernel(AppendArgs a)
     T *pk = static_cast<T *>(a.pool_kd);
     T *pv = static_cast<T *>(a.pool_vd);
 
-    for (int u = warp; u < a.Hkv * touched; u += nwarps) {
-        const int g = u / touched;
-        const int first = L + u % touched;  // first new position landing in this slot
-        const int slot = first % w;
-        const size_t ring = ((size_t)(b * a.Hkv + g) * w + slot) * kHeadDim;
-        const float *Dk = a.Dk + (size_t)g * kHeadDim * DD;
-        const float *Dv = a.Dv + (size_t)g * kHeadDim * DD;
-        const int old = first - w;
-        if (old >= 0) {  // the slot's occupant leaves the window
-            T *rk = pool_row<T, DD>(a, pk, b, g, old);
-            T *rv = pool_row<T, DD>(a, pv, b, g, old);
-            if (rk)
-                project_row_warp<T, DD>(wk + ring, Dk, rk, lane);
-            if (rv)
-                project_row_warp<T, DD>(wv + ring, Dv, rv, lane);
+    // ---- issued at entry: the length, this thread's first W column and one
+    // granule of the last min(n, w) new rows (those land in the ring when the
+    // sequence appends all n)
+    if (tid == 0) {
+        s_L = a.seq_lens[b];
+        s_nb = a.n_per_seq ? a.n_per_seq[b] : n;
+    }
+    float wc[kHeadDim];
+    auto load_w = [&](int ch) {
+        const int kv = ch / (Hkv * DD), g = (ch / DD) % Hkv, c = ch % DD;
+        const float *W = (kv ? a.Dv : a.Dk) + (size_t)g * kHeadDim * DD + c;
+#pragma unroll
+        for (int t = 0; t < kHeadDim; ++t)
+            wc[t] = __ldg(W + (size_t)t * DD);
+    };
+    if (tid < nchains)
+        load_w(tid);
+    // granule i of the rows j0, j0 + 1, ... of k_new / v_new (i runs over
+    // [row][kv][g][granule])
+    auto new_granule = [&](int i, int j0) {
+        const int q = i % GPR, rest = i / GPR;
+        const int g = rest % Hkv, kv = (rest / Hkv) & 1, j = j0 + rest / (2 * Hkv);
+        return (kv ? vnew : knew) + (((size_t)b * Hkv + g) * n + j) * kHeadDim + q * E;
+    };
+    const int pre_rows = min(n, w);
+    uint4 pre = make_uint4(0u, 0u, 0u, 0u);
+    if (tid < 2 * Hkv * pre_rows * GPR)
+        pre = *reinterpret_cast<const uint4 *>(new_granule(tid, n - pre_rows));
+    __syncthreads();
+    if (tid == 0) {
+        const int L = s_L, nb = s_nb;
+        const long long Lnew = (long long)L + nb;
+        int ok = 1;
+        if (L < 0 || nb < 0 || nb > n) {
+            report(a.status, DAR_ERR_INVALID_ARG);
+            ok = 0;
+        } else if (Lnew - w > (long long)a.maxp * kPage || Lnew > 0x7fffffffLL) {
+            report(a.status, DAR_ERR_CAPACITY);
+            ok = 0;
         }
-        __syncwarp();
-        for (int p = first; p < Lnew; p += w) {
-            const size_t src = ((size_t)(b * a.Hkv + g) * n + (p - L)) * kHeadDim;
-            if (p + w < Lnew) {  // leaves the window within this call
-                T *rk = pool_row<T, DD>(a, pk, b, g, p);
-                T *rv = pool_row<T, DD>(a, pv, b, g, p);
-                if (rk)
-                    project_row_warp<T, DD>(knew + src, Dk, rk, lane);
-                if (rv)
-                    project_row_warp<T, DD>(vnew + src, Dv, rv, lane);
-            } else {
-                copy_row_warp(knew + src, wk + ring, lane);
-                copy_row_warp(vnew + src, wv + ring, lane);
-            }
-            __syncwarp();
-        }
+        s_ok = ok;
     }
     __syncthreads();
-    if (threadIdx.x == 0)
+    if (!s_ok || s_nb == 0)
+        return;
+    const int L = s_L, nb = s_nb, Lnew = L + nb;
+
+    // ---- positions leaving the window: [p_lo, p_hi)
+    const int p_lo = max(0, L - w), p_hi = max(0, Lnew - w);
+    for (int m0 = p_lo; m0 < p_hi; m0 += R) {
+        const int nr = min(R, p_hi - m0);
+        for (int i = tid; i < nr * 2 * Hkv * GPR; i += blockDim.x) {  // stage [row][kv][g][64]
+            const int q = i % GPR, rest = i / GPR;
+            const int g = rest % Hkv, kv = (rest / Hkv) & 1, r = rest / (2 * Hkv);
+            const int p = m0 + r;
+            const T *src = p < L ? (kv ? wv : wk) + (((size_t)b * Hkv + g) * w + p % w) * kHeadDim
+                                 : (kv ? vnew : knew) + (((size_t)b * Hkv + g) * n + (p - L)) * kHeadDim;
+            reinterpret_cast<uint4 *>(s_x)[i] = *reinterpret_cast<const uint4 *>(src + q * E);
+        }
+        if (tid < nr) {
+            const int lp = (m0 + tid) / kPage;
+            const int id = lp < a.maxp ? a.block_table[(size_t)b * a.maxp + lp] : -1;
+            const bool valid = id >= 0 && id < a.num_pages;
+            if (!valid)
+                report(a.status, DAR_ERR_CAPACITY);
+            s_pid[tid] = valid ? id : -1;
+        }
+        __syncthreads();
+        for (int ch0 = 0; ch0 < nchains; ch0 += blockDim.x) {
+            const int ch = ch0 + tid;
+            if (ch >= nchains)
+                break;
+            if (ch0 > 0)
+                load_w(ch);
+            const int kv = ch / (Hkv * DD), g = (ch / DD) % Hkv, c = ch % DD;
+            T *pool = kv ? pv : pk;
+            for (int r = 0; r < nr; ++r) {
+                const uint4 *x4 = reinterpret_cast<const uint4 *>(s_x + ((size_t)(r * 2 + kv) * Hkv + g) * kHeadDim);
+                float acc = 0.0f;  // Eq. 1: one fp32 FMA chain over t = 0..63
+#pragma unroll
+                for (int q = 0; q < GPR; ++q) {
+                    float xf[E];
+                    unpack(x4[q], xf, T());
+#pragma unroll
+                    for (int e = 0; e < E; ++e)
+                        acc = __fmaf_rn(xf[e], wc[q * E + e], acc);
+                }
+                const int id = s_pid[r], p = m0 + r;
+                if (id >= 0)
+                    pool[(((size_t)id * Hkv + g) * kPage + p % kPage) * DD + c] = from_f32<T>(acc);
+            }
+        }
+        // the first chain group's W columns are needed again in the next round
+        if (nchains > (int)blockDim.x && m0 + R < p_hi && tid < nchains)
+            load_w(tid);
+        __syncthreads();
+    }
+
+    // ---- new tokens that stay in the window: rows j_lo .. nb-1 (positions
+    // L + j); every ring read above is complete
+    const int j_lo = max(0, nb - w);
+    const int granules = 2 * Hkv * (nb - j_lo) * GPR;
+    const bool use_pre = nb == n;  // then the prefetched granules are exactly these
+    for (int i = tid; i < granules; i += blockDim.x) {
+        const int q = i % GPR, rest = i / GPR;
+        const int g = rest % Hkv, kv = (rest / Hkv) & 1, j = j_lo + rest / (2 * Hkv);
+        const uint4 v = (use_pre && i == tid) ? pre : *reinterpret_cast<const uint4 *>(new_granule(i, j_lo));
+        T *dst = (kv ? wv : wk) + (((size_t)b * Hkv + g) * w + (L + j) % w) * kHeadDim + q * E;
+        *reinterpret_cast<uint4 *>(dst) = v;
+    }
+    __syncthreads();
+    if (tid == 0)
         a.seq_lens[b] = Lnew;
 }
 
@@ -227,14 +251,22 @@ cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float
 template <typename T>
 static cudaError_t cache_append_t(int dd, const AppendArgs &a, cudaStream_t s)
 {
-    // one warp per (KV head, touched slot) unit, up to 32 warps per sequence
-    const long long units = (long long)a.Hkv * (a.n < a.w ? a.n : a.w);
-    const int threads = 32 * (int)(units < 1 ? 1 : units > 32 ? 32 : units);
+    const size_t smem = (size_t)app_rows<T>(a.Hkv) * 2 * a.Hkv * kHeadDim * sizeof(T);
+    static bool attr = false;  // one-time opt-in to more than 48 KB of shared memory
+    if (!attr) {
+        for (auto k : {cache_append_kernel<T, 8>, cache_append_kernel<T, 16>, cache_append_kernel<T, 32>,
+                       cache_append_kernel<T, 64>}) {
+            const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kAppStageBytes);
+            if (e != cudaSuccess)
+                return e;
+        }
+        attr = true;
+    }
     switch (dd) {
-    case 8: cache_append_kernel<T, 8><<<a.B, threads, 0, s>>>(a); break;
-    case 16: cache_append_kernel<T, 16><<<a.B, threads, 0, s>>>(a); break;
-    case 32: cache_append_kernel<T, 32><<<a.B, threads, 0, s>>>(a); break;
-    case 64: cache_append_kernel<T, 64><<<a.B, threads, 0, s>>>(a); break;
+    case 8: cache_append_kernel<T, 8><<<a.B, kAppThreads, smem, s>>>(a); break;
+    case 16: cache_append_kernel<T, 16><<<a.B, kAppThreads, smem, s>>>(a); break;
+    case 32: cache_append_kernel<T, 32><<<a.B, kAppThreads, smem, s>>>(a); break;
+    case 64: cache_append_kernel<T, 64><<<a.B, kAppThreads, smem, s>>>(a); break;
     default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();

@@ -1,36 +1,49 @@
 // dar_decode.cu -- one decode step of DAR attention over the mixed-dimension
 // cache (Eq. 3-4 for the query at position L_b - 1; cache scheme of Sec. 5).
 //
-// Work decomposition (split-K over the sequence):
-//   item = (sequence b, KV head g, head slice hs, chunk c).  Chunks 0..nwc-1
-//   cover the ring (full d = 64 keys/values, `cw` tokens each); the rest cover
-//   the pages (d_down vectors, `cd` tokens each, page aligned).  Each launch
-//   scales both chunk sizes so that there are a few items per warp; a warp
-//   takes its first item statically and later ones from an atomic counter,
-//   fetched one item ahead so the atomic's latency is never waited on.
+// Two kernels on the caller's stream, both launched with programmatic stream
+// serialisation:
+//
+//  prep     q~ = q Uk^T for every query row (W_up absorbed into the query,
+//           exact by linearity of Eq. 2) and zeroed group counters.  Neither
+//           needs the cache, so this overlaps the kernel before it (normally
+//           the cache append); it waits for that kernel before exiting.
+//  stream   split-K over the sequence.  Every CTA builds the per-sequence
+//           tables (lengths, chunk sizes, chunk counts) in shared memory.
+//           Work items are (sequence b, KV head g, head slice hs, chunk c),
+//           ordered by sequence, group (g, hs) and chunk; chunks 0..nwc-1
+//           cover the ring (full d = 64 keys/values), the rest the pages
+//           (d_down vectors, page aligned).  CTA k owns a contiguous range of
+//           items and its warps take them in order from a shared-memory
+//           counter.  Each item leaves one partial result (running max m, sum
+//           l, unnormalised acc) per head in the workspace.  At its end a CTA
+//           merges the groups it covered completely -- one softmax over all
+//           chunks (Eq. 4), the global part lifted once with Uv,
+//           o = (acc_local + acc_global Uv) / l -- and a group shared with
+//           other CTAs is merged by the CTA that completes its chunk count.
 //
 // Streaming: every warp owns a ring of kStages shared-memory slots of
-// kSlotBytes (keys in the first half, values in the second).  Lane 0 fills a
-// slot with 1-D TMA bulk copies (cp.async.bulk, completion counted on the
-// slot's mbarrier) and the warp consumes slots in order, refilling each one as
-// soon as it has been read, across item boundaries; page ids are loaded one
-// item ahead.  So every warp keeps up to kStages * kSlotBytes of cache in
-// flight while it computes.
+// kSlotBytes (keys in the first half, values in the second) plus a small
+// header per slot.  Lane 0 fills a slot with TMA copies (2-D tensor copies of
+// 128-byte lines into 128-byte-swizzled tiles for the tensor-core consumer --
+// pages of d_down < 64 are viewed as lines holding 64 / d_down tokens, since
+// boxes of short rows stream markedly slower -- and 1-D bulk copies otherwise;
+// completion counted on the slot's mbarrier) and, with the first stage of an
+// item, copies the item's query rows (q for the ring, q~ for the pages) into
+// the slot's header.  The warp consumes slots in order and refills each one
+// as soon as it has been read, across item boundaries, so it keeps up to
+// kStages * kSlotBytes of cache in flight while it computes.
 //
 // Compute (bf16, d_down >= 16): the two small contractions of a stage run on
 // the tensor cores with warp-level mma.sync m16n8k16 (bf16 in, fp32 out): the
 // GH query heads of the slice are rows of A, 8 tokens a column block of B,
-// fed by ldmatrix from swizzled 2-D TMA tiles; the scores stay in registers,
+// fed by ldmatrix from the swizzled tiles; the scores stay in registers,
 // become P (bf16) and multiply V (ldmatrix.trans).  Global tokens are scored
-// against q~ = q Uk^T (W_up absorbed into the query, exact by linearity of
-// Eq. 2) and their values are summed in d_down space.  Other cases (fp32
-// storage, d_down = 8) use the CUDA cores: LPT lanes own one token row (one
-// 16-byte granule each).  One online softmax (running max m, sum l, log2
-// domain) covers an item.
-//
-// Combine: each item writes (m, l, acc) per head; the warp that arrives last
-// for (b, g, hs) merges all chunks, lifts the global part once with Uv and
-// writes o = (acc_local + acc_global Uv) / l.  No warp waits on another warp.
+// against q~ and their values are summed in d_down space.  When a KV head
+// serves a single query head, page stages instead give each lane whole tokens
+// on the CUDA cores (the tensor-core tile would be 15/16 idle).  Other cases
+// (fp32 storage, d_down = 8) use the CUDA cores with LPT lanes per token row.
+// One online softmax (log2 domain) covers an item.
 #include <type_traits>
 
 #include "dar_common.cuh"
@@ -44,9 +57,13 @@ constexpr int kDecThreads = kDecWarps * 32;
 constexpr int kStages = 3;
 constexpr int kSlotBytes = 8192;
 constexpr int kHalf = kSlotBytes / 2;
-constexpr int kItemStages = 4;     // stages per minimum-size item
-constexpr int kMaxChunkScale = 16;  // items grow to at most 16x the minimum (64 pages)
-constexpr int kItemsPerWarp = 3;    // chunk sizes aim at about this many items per warp
+constexpr int kHdrBytes = 1024;     // per slot: up to 4 query rows of 64 fp32
+constexpr int kItemStages = 2;      // stages per minimum-size chunk
+constexpr int kMaxChunkScale = 32;  // chunks grow to at most 32x the minimum
+constexpr int kItemsPerWarp = 6;    // chunk sizes aim at about this many items per warp
+constexpr int kPrepThreads = 256;   // prep block size
+
+static_assert(DAR_DECODE_MAX_BATCH % kDecThreads == 0, "stream threads hold whole groups of sequences");
 
 // bf16 caches with d_down >= 16 use the tensor-core consumer (fed by 2-D TMA).
 template <typename T, int DD>
@@ -55,16 +72,27 @@ __host__ __device__ constexpr bool decode_uses_mma()
     return sizeof(T) == 2 && DD >= 16;
 }
 
+// Tokens per stage: ring rows of 64 elements, page rows of DD elements.
+template <typename T>
+__host__ __device__ constexpr int tps_ring()
+{
+    return kHalf / (kHeadDim * (int)sizeof(T));
+}
+template <typename T, int DD>
+__host__ __device__ constexpr int tps_page()
+{
+    return kHalf / (DD * (int)sizeof(T));
+}
+
 // --------------------------------------------------------------------- PTX
 
 using sm100::bulk_g2s;
 using sm100::ldsm_x4;
 using sm100::ldsm_x4_t;
-using sm100::mma_bf16_16816;
-using sm100::smem_u32;
 using sm100::mbar_expect_tx;
 using sm100::mbar_init;
-using sm100::mbar_try_wait;
+using sm100::mma_bf16_16816;
+using sm100::smem_u32;
 
 // Bounded wait (see sm100::mbar_wait); a warp that gives up reports to *status.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, int32_t *status)
@@ -75,97 +103,126 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, int32_
     return false;
 }
 
-// --------------------------------------------------------------------- items
-
+// A work item: chunk c of (sequence b, KV head g, head slice hs).
 struct Item {
     int it;  // -1 = none
-    int b, g, hs, c;
-    bool window;
-    int t0, t1;  // token range (ring slots, or distant positions)
-    int nst;     // stages
-    int nwc, nchunks;
+    int b, g, h0, window, t0, t1, nst, rec0;
+    int2 pid;  // lane j: ids of the item's pages j and 32 + j
 };
 
-struct SeqTables {
-    const int *pre;  // [B + 1] exclusive prefix of chunk counts
-    const int *len;  // [B] validated length (-1 invalid)
-    int cw, cd;      // chunk sizes of this launch (multiples of the host's minimum sizes)
-};
+// Stage metadata a slot carries from the issuing lane to the consumer.
+//   x: record index of the item's first head; y: stage | ring << 16 |
+//   last << 17 | page mask << 24; z: valid tokens in the stage.
+constexpr int kMetaRing = 1 << 16;
+constexpr int kMetaLast = 1 << 17;
 
-template <int TPS_W, int TPS_D>
-__device__ __forceinline__ Item decode_item(int it, int items, const DecodeArgs &a, SeqTables st)
-{
-    Item I;
-    I.it = it < items ? it : -1;
-    I.b = I.g = I.hs = I.c = I.t0 = I.t1 = I.nst = I.nwc = I.nchunks = 0;
-    I.window = false;
-    if (I.it < 0)
-        return I;
-    const int per_chunk = a.Hkv * a.HS;
-    const int u = it / per_chunk, rem = it % per_chunk;
-    I.g = rem / a.HS;
-    I.hs = rem % a.HS;
-    int lo = 0, hi = a.B;  // largest b with pre[b] <= u
-    while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (st.pre[mid] <= u)
-            lo = mid;
-        else
-            hi = mid;
-    }
-    I.b = lo;
-    I.c = u - st.pre[lo];
-    const int L = st.len[lo];
-    const int nwin = min(L, a.w), ndist = L - nwin;
-    I.nwc = (nwin + st.cw - 1) / st.cw;
-    I.nchunks = I.nwc + (ndist + st.cd - 1) / st.cd;
-    I.window = I.c < I.nwc;
-    if (I.window) {
-        I.t0 = I.c * st.cw;
-        I.t1 = min(nwin, I.t0 + st.cw);
-        I.nst = (I.t1 - I.t0 + TPS_W - 1) / TPS_W;
-    } else {
-        I.t0 = (I.c - I.nwc) * st.cd;
-        I.t1 = min(ndist, I.t0 + st.cd);
-        I.nst = (I.t1 - I.t0 + TPS_D - 1) / TPS_D;
-    }
-    return I;
-}
-
-template <int GH>
-struct WarpSmem {
-    float q[GH][kHeadDim];   // scaled queries
-    float qt[GH][kHeadDim];  // q~ (first dd entries); combine scratch
-};
-
-template <int GH>
+// Dynamic shared memory of the stream kernel for a batch of B sequences:
+// alignment slack, slots, headers, barriers, stage metadata, the tables.
 constexpr size_t decode_smem_bytes(int B)
 {
-    return 1024 + (size_t)kDecWarps * kStages * kSlotBytes + (size_t)kDecWarps * kStages * (8 + 8) +
-           (size_t)kDecWarps * sizeof(WarpSmem<GH>) + (size_t)(2 * B + 1) * sizeof(int);
+    return 1024 + (size_t)kDecWarps * kStages * (kSlotBytes + kHdrBytes + sizeof(uint64_t) + sizeof(int4)) +
+           (size_t)(2 * B + 1) * sizeof(int);
 }
 
-// --------------------------------------------------------------------- kernel
+// --------------------------------------------------------------------- prep
+
+// q~ = q Uk^T for every (b, h) row, one row per warp (fp32, four partial sums
+// over t mod 4), and zeroed group counters.  Neither depends on the cache, so
+// with programmatic launch this kernel runs while the kernel before it
+// (normally the cache append) finishes; it waits for that kernel before
+// exiting, so the stream kernel, which waits for this one, sees the finished
+// cache.
+template <typename T, int DD>
+__global__ void __launch_bounds__(kPrepThreads) decode_prep_kernel(DecodeArgs a)
+{
+    constexpr int QR = DD > 32 ? 2 : 1;  // q~ entries per lane
+    constexpr int kWarps = kPrepThreads / 32;
+    sm100::grid_dep_launch();  // the stream kernel may start its set-up now
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int rows = a.B * a.Hq;
+    for (int row = blockIdx.x * kWarps + warp; row < rows; row += gridDim.x * kWarps) {
+        const T *qrow = static_cast<const T *>(a.q) + (size_t)row * kHeadDim;
+        const float q0 = to_f32(qrow[lane]), q1 = to_f32(qrow[lane + 32]);
+        const int g = (row % a.Hq) / a.G;
+#pragma unroll
+        for (int rr = 0; rr < QR; ++rr) {
+            const int c = lane + 32 * rr;
+            const float4 *u4 = reinterpret_cast<const float4 *>(a.Uk + ((size_t)g * DD + (c < DD ? c : 0)) * kHeadDim);
+            float4 uk[kHeadDim / 4];
+#pragma unroll
+            for (int t4 = 0; t4 < kHeadDim / 4; ++t4)
+                uk[t4] = c < DD ? __ldg(u4 + t4) : make_float4(0.f, 0.f, 0.f, 0.f);
+            float p[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int t4 = 0; t4 < kHeadDim / 4; ++t4) {
+                const float uu[4] = {uk[t4].x, uk[t4].y, uk[t4].z, uk[t4].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int t = 4 * t4 + e;
+                    const float qv = __shfl_sync(0xffffffffu, t < 32 ? q0 : q1, t & 31);
+                    p[e] = fmaf(qv, uu[e], p[e]);
+                }
+            }
+            if (c < DD)
+                a.qt[(size_t)row * DD + c] = (p[0] + p[1]) + (p[2] + p[3]);
+        }
+    }
+    const int ngroups = a.B * a.Hkv * a.HS;
+    for (int i = blockIdx.x * kPrepThreads + threadIdx.x; i < ngroups; i += gridDim.x * kPrepThreads)
+        a.counters[i] = 0;
+    sm100::grid_dep_wait();
+}
+
+// --------------------------------------------------------------------- stream
+
+// Byte offset of 16-byte chunk `ch` of token t in a stage tile of ROW-element
+// bf16 rows as the 2-D TMA wrote it: the tile is viewed as 128-byte lines
+// (64 / ROW tokens per line) with the 128-byte swizzle, i.e. the chunk index
+// within a line XOR (line % 8).  Eight consecutive tokens of one chunk column
+// then fall in eight different bank groups (conflict-free ldmatrix).
+template <int ROW>
+__device__ __forceinline__ uint32_t tile_off(int t, int ch)
+{
+    constexpr int TR = kHeadDim / ROW;  // tokens per 128-byte line
+    const int line = t / TR;
+    const int c = (t % TR) * (ROW / 8) + ch;
+    return (uint32_t)(line * 128 + ((c ^ (line & 7)) << 4));
+}
+
+// Zero the value rows of a stage that the softmax masks out (tokens past the
+// stage's end, pages not copied): their P entries are zero, but stale or
+// never-written bytes there could be Inf/NaN and 0 * NaN would reach acc.
+// The fence orders these generic writes before the TMA that refills the slot.
+template <int ROW, int TPS>
+__device__ __forceinline__ void zero_masked_rows(unsigned char *v, int ntok, unsigned pmask, int lane)
+{
+    constexpr int CH = ROW / 8;  // 16-byte chunks per token
+#pragma unroll 4
+    for (int i = lane; i < TPS * CH; i += 32) {
+        const int t = i / CH;
+        if (!(t < ntok && ((pmask >> (t / kPage)) & 1u)))
+            *reinterpret_cast<uint4 *>(v + tile_off<ROW>(t, i % CH)) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    sm100::fence_proxy_async_smem();
+    __syncwarp();
+}
 
 // Tensor-core consumer for one stage of ROW-wide rows (64 = ring keys/values,
-// d_down = pages), TPS tokens, rows swizzled as the 2-D TMA wrote them.
+// d_down = pages), TPS tokens, laid out as tile_off<ROW> describes.
 // q_a: A fragments (KS k-steps) of the GH query rows; o: output fragments
 // (ROW/8 n-tiles); m, lpart: the row's running max and this lane's part of the
-// running sum (quad-uniform m).
-template <int ROW, int TPS, int GH>
+// running sum (quad-uniform m).  kMasked: some tokens of the stage are invalid.
+template <int ROW, int TPS, int GH, bool kMasked>
 __device__ __forceinline__ void mma_stage(uint32_t sK, uint32_t sV, int ntok, unsigned pmask,
                                           const uint32_t (&q_a)[(ROW >= 16 ? ROW / 16 : 1)][4],
                                           float (&o)[ROW / 8][4], float &m, float &lpart, float c2, int lane)
 {
-    constexpr int KS = ROW / 16;   // k-steps of the score product
-    constexpr int ND = ROW / 8;    // n-tiles of the output
-    constexpr int RB = ROW * 2;    // bytes per row
-    constexpr int SWM = RB / 16 - 1;
+    constexpr int KS = ROW / 16;  // k-steps of the score product
+    constexpr int ND = ROW / 8;   // n-tiles of the output
     constexpr int TB = TPS < 64 ? TPS : 64;  // tokens per block of the online softmax
     constexpr int NT = TB / 8;
-    const int g = lane >> 2, c = lane & 3;
+    const int c = lane & 3;
     const int mi = lane >> 3, ri = lane & 7;
-    auto swz = [](int t) { return ((t * RB) >> 7) & SWM; };
 #pragma unroll 1
     for (int t0 = 0; t0 < TPS; t0 += TB) {
         // ---- scores S[g][token] = q . k  for TB tokens
@@ -180,7 +237,7 @@ __device__ __forceinline__ void mma_stage(uint32_t sK, uint32_t sV, int ntok, un
                 const int tok = t0 + 8 * (2 * np + (mi >> 1)) + ri;
                 const int ch = 2 * ks + (mi & 1);
                 uint32_t r[4];
-                ldsm_x4(sK + tok * RB + ((ch ^ swz(tok)) << 4), r);
+                ldsm_x4(sK + tile_off<ROW>(tok, ch), r);
                 mma_bf16_16816(sc[2 * np], q_a[ks], r[0], r[1]);
                 mma_bf16_16816(sc[2 * np + 1], q_a[ks], r[2], r[3]);
             }
@@ -191,9 +248,11 @@ __device__ __forceinline__ void mma_stage(uint32_t sK, uint32_t sV, int ntok, un
         for (int n = 0; n < NT; ++n) {
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-                const int tl = t0 + 8 * n + 2 * c + e;
-                const bool ok = tl < ntok && ((pmask >> (tl / kPage)) & 1u);
-                sc[n][e] = ok ? sc[n][e] : -INFINITY;
+                if constexpr (kMasked) {
+                    const int tl = t0 + 8 * n + 2 * c + e;
+                    const bool ok = tl < ntok && ((pmask >> (tl / kPage)) & 1u);
+                    sc[n][e] = ok ? sc[n][e] : -INFINITY;
+                }
                 mx = fmaxf(mx, sc[n][e]);
             }
         }
@@ -228,12 +287,304 @@ __device__ __forceinline__ void mma_stage(uint32_t sK, uint32_t sV, int ntok, un
             for (int dp = 0; dp < ND / 2; ++dp) {
                 const int ch = 2 * dp + (mi >> 1);
                 uint32_t r[4];
-                ldsm_x4_t(sV + tok * RB + ((ch ^ swz(tok)) << 4), r);
+                ldsm_x4_t(sV + tile_off<ROW>(tok, ch), r);
                 mma_bf16_16816(o[2 * dp], pa, r[0], r[1]);
                 mma_bf16_16816(o[2 * dp + 1], pa, r[2], r[3]);
             }
         }
     }
+}
+
+// CUDA-core consumer for one page stage when a KV head serves one query head
+// (the tensor-core tile would carry 15 idle rows): lane l owns tokens
+// l, l + 32, ...; qd is q~ scaled to the log2 domain; m is the warp's running
+// max, l and o this lane's parts of the running sum and value accumulator.
+// Masked tokens never touch o, so their rows may hold anything.
+template <int DD, int TPS>
+__device__ __forceinline__ void lane_stage(uint32_t sK, uint32_t sV, int ntok, unsigned pmask, const float (&qd)[DD],
+                                           float (&o)[DD], float &m, float &l, int lane)
+{
+    constexpr int TPL = TPS / 32;  // tokens per lane
+    constexpr int CH = DD / 8;     // 16-byte chunks per row
+    static_assert(TPS % 32 == 0, "whole tokens per lane");
+    float sc[TPL];
+    bool ok[TPL];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < TPL; ++i) {
+        const int t = lane + 32 * i;
+        ok[i] = t < ntok && ((pmask >> (t / kPage)) & 1u);
+        float acc = 0.f;
+#pragma unroll
+        for (int ch = 0; ch < CH; ++ch) {
+            uint4 k4;
+            asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                         : "=r"(k4.x), "=r"(k4.y), "=r"(k4.z), "=r"(k4.w)
+                         : "r"(sK + tile_off<DD>(t, ch)));
+            float kf[8];
+            unpack(k4, kf, bf16());
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                acc = fmaf(qd[8 * ch + e], kf[e], acc);
+        }
+        sc[i] = ok[i] ? acc : -INFINITY;
+        mx = fmaxf(mx, sc[i]);
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1)
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    if (mx > m) {  // warp-uniform: rescale only when the running max grows
+        const float alpha = m == -INFINITY ? 0.f : sm100::ex2_approx(m - mx);
+        l *= alpha;
+#pragma unroll
+        for (int c = 0; c < DD; ++c)
+            o[c] *= alpha;
+        m = mx;
+    }
+#pragma unroll
+    for (int i = 0; i < TPL; ++i) {
+        if (!ok[i])
+            continue;
+        const int t = lane + 32 * i;
+        const float p = sm100::ex2_approx(sc[i] - m);
+        l += p;
+#pragma unroll
+        for (int ch = 0; ch < CH; ++ch) {
+            uint4 v4;
+            asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                         : "=r"(v4.x), "=r"(v4.y), "=r"(v4.z), "=r"(v4.w)
+                         : "r"(sV + tile_off<DD>(t, ch)));
+            float vf[8];
+            unpack(v4, vf, bf16());
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                o[8 * ch + e] = fmaf(p, vf[e], o[8 * ch + e]);
+        }
+    }
+}
+
+// One halving step of a warp reduce-scatter: lanes with `mask` set keep the
+// upper half of their values, the others the lower half, each adding its
+// partner's copy of the half it keeps.
+template <int N>
+__device__ __forceinline__ void rs_step(const float (&in)[N], float (&out)[N / 2], int mask, int lane)
+{
+    const bool upper = (lane & mask) != 0;
+#pragma unroll
+    for (int j = 0; j < N / 2; ++j) {
+        const float send = upper ? in[j] : in[j + N / 2];
+        const float keep = upper ? in[j + N / 2] : in[j];
+        out[j] = keep + __shfl_xor_sync(0xffffffffu, send, mask);
+    }
+}
+
+// Warp sum of o[0..DD) (DD = 16 or 32): returns the total of entry
+// lane / (32 / DD), held by 32 / DD lanes each.
+template <int DD>
+__device__ __forceinline__ float reduce_scatter(const float (&o)[DD], int lane)
+{
+    float a16[16], a8[8], a4[4], a2[2], a1[1];
+    if constexpr (DD == 32) {
+        rs_step<32>(o, a16, 16, lane);
+        rs_step<16>(a16, a8, 8, lane);
+        rs_step<8>(a8, a4, 4, lane);
+        rs_step<4>(a4, a2, 2, lane);
+        rs_step<2>(a2, a1, 1, lane);
+        return a1[0];
+    } else {
+        static_assert(DD == 16, "reduce_scatter handles 16 or 32 values");
+        rs_step<16>(o, a8, 16, lane);
+        rs_step<8>(a8, a4, 8, lane);
+        rs_step<4>(a4, a2, 4, lane);
+        rs_step<2>(a2, a1, 2, lane);
+        return a1[0] + __shfl_xor_sync(0xffffffffu, a1[0], 1);
+    }
+}
+
+// Per-sequence tables of one decode call, built by every CTA of the stream
+// kernel into its shared memory (kSeqPerThread sequences per thread, one
+// block-wide scan): s_len[b] = validated length (-1 if beyond the cache's
+// capacity), s_pre[b] = chunks of the sequences before b (s_pre[B] = all),
+// and the chunk sizes (cw, cd) = f * (minimum sizes), f chosen so that the
+// grid gets about kItemsPerWarp items per warp.  Larger chunks only lower the
+// chunk counts, so the workspace sized for the minimum chunks always fits.
+constexpr int kSeqPerThread = DAR_DECODE_MAX_BATCH / kDecThreads;
+
+__device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, int *s_len, long long *s_red,
+                                             int *s_scan, int *s_f)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int B = a.B, w = a.w;
+    int Ls[kSeqPerThread];
+#pragma unroll
+    for (int k = 0; k < kSeqPerThread; ++k) {
+        const int b = threadIdx.x * kSeqPerThread + k;
+        Ls[k] = b < B ? a.seq_lens[b] : 0;
+    }
+    long long units = 0;
+#pragma unroll
+    for (int k = 0; k < kSeqPerThread; ++k) {
+        const int b = threadIdx.x * kSeqPerThread + k;
+        int L = Ls[k];
+        if (b < B && (L < 0 || (long long)L - w > (long long)a.maxp * kPage)) {
+            if (blockIdx.x == 0)
+                report(a.status, DAR_ERR_CAPACITY);
+            L = -1;
+        }
+        Ls[k] = L;
+        if (b < B)
+            s_len[b] = L;
+        const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
+        units += (nwin + a.cw - 1) / a.cw + (ndist + a.cd - 1) / a.cd;
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1)
+        units += __shfl_xor_sync(0xffffffffu, units, off);
+    if (lane == 0)
+        s_red[warp] = units;
+    __syncthreads();
+    if (warp == 0) {
+        units = lane < kDecWarps ? s_red[lane] : 0;
+#pragma unroll
+        for (int off = 16; off; off >>= 1)
+            units += __shfl_xor_sync(0xffffffffu, units, off);
+        if (lane == 0) {
+            const long long target = (long long)gridDim.x * kDecWarps * kItemsPerWarp;
+            long long f = (units * a.Hkv * a.HS + target - 1) / target;
+            const long long fmax = (long long)(64 * kPage) / a.cd;  // a page chunk spans at most 64 pages
+            f = f > fmax ? fmax : f;
+            f = f > kMaxChunkScale ? kMaxChunkScale : f;
+            *s_f = f < 1 ? 1 : (int)f;
+        }
+    }
+    __syncthreads();
+    const int cw = a.cw * *s_f, cd = a.cd * *s_f;
+    int cnt[kSeqPerThread], mine = 0;
+#pragma unroll
+    for (int k = 0; k < kSeqPerThread; ++k) {
+        const int L = Ls[k];
+        const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
+        cnt[k] = (nwin + cw - 1) / cw + (ndist + cd - 1) / cd;
+        mine += cnt[k];
+    }
+    int incl = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off)
+            incl += y;
+    }
+    if (lane == 31)
+        s_scan[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int v = lane < kDecWarps ? s_scan[lane] : 0;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, v, off);
+            if (lane >= off)
+                v += y;
+        }
+        if (lane < kDecWarps)
+            s_scan[lane] = v;  // inclusive over warps
+    }
+    __syncthreads();
+    int run = incl - mine + (warp > 0 ? s_scan[warp - 1] : 0);
+#pragma unroll
+    for (int k = 0; k < kSeqPerThread; ++k) {
+        const int b = threadIdx.x * kSeqPerThread + k;
+        if (b < B)
+            s_pre[b] = run;
+        run += cnt[k];
+    }
+    if (threadIdx.x == kDecThreads - 1)
+        s_pre[B] = run;  // all chunks
+    __syncthreads();
+    return make_int2(cw, cd);
+}
+
+// One (b, h) output row from its chunk records, by one warp:
+// o = (sum_c f_c acc_c[local] + (sum_c f_c acc_c[global]) Uv) / sum_c f_c l_c,
+// f_c = 2^(m_c - max m) (Eq. 4: one softmax over all chunks).  Lane j holds
+// chunk j's (m, l); lane i holds entries 2i, 2i+1 of every chunk's acc.  The
+// loads of the first kCombChunks chunks are issued together.
+constexpr int kCombChunks = 32;
+
+template <typename T, int DD>
+__device__ __forceinline__ void combine_row(const DecodeArgs &a, int b, int h, int g, int nwc, int nch, int lane)
+{
+    const size_t rec0 = ((size_t)b * a.Hq + h) * a.maxc;
+    const int jmax = min(nch, kCombChunks);
+    float mj = -INFINITY, lj = 0.f;
+    if (lane < jmax) {
+        mj = __ldcg(a.rec_m + rec0 + lane);
+        lj = __ldcg(a.rec_l + rec0 + lane);
+    }
+    float2 av[kCombChunks];
+#pragma unroll
+    for (int j = 0; j < kCombChunks; ++j)
+        av[j] = j < jmax ? __ldcg(reinterpret_cast<const float2 *>(a.rec_acc + (rec0 + j) * kHeadDim) + lane)
+                         : make_float2(0.f, 0.f);
+    // entries past a page chunk's d_down values are never combined: they may hold anything
+    float M = mj;
+    for (int c0 = kCombChunks; c0 < nch; c0 += 32)
+        if (c0 + lane < nch)
+            M = fmaxf(M, __ldcg(a.rec_m + rec0 + c0 + lane));
+#pragma unroll
+    for (int off = 16; off; off >>= 1)
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float o0 = 0.f, o1 = 0.f, gd0 = 0.f, gd1 = 0.f;
+    const float f0 = lane < jmax ? exp2f(mj - M) : 0.f;
+    float lsum = f0 * lj;
+#pragma unroll
+    for (int j = 0; j < kCombChunks; ++j) {
+        const float fj = __shfl_sync(0xffffffffu, f0, j);
+        if (j < jmax) {
+            if (j < nwc) {
+                o0 = fmaf(fj, av[j].x, o0);
+                o1 = fmaf(fj, av[j].y, o1);
+            } else if (2 * lane < DD) {
+                gd0 = fmaf(fj, av[j].x, gd0);
+                gd1 = fmaf(fj, av[j].y, gd1);
+            }
+        }
+    }
+    for (int c0 = kCombChunks; c0 < nch; c0 += 32) {  // long sequences with small chunks
+        float f = 0.f;
+        if (c0 + lane < nch) {
+            f = exp2f(__ldcg(a.rec_m + rec0 + c0 + lane) - M);
+            lsum = fmaf(f, __ldcg(a.rec_l + rec0 + c0 + lane), lsum);
+        }
+        const int jn = min(32, nch - c0);
+        for (int j = 0; j < jn; ++j) {
+            const float fj = __shfl_sync(0xffffffffu, f, j);
+            const int cc = c0 + j;
+            const float2 v = __ldcg(reinterpret_cast<const float2 *>(a.rec_acc + (rec0 + cc) * kHeadDim) + lane);
+            if (cc < nwc) {
+                o0 = fmaf(fj, v.x, o0);
+                o1 = fmaf(fj, v.y, o1);
+            } else if (2 * lane < DD) {
+                gd0 = fmaf(fj, v.x, gd0);
+                gd1 = fmaf(fj, v.y, gd1);
+            }
+        }
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1)
+        lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+    // lift the global part once: o += gd Uv[g]   (gd[c] sits in lane c / 2)
+    const float *Uv = a.Uv + (size_t)g * DD * kHeadDim;
+#pragma unroll
+    for (int cc = 0; cc < DD; ++cc) {
+        const float gv = __shfl_sync(0xffffffffu, (cc & 1) ? gd1 : gd0, cc >> 1);
+        const float2 u2 = __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
+        o0 = fmaf(gv, u2.x, o0);
+        o1 = fmaf(gv, u2.y, o1);
+    }
+    const float inv = 1.f / lsum;
+    T *orow = static_cast<T *>(a.out) + ((size_t)b * a.Hq + h) * kHeadDim;
+    orow[2 * lane] = from_f32<T>(o0 * inv);
+    orow[2 * lane + 1] = from_f32<T>(o1 * inv);
 }
 
 template <typename T, int DD, int GH>
@@ -245,113 +596,64 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     constexpr int E = Granule<T>::kElems;
     constexpr int ES = sizeof(T);
     constexpr bool kMma = decode_uses_mma<T, DD>();
-    constexpr int TPS_W = kHalf / (kHeadDim * ES);           // tokens per ring stage
-    constexpr int TPS_D = kHalf / (DD * ES);                 // tokens per page stage
+    constexpr int TPS_W = tps_ring<T>();
+    constexpr int TPS_D = tps_page<T, DD>();
     constexpr int PPS = TPS_D >= kPage ? TPS_D / kPage : 1;  // pages touched per stage
+    constexpr unsigned kFullPages = (1u << PPS) - 1u;
     static_assert(TPS_D % kPage == 0 || kPage % TPS_D == 0, "stages must tile pages");
     static_assert(PPS <= 8, "stage page mask holds 8 pages");
+    static_assert(GH * kHeadDim * ES <= kHdrBytes && GH * DD * 4 <= kHdrBytes, "header holds the query rows");
+    // one query head per KV head: page stages on the CUDA cores, one token per lane
+    constexpr bool kLanePages = kMma && GH == 1 && DD == 16;
 
     extern __shared__ __align__(128) unsigned char smem_raw[];
     // swizzled TMA tiles need 1024-byte alignment (static shared data may precede this)
     unsigned char *slots = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));  // [warps][stages][slot]
-    uint64_t *bars = reinterpret_cast<uint64_t *>(slots + (size_t)kDecWarps * kStages * kSlotBytes);
-    int *meta = reinterpret_cast<int *>(bars + kDecWarps * kStages);  // [warps][stages][2]
-    WarpSmem<GH> *wsm = reinterpret_cast<WarpSmem<GH> *>(meta + kDecWarps * kStages * 2);
-    int *s_pre = reinterpret_cast<int *>(wsm + kDecWarps);
-    int *s_len = s_pre + a.B + 1;
-    __shared__ int s_geo[2];  // chunk sizes of this launch
+    unsigned char *hdrs = slots + (size_t)kDecWarps * kStages * kSlotBytes;  // [warps][stages][header]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(hdrs + (size_t)kDecWarps * kStages * kHdrBytes);
+    int4 *meta = reinterpret_cast<int4 *>(bars + kDecWarps * kStages);
+    int *s_pre = reinterpret_cast<int *>(meta + kDecWarps * kStages);  // [B + 1]
+    int *s_len = s_pre + a.B + 1;                                      // [B]
+    __shared__ long long s_red[kDecWarps];
+    __shared__ int s_scan[kDecWarps], s_f;
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int B = a.B, w = a.w;
-
-    if (threadIdx.x < kDecWarps * kStages)
-        mbar_init(&bars[threadIdx.x], 1);
-    if (blockIdx.x == 0) {  // warm L2 with the small tables every CTA reads first
-        for (int i = threadIdx.x * 32; i < B; i += kDecThreads * 32)
-            asm volatile("prefetch.global.L2 [%0];" ::"l"(a.seq_lens + i));
-    }
-    // ---- chunk sizes and counts (warp 0).  The host sized the workspace for the
-    // minimum chunks (a.cw, a.cd); the launch scales both by one factor f so that
-    // the number of items is about the number of warps (one long stream per
-    // warp).  Larger chunks only lower the chunk count, so records still fit.
-    if (warp == 0) {
-        const int per = (B + 31) / 32;
-        const int lo = min(B, lane * per), hi = min(B, lo + per);
-        long long units = 0;
-        for (int b = lo; b < hi; ++b) {
-            int L = a.seq_lens[b];
-            if (L < 0 || (long long)L - w > (long long)a.maxp * kPage)
-                L = -1;
-            s_len[b] = L;
-            if (L > 0) {
-                const int nwin = min(L, w), ndist = L - nwin;
-                units += (nwin + a.cw - 1) / a.cw + (ndist + a.cd - 1) / a.cd;
-            }
-        }
-#pragma unroll
-        for (int off = 16; off; off >>= 1)
-            units += __shfl_xor_sync(0xffffffffu, units, off);
-        const long long target = (long long)gridDim.x * kDecWarps * kItemsPerWarp;
-        long long f = (units * a.Hkv * a.HS + target - 1) / target;
-        const long long fmax = (long long)(64 * kPage) / a.cd;  // an item spans at most 64 pages
-        f = f > fmax ? fmax : f;
-        f = f > kMaxChunkScale ? kMaxChunkScale : f;
-        f = f < 1 ? 1 : f;
-        const int cw = a.cw * (int)f, cd = a.cd * (int)f;
-        int run = 0;
-        for (int b = lo; b < hi; ++b) {
-            const int L = s_len[b];
-            int cnt = 0;
-            if (L > 0) {
-                const int nwin = min(L, w), ndist = L - nwin;
-                cnt = (nwin + cw - 1) / cw + (ndist + cd - 1) / cd;
-            }
-            s_pre[b] = cnt;
-            run += cnt;
-        }
-        int incl = run;
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, off);
-            if (lane >= off)
-                incl += y;
-        }
-        int base = incl - run;
-        for (int b = lo; b < hi; ++b) {
-            const int cnt = s_pre[b];
-            s_pre[b] = base;
-            base += cnt;
-        }
-        if (lane == 31) {
-            s_pre[B] = incl;
-            s_geo[0] = cw;
-            s_geo[1] = cd;
-        }
-    }
+    unsigned char *my_slots = slots + (size_t)warp * kStages * kSlotBytes;
+    unsigned char *my_hdrs = hdrs + (size_t)warp * kStages * kHdrBytes;
+    uint64_t *my_bars = bars + warp * kStages;
+    int4 *my_meta = meta + warp * kStages;
+    __shared__ int s_next;  // this CTA's item counter
+    if (lane < kStages)
+        mbar_init(&my_bars[lane], 1);
+    if (threadIdx.x == 0)
+        s_next = 0;
     sm100::mbar_init_fence();
     __syncthreads();
-
-    // sequences with nothing to attend to get a zero output
-    if (blockIdx.x == 0) {
+    if constexpr (kMma) {
+        if (threadIdx.x == 0) {
+            sm100::prefetch_tensormap(&tm_wk);
+            sm100::prefetch_tensormap(&tm_wv);
+            sm100::prefetch_tensormap(&tm_pk);
+            sm100::prefetch_tensormap(&tm_pv);
+        }
+    }
+    // everything below reads the cache and q~ (the prep kernel waited for the
+    // kernel before it, so both are final)
+    sm100::grid_dep_wait();
+    const int2 chunk = build_tables(a, s_pre, s_len, s_red, s_scan, &s_f);
+    const int cw = chunk.x, cd = chunk.y;
+    if (blockIdx.x == 0) {  // sequences with nothing to attend to get a zero output
         T *out = static_cast<T *>(a.out);
-        for (int b = warp; b < B; b += kDecWarps) {
+        for (int b = warp; b < a.B; b += kDecWarps) {
             if (s_len[b] > 0)
                 continue;
-            if (s_len[b] < 0 && lane == 0)
-                report(a.status, DAR_ERR_CAPACITY);
             for (int i = lane; i < a.Hq * kHeadDim; i += 32)
                 out[(size_t)b * a.Hq * kHeadDim + i] = from_f32<T>(0.f);
         }
     }
 
-    const SeqTables tabs{s_pre, s_len, s_geo[0], s_geo[1]};
-    const int items = s_pre[B] * a.Hkv * a.HS;
-    const int nwarps_total = gridDim.x * kDecWarps;
-    unsigned char *my_slots = slots + (size_t)warp * kStages * kSlotBytes;
-    uint64_t *my_bars = bars + warp * kStages;
-    int *my_meta = meta + warp * kStages * 2;
-    WarpSmem<GH> &sc = wsm[warp];
+    const int w = a.w;
     const T *qg = static_cast<const T *>(a.q);
     const T *wk = static_cast<const T *>(a.win_k);
     const T *wv = static_cast<const T *>(a.win_v);
@@ -359,44 +661,79 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     const T *pv = static_cast<const T *>(a.pool_vd);
     bool alive = true;
 
-    // ---- issue side.  Item indices come from the counter one item ahead; the
-    // page ids of the item being copied in and of the next one are held in
-    // registers (lane j: pages j and 32 + j of the item).
-    const int gw = blockIdx.x + gridDim.x * warp;
-    // The counter hands out items from 2 * nwarps on (the first two per warp are
-    // static).  Lane 0 keeps the fetched index unread until the following item
-    // switch, so the atomic's round trip overlaps a whole item.
-    auto fetch_index = [&]() {
+    // ---- issue side.  Items are ordered by sequence, then (KV head, slice)
+    // group, then chunk; CTA k owns the contiguous range [lo, hi) and hands it
+    // to its warps in order from a shared-memory counter.  An item is decoded
+    // from the tables; the block-table ids of its pages are loaded two items
+    // before they are used (`iss` is being copied in, `nxt` and `nn` follow).
+    const int per_chunk = a.Hkv * a.HS;
+    const int items = s_pre[a.B] * per_chunk;
+    const int lo = (int)((long long)blockIdx.x * items / gridDim.x);
+    const int hi = (int)((long long)(blockIdx.x + 1) * items / gridDim.x);
+    auto seq_of = [&](int it) {  // the sequence whose items include `it`
+        int lb = 0, hb = a.B;
+        while (hb - lb > 1) {
+            const int mid = (lb + hb) >> 1;
+            if (s_pre[mid] * per_chunk <= it)
+                lb = mid;
+            else
+                hb = mid;
+        }
+        return lb;
+    };
+    auto fetch_item = [&](int it) {
+        Item I;
+        I.it = -1;
+        I.b = I.g = I.h0 = I.window = I.t0 = I.t1 = I.nst = I.rec0 = 0;
+        I.pid = make_int2(-1, -1);
+        if (it < hi) {
+            const int b = seq_of(it);
+            const int nch = s_pre[b + 1] - s_pre[b];
+            const int r = it - s_pre[b] * per_chunk;
+            const int gh = r / nch, c = r % nch;
+            const int L = s_len[b], nwin = min(L, w), ndist = L - nwin;
+            const int nwc = (nwin + cw - 1) / cw;
+            I.it = it;
+            I.b = b;
+            I.g = gh / a.HS;
+            I.h0 = I.g * a.G + (gh % a.HS) * a.GH;
+            if (c < nwc) {
+                I.window = 1;
+                I.t0 = c * cw;
+                I.t1 = min(nwin, I.t0 + cw);
+                I.nst = (I.t1 - I.t0 + TPS_W - 1) / TPS_W;
+            } else {
+                I.t0 = (c - nwc) * cd;
+                I.t1 = min(ndist, I.t0 + cd);
+                I.nst = (I.t1 - I.t0 + TPS_D - 1) / TPS_D;
+                const int p0 = I.t0 / kPage, np = (I.t1 - 1) / kPage - p0 + 1;
+                const int32_t *bt = a.block_table + (size_t)b * a.maxp + p0;
+                if (lane < np)
+                    I.pid.x = __ldg(bt + lane);
+                if (lane + 32 < np)
+                    I.pid.y = __ldg(bt + lane + 32);
+            }
+            I.rec0 = (b * a.Hq + I.h0) * a.maxc + c;
+        }
+        return I;
+    };
+    auto next_index = [&]() {
         int v = 0;
         if (lane == 0)
-            v = atomicAdd(a.sched, 1) + 2 * nwarps_total;
-        return v;
+            v = lo + atomicAdd(&s_next, 1);
+        return __shfl_sync(0xffffffffu, v, 0);
     };
-    auto use_index = [&](int v) { return __shfl_sync(0xffffffffu, v, 0); };
-    auto load_pages = [&](const Item &I) {
-        int2 id = make_int2(-1, -1);
-        if (I.it >= 0 && !I.window) {
-            const int p0 = I.t0 / kPage, np = (I.t1 - 1) / kPage - p0 + 1;
-            const int32_t *row = a.block_table + (size_t)I.b * a.maxp + p0;
-            if (lane < np)
-                id.x = row[lane];
-            if (lane + 32 < np)
-                id.y = row[lane + 32];
-        }
-        return id;
-    };
-    Item iss = decode_item<TPS_W, TPS_D>(gw, items, a, tabs);
-    int2 iss_pid = load_pages(iss);
-    Item nxt = decode_item<TPS_W, TPS_D>(gw + nwarps_total, items, a, tabs);
-    int2 nxt_pid = load_pages(nxt);
-    int pending_raw = nxt.it >= 0 ? fetch_index() : items;  // lane 0: the item after `nxt`
+    Item iss = fetch_item(next_index());
+    Item nxt = iss.it >= 0 ? fetch_item(next_index()) : fetch_item(hi);
+    Item nn = nxt.it >= 0 ? fetch_item(next_index()) : fetch_item(hi);
+
     int iss_s = 0;
-    int issued = 0, consumed = 0;               // stages issued / consumed by this warp
-    int iss_slot = 0, con_slot = 0;             // ring positions
-    unsigned con_phase = 0;                     // parity of the consumer's current pass over the ring
-    auto page_id = [&](int j) {  // page j (0..63) of the item being issued
-        const int x = __shfl_sync(0xffffffffu, iss_pid.x, j & 31);
-        const int y = __shfl_sync(0xffffffffu, iss_pid.y, j & 31);
+    int issued = 0, consumed = 0;    // stages issued / consumed by this warp
+    int iss_slot = 0, con_slot = 0;  // ring positions
+    unsigned con_phase = 0;          // parity of the consumer's current pass over the ring
+    auto page_id = [&](int j) {      // page j (0..63) of the item being issued
+        const int x = __shfl_sync(0xffffffffu, iss.pid.x, j & 31);
+        const int y = __shfl_sync(0xffffffffu, iss.pid.y, j & 31);
         return j < 32 ? x : y;
     };
 
@@ -406,35 +743,50 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         unsigned char *dst = my_slots + (size_t)slot * kSlotBytes;
         uint64_t *bar = &my_bars[slot];
         const int s = iss_s;
+        const int info = s | (s + 1 == iss.nst ? kMetaLast : 0);
+        // the item's query rows travel with its first stage
+        unsigned hdr_bytes = 0;
+        const void *hsrc = nullptr;
+        if (s == 0) {
+            if (iss.window) {
+                hdr_bytes = GH * kHeadDim * ES;
+                hsrc = qg + ((size_t)iss.b * a.Hq + iss.h0) * kHeadDim;
+            } else {
+                hdr_bytes = GH * DD * 4;
+                hsrc = a.qt + ((size_t)iss.b * a.Hq + iss.h0) * DD;
+            }
+        }
         if (iss.window) {
             const int tb = iss.t0 + s * TPS_W, te = min(iss.t1, tb + TPS_W);
             if (lane == 0) {
-                my_meta[slot * 2 + 0] = iss.it;
-                my_meta[slot * 2 + 1] = (s << 8) | 0xff;
+                my_meta[slot] = make_int4(iss.rec0, info | kMetaRing | (0xff << 24), te - tb, 0);
+                const int y = (iss.b * a.Hkv + iss.g) * w + tb;
                 if constexpr (kMma) {  // whole boxes of TPS_W rows, 128-byte swizzle
-                    const int y = (iss.b * a.Hkv + iss.g) * w + tb;
-                    mbar_expect_tx(bar, 2 * TPS_W * kHeadDim * ES);
+                    mbar_expect_tx(bar, 2 * TPS_W * kHeadDim * ES + hdr_bytes);
                     sm100::tma_load_2d_u(smem_u32(dst), &tm_wk, 0, y, bar);
                     sm100::tma_load_2d_u(smem_u32(dst + kHalf), &tm_wv, 0, y, bar);
                 } else {
                     const unsigned bytes = (unsigned)(te - tb) * kHeadDim * ES;
-                    const size_t off = ((size_t)(iss.b * a.Hkv + iss.g) * w + tb) * kHeadDim;
-                    mbar_expect_tx(bar, 2 * bytes);
+                    const size_t off = (size_t)y * kHeadDim;
+                    mbar_expect_tx(bar, 2 * bytes + hdr_bytes);
                     bulk_g2s(dst, wk + off, bytes, bar);
                     bulk_g2s(dst + kHalf, wv + off, bytes, bar);
                 }
+                if (hdr_bytes)
+                    bulk_g2s(my_hdrs + slot * kHdrBytes, hsrc, hdr_bytes, bar);
             }
         } else {
             const int tb = iss.t0 + s * TPS_D, te = min(iss.t1, tb + TPS_D);
             const int pfirst = tb / kPage - iss.t0 / kPage;  // index within the item's pages
+            int id[PPS];
             unsigned mask = 0, total = 0;
 #pragma unroll
             for (int j = 0; j < PPS; ++j) {
-                const int id = page_id(pfirst + j);
+                id[j] = page_id(pfirst + j);
                 const int ptb = max(tb, (tb / kPage + j) * kPage);
                 const int pte = min(te, (tb / kPage + j + 1) * kPage);
                 if (pte > ptb) {
-                    if (id >= 0 && id < a.num_pages) {
+                    if (id[j] >= 0 && id[j] < a.num_pages) {
                         mask |= 1u << j;
                         // the 2-D path copies whole boxes of min(64, TPS_D) rows
                         total += (unsigned)(kMma ? (TPS_D < kPage ? TPS_D : kPage) : (pte - ptb)) * DD * ES;
@@ -444,64 +796,55 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                 }
             }
             if (lane == 0) {
-                my_meta[slot * 2 + 0] = iss.it;
-                my_meta[slot * 2 + 1] = (s << 8) | (int)mask;
-                mbar_expect_tx(bar, 2 * total);
-            }
+                my_meta[slot] = make_int4(iss.rec0, info | (int)(mask << 24), te - tb, 0);
+                mbar_expect_tx(bar, 2 * total + hdr_bytes);
 #pragma unroll
-            for (int j = 0; j < PPS; ++j) {
-                const int id = page_id(pfirst + j);
-                const int ptb = max(tb, (tb / kPage + j) * kPage);
-                const int pte = min(te, (tb / kPage + j + 1) * kPage);
-                if (lane == 0 && ((mask >> j) & 1u)) {
-                    const size_t doff = (size_t)(ptb - tb) * DD * ES;
-                    if constexpr (kMma) {
-                        const int y = (id * a.Hkv + iss.g) * kPage + (ptb % kPage);
-                        sm100::tma_load_2d_u(smem_u32(dst + doff), &tm_pk, 0, y, bar);
-                        sm100::tma_load_2d_u(smem_u32(dst + kHalf + doff), &tm_pv, 0, y, bar);
-                    } else {
-                        const unsigned bytes = (unsigned)(pte - ptb) * DD * ES;
-                        const size_t src = (((size_t)id * a.Hkv + iss.g) * kPage + (ptb % kPage)) * DD;
-                        bulk_g2s(dst + doff, pk + src, bytes, bar);
-                        bulk_g2s(dst + kHalf + doff, pv + src, bytes, bar);
+                for (int j = 0; j < PPS; ++j) {
+                    if ((mask >> j) & 1u) {
+                        const int ptb = max(tb, (tb / kPage + j) * kPage);
+                        const int pte = min(te, (tb / kPage + j + 1) * kPage);
+                        const size_t doff = (size_t)(ptb - tb) * DD * ES;
+                        if constexpr (kMma) {  // page (id, g) = DD lines of 128 bytes
+                            const int y = (id[j] * a.Hkv + iss.g) * DD + (ptb % kPage) * DD / kHeadDim;
+                            sm100::tma_load_2d_u(smem_u32(dst + doff), &tm_pk, 0, y, bar);
+                            sm100::tma_load_2d_u(smem_u32(dst + kHalf + doff), &tm_pv, 0, y, bar);
+                        } else {
+                            const unsigned bytes = (unsigned)(pte - ptb) * DD * ES;
+                            const size_t src = (((size_t)id[j] * a.Hkv + iss.g) * kPage + (ptb % kPage)) * DD;
+                            bulk_g2s(dst + doff, pk + src, bytes, bar);
+                            bulk_g2s(dst + kHalf + doff, pv + src, bytes, bar);
+                        }
                     }
                 }
+                if (hdr_bytes)
+                    bulk_g2s(my_hdrs + slot * kHdrBytes, hsrc, hdr_bytes, bar);
             }
         }
         __syncwarp();
         ++issued;
         if (++iss_s == iss.nst) {  // move on to the next item
             iss = nxt;
-            iss_pid = nxt_pid;
             iss_s = 0;
             if (iss.it >= 0) {
-                nxt = decode_item<TPS_W, TPS_D>(use_index(pending_raw), items, a, tabs);
-                nxt_pid = load_pages(nxt);
-                pending_raw = nxt.it >= 0 ? fetch_index() : items;
+                nxt = nn;
+                nn = nxt.it >= 0 ? fetch_item(next_index()) : fetch_item(hi);
             }
         }
     };
-    // Start from zeroed slots: a stage whose copies do not cover the whole slot
-    // (a short last page) leaves rows that are masked out but still enter the
-    // tensor-core products, so they must hold finite values.
-    {
-        uint4 *z = reinterpret_cast<uint4 *>(my_slots);
-        for (int i = lane; i < kStages * kSlotBytes / 16; i += 32)
-            z[i] = make_uint4(0, 0, 0, 0);
-        sm100::fence_proxy_async_smem();
-        __syncwarp();
-    }
     while (issued - consumed < kStages && iss.it >= 0)
         issue_one();
 
     // ---- consume side
-    Item cur = decode_item<TPS_W, TPS_D>(-1, 0, a, tabs);
-    // tensor-core consumer state: A fragments of q (ring) / q~ (pages), output
+    // tensor-core consumer state: A fragments of q (ring) or q~ (pages), output
     // fragments of row g = lane / 4 (query head h0 + g when g < GH)
     constexpr int KSD = DD >= 16 ? DD / 16 : 1;
+    constexpr int NDD = DD / 8 > 0 ? DD / 8 : 1;
     uint32_t qa_w[4][4], qa_d[KSD][4];
-    float ow[8][4], od[DD / 8 > 0 ? DD / 8 : 1][4];
+    float ow[8][4], od[NDD][4];
     float mm = -INFINITY, lp = 0.f;
+    // lane-per-token page consumer state (kLanePages)
+    float qd[kLanePages ? DD : 1], ol[kLanePages ? DD : 1];
+    // CUDA-core consumer state (per head of the slice)
     float m[GH], l[GH], acc[GH][E], qr[GH][E];
 #pragma unroll
     for (int k = 0; k < GH; ++k) {
@@ -519,93 +862,66 @@ __global__ void __launch_bounds__(kDecThreads, 1)
             break;
         }
         __syncwarp();
-        const int mit = my_meta[slot * 2 + 0];
-        const int minfo = my_meta[slot * 2 + 1];
-        const int s = minfo >> 8;
-        const unsigned pmask = (unsigned)(minfo & 0xff);
+        const int4 md = my_meta[slot];
+        const int s = md.y & 0xffff;
+        const bool win = (md.y & kMetaRing) != 0;
+        const bool last = (md.y & kMetaLast) != 0;
+        const unsigned pmask = ((unsigned)md.y >> 24) & 0xffu;
+        const int ntok = md.z;
+        const unsigned char *hdr = my_hdrs + slot * kHdrBytes;
         if (s == 0) {
-            // ---- new item: stage the queries (and q~ for the pages)
-            cur = decode_item<TPS_W, TPS_D>(mit, items, a, tabs);
-            const int h0 = cur.g * a.G + cur.hs * GH;
-            const bool pages = !cur.window;
-            const float *Ukg = a.Uk + (size_t)cur.g * DD * kHeadDim;
-            // issue this lane's first Uk row and the query rows together (one round trip)
-            float4 ur[kHeadDim / 4];
-            if (pages && lane < GH * DD) {
-                const float4 *src4 = reinterpret_cast<const float4 *>(Ukg + (size_t)(lane % DD) * kHeadDim);
-#pragma unroll
-                for (int t4 = 0; t4 < kHeadDim / 4; ++t4)
-                    ur[t4] = __ldg(src4 + t4);
-            }
-            const float qs = kMma ? 1.f : a.qscale;  // the tensor-core path scales the scores instead
-#pragma unroll
-            for (int k = 0; k < GH; ++k) {
-                const T *qrow = qg + ((size_t)cur.b * a.Hq + h0 + k) * kHeadDim;
-                sc.q[k][lane] = to_f32(qrow[lane]) * qs;
-                sc.q[k][lane + 32] = to_f32(qrow[lane + 32]) * qs;
-            }
-            __syncwarp();
-            if (pages) {
-                // q~[k][c] = sum_t q[k][t] Uk[g][c][t]
-                for (int o = lane; o < GH * DD; o += 32) {
-                    const int k = o / DD, cc = o % DD;
-                    if (o != lane) {
-                        const float4 *src4 = reinterpret_cast<const float4 *>(Ukg + (size_t)cc * kHeadDim);
-#pragma unroll
-                        for (int t4 = 0; t4 < kHeadDim / 4; ++t4)
-                            ur[t4] = __ldg(src4 + t4);
-                    }
-                    float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f;
-#pragma unroll
-                    for (int t4 = 0; t4 < kHeadDim / 4; ++t4) {
-                        p0 = fmaf(sc.q[k][4 * t4 + 0], ur[t4].x, p0);
-                        p1 = fmaf(sc.q[k][4 * t4 + 1], ur[t4].y, p1);
-                        p2 = fmaf(sc.q[k][4 * t4 + 2], ur[t4].z, p2);
-                        p3 = fmaf(sc.q[k][4 * t4 + 3], ur[t4].w, p3);
-                    }
-                    sc.qt[k][cc] = (p0 + p1) + (p2 + p3);
-                }
-                __syncwarp();
-            }
+            // ---- new item: its query rows arrived in this slot's header
             if constexpr (kMma) {
-                // A fragments: row g holds head h0 + g (rows >= GH are zero)
                 const int g = lane >> 2, c = lane & 3;
-                auto frag = [&](const float *row, int k0) -> uint32_t {
-                    if (g >= GH)
-                        return 0u;
-                    __nv_bfloat162 v = __floats2bfloat162_rn(row[k0], row[k0 + 1]);
-                    return *reinterpret_cast<uint32_t *>(&v);
-                };
-                const float *qrow = sc.q[g < GH ? g : 0];
-                const float *qtrow = sc.qt[g < GH ? g : 0];
+                if (win) {
+                    const uint32_t *hq = reinterpret_cast<const uint32_t *>(hdr) + (g < GH ? g : 0) * (kHeadDim / 2);
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks) {
-                    qa_w[ks][0] = frag(qrow, 16 * ks + 2 * c);
-                    qa_w[ks][2] = frag(qrow, 16 * ks + 2 * c + 8);
-                    qa_w[ks][1] = qa_w[ks][3] = 0u;
+                    for (int ks = 0; ks < 4; ++ks) {
+                        qa_w[ks][0] = g < GH ? hq[8 * ks + c] : 0u;
+                        qa_w[ks][2] = g < GH ? hq[8 * ks + c + 4] : 0u;
+                        qa_w[ks][1] = qa_w[ks][3] = 0u;
+                    }
+#pragma unroll
+                    for (int d = 0; d < 8; ++d)
+                        ow[d][0] = ow[d][1] = ow[d][2] = ow[d][3] = 0.f;
+                } else if constexpr (kLanePages) {
+                    const float *hqt = reinterpret_cast<const float *>(hdr);
+#pragma unroll
+                    for (int c = 0; c < DD; ++c) {
+                        qd[c] = hqt[c] * a.qscale;
+                        ol[c] = 0.f;
+                    }
+                } else {
+                    const float *hqt = reinterpret_cast<const float *>(hdr) + (g < GH ? g : 0) * DD;
+                    auto pack = [&](int k0) -> uint32_t {
+                        if (g >= GH)
+                            return 0u;
+                        const float2 v2 = *reinterpret_cast<const float2 *>(hqt + k0);
+                        __nv_bfloat162 v = __floats2bfloat162_rn(v2.x, v2.y);
+                        return *reinterpret_cast<uint32_t *>(&v);
+                    };
+#pragma unroll
+                    for (int ks = 0; ks < KSD; ++ks) {
+                        qa_d[ks][0] = pack(16 * ks + 2 * c);
+                        qa_d[ks][2] = pack(16 * ks + 2 * c + 8);
+                        qa_d[ks][1] = qa_d[ks][3] = 0u;
+                    }
+#pragma unroll
+                    for (int d = 0; d < NDD; ++d)
+                        od[d][0] = od[d][1] = od[d][2] = od[d][3] = 0.f;
                 }
-#pragma unroll
-                for (int ks = 0; ks < KSD; ++ks) {
-                    qa_d[ks][0] = frag(qtrow, 16 * ks + 2 * c);
-                    qa_d[ks][2] = frag(qtrow, 16 * ks + 2 * c + 8);
-                    qa_d[ks][1] = qa_d[ks][3] = 0u;
-                }
-#pragma unroll
-                for (int d = 0; d < 8; ++d)
-                    ow[d][0] = ow[d][1] = ow[d][2] = ow[d][3] = 0.f;
-#pragma unroll
-                for (int d = 0; d < (DD / 8 > 0 ? DD / 8 : 1); ++d)
-                    od[d][0] = od[d][1] = od[d][2] = od[d][3] = 0.f;
                 mm = -INFINITY;
                 lp = 0.f;
             } else {
-                const int ROWc = cur.window ? kHeadDim : DD;
+                const int ROWc = win ? kHeadDim : DD;
                 const int sub = lane % (ROWc / E);
 #pragma unroll
                 for (int k = 0; k < GH; ++k) {
 #pragma unroll
                     for (int e = 0; e < E; ++e)
-                        qr[k][e] = cur.window ? sc.q[k][sub * E + e] : sc.qt[k][sub * E + e];
+                        qr[k][e] = (win ? to_f32(reinterpret_cast<const T *>(hdr)[k * kHeadDim + sub * E + e])
+                                        : reinterpret_cast<const float *>(hdr)[k * DD + sub * E + e]) *
+                                   a.qscale;
                     m[k] = -INFINITY;
                     l[k] = 0.f;
 #pragma unroll
@@ -616,7 +932,7 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         }
 
         // ---- this stage's tokens
-        const unsigned char *src = my_slots + (size_t)slot * kSlotBytes;
+        unsigned char *src = my_slots + (size_t)slot * kSlotBytes;
         auto run_stage = [&](auto row_tag) {
             constexpr int ROW = decltype(row_tag)::value;
             constexpr int LPT = ROW / E;
@@ -625,8 +941,6 @@ __global__ void __launch_bounds__(kDecThreads, 1)
             constexpr int NI = TPS / TPI;  // warp-wide 16-byte loads per half slot
             constexpr int U = NI < 4 ? NI : 4;
             const int grp = lane / LPT, sub = lane % LPT;
-            const int tb = cur.t0 + s * TPS;
-            const int ntok = min(cur.t1 - tb, TPS);
 #pragma unroll
             for (int u0 = 0; u0 < NI; u0 += U) {
                 float sk[GH][U];
@@ -693,15 +1007,26 @@ __global__ void __launch_bounds__(kDecThreads, 1)
             }
         };
         if constexpr (kMma) {
-            const uint32_t sK = smem_u32(src), sV = smem_u32(src + kHalf);
-            if (cur.window)
-                mma_stage<kHeadDim, TPS_W, GH>(sK, sV, min(cur.t1 - (cur.t0 + s * TPS_W), TPS_W), 0xffu, qa_w, ow,
-                                              mm, lp, a.qscale, lane);
-            else
-                mma_stage<DD, TPS_D, GH>(sK, sV, min(cur.t1 - (cur.t0 + s * TPS_D), TPS_D), pmask, qa_d, od, mm,
-                                         lp, a.qscale, lane);
+            const uint32_t sK = smem_u32(src), sV = sK + kHalf;
+            if (win) {
+                if (ntok == TPS_W) {
+                    mma_stage<kHeadDim, TPS_W, GH, false>(sK, sV, ntok, 0xffu, qa_w, ow, mm, lp, a.qscale, lane);
+                } else {
+                    zero_masked_rows<kHeadDim, TPS_W>(src + kHalf, ntok, 0xffu, lane);
+                    mma_stage<kHeadDim, TPS_W, GH, true>(sK, sV, ntok, 0xffu, qa_w, ow, mm, lp, a.qscale, lane);
+                }
+            } else if constexpr (kLanePages) {
+                lane_stage<DD, TPS_D>(sK, sV, ntok, pmask, qd, ol, mm, lp, lane);
+            } else {
+                if (ntok == TPS_D && pmask == kFullPages) {
+                    mma_stage<DD, TPS_D, GH, false>(sK, sV, ntok, pmask, qa_d, od, mm, lp, a.qscale, lane);
+                } else {
+                    zero_masked_rows<DD, TPS_D>(src + kHalf, ntok, pmask, lane);
+                    mma_stage<DD, TPS_D, GH, true>(sK, sV, ntok, pmask, qa_d, od, mm, lp, a.qscale, lane);
+                }
+            }
         } else {
-            if (cur.window)
+            if (win)
                 run_stage(std::integral_constant<int, kHeadDim>());
             else
                 run_stage(std::integral_constant<int, DD>());
@@ -715,25 +1040,39 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         if (iss.it >= 0)
             issue_one();  // refill the slot just read
 
-        if (s + 1 < cur.nst)
+        if (!last)
             continue;
 
         // ---- item done: write the partial result (m, l, acc) of every head
-        const int h0 = cur.g * a.G + cur.hs * GH;
-        if constexpr (kMma) {
+        const size_t rec0 = (size_t)md.x;
+        if (kLanePages && !win) {
+            if constexpr (kLanePages) {
+#pragma unroll
+                for (int off = 16; off; off >>= 1)
+                    lp += __shfl_xor_sync(0xffffffffu, lp, off);
+                const float tot = reduce_scatter<DD>(ol, lane);
+                constexpr int LPE = 32 / DD;  // lanes holding each entry
+                if (lane % LPE == 0)
+                    a.rec_acc[rec0 * kHeadDim + lane / LPE] = tot;
+                if (lane == 0) {
+                    a.rec_m[rec0] = mm;
+                    a.rec_l[rec0] = lp;
+                }
+            }
+        } else if constexpr (kMma) {
             lp += __shfl_xor_sync(0xffffffffu, lp, 1);
             lp += __shfl_xor_sync(0xffffffffu, lp, 2);
             const int g = lane >> 2, c = lane & 3;
             if (g < GH) {
-                const size_t rec = ((size_t)cur.b * a.Hq + h0 + g) * a.maxc + cur.c;
+                const size_t rec = rec0 + (size_t)g * a.maxc;
                 float *ra = a.rec_acc + rec * kHeadDim;
-                if (cur.window) {
+                if (win) {
 #pragma unroll
                     for (int d = 0; d < 8; ++d)
                         *reinterpret_cast<float2 *>(ra + 8 * d + 2 * c) = make_float2(ow[d][0], ow[d][1]);
                 } else {
 #pragma unroll
-                    for (int d = 0; d < (DD / 8 > 0 ? DD / 8 : 1); ++d)
+                    for (int d = 0; d < NDD; ++d)
                         *reinterpret_cast<float2 *>(ra + 8 * d + 2 * c) = make_float2(od[d][0], od[d][1]);
                 }
                 if (c == 0) {
@@ -742,114 +1081,40 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                 }
             }
         } else {
-        const int LPTc = (cur.window ? kHeadDim : DD) / E;
-        for (int off = LPTc; off < 32; off <<= 1) {
+            const int LPTc = (win ? kHeadDim : DD) / E;
+            for (int off = LPTc; off < 32; off <<= 1) {
+#pragma unroll
+                for (int k = 0; k < GH; ++k) {
+                    const float mo = __shfl_xor_sync(0xffffffffu, m[k], off);
+                    const float lo = __shfl_xor_sync(0xffffffffu, l[k], off);
+                    const float mn = fmaxf(m[k], mo);
+                    const float fa = (m[k] == -INFINITY) ? 0.f : exp2f(m[k] - mn);
+                    const float fb = (mo == -INFINITY) ? 0.f : exp2f(mo - mn);
+                    l[k] = l[k] * fa + lo * fb;
+#pragma unroll
+                    for (int e = 0; e < E; ++e) {
+                        const float ao = __shfl_xor_sync(0xffffffffu, acc[k][e], off);
+                        acc[k][e] = acc[k][e] * fa + ao * fb;
+                    }
+                    m[k] = mn;
+                }
+            }
 #pragma unroll
             for (int k = 0; k < GH; ++k) {
-                const float mo = __shfl_xor_sync(0xffffffffu, m[k], off);
-                const float lo = __shfl_xor_sync(0xffffffffu, l[k], off);
-                const float mn = fmaxf(m[k], mo);
-                const float fa = (m[k] == -INFINITY) ? 0.f : exp2f(m[k] - mn);
-                const float fb = (mo == -INFINITY) ? 0.f : exp2f(mo - mn);
-                l[k] = l[k] * fa + lo * fb;
+                const size_t rec = rec0 + (size_t)k * a.maxc;
+                if (lane < LPTc) {
+                    float4 *dstv = reinterpret_cast<float4 *>(a.rec_acc + rec * kHeadDim + lane * E);
 #pragma unroll
-                for (int e = 0; e < E; ++e) {
-                    const float ao = __shfl_xor_sync(0xffffffffu, acc[k][e], off);
-                    acc[k][e] = acc[k][e] * fa + ao * fb;
+                    for (int e4 = 0; e4 < E / 4; ++e4)
+                        dstv[e4] = make_float4(acc[k][4 * e4], acc[k][4 * e4 + 1], acc[k][4 * e4 + 2],
+                                               acc[k][4 * e4 + 3]);
                 }
-                m[k] = mn;
-            }
-        }
-#pragma unroll
-        for (int k = 0; k < GH; ++k) {
-            const size_t rec = ((size_t)cur.b * a.Hq + h0 + k) * a.maxc + cur.c;
-            if (lane < LPTc) {
-                float4 *dstv = reinterpret_cast<float4 *>(a.rec_acc + rec * kHeadDim + lane * E);
-#pragma unroll
-                for (int e4 = 0; e4 < E / 4; ++e4)
-                    dstv[e4] = make_float4(acc[k][4 * e4], acc[k][4 * e4 + 1], acc[k][4 * e4 + 2],
-                                           acc[k][4 * e4 + 3]);
-            }
-            if (lane == 0) {
-                a.rec_m[rec] = m[k];
-                a.rec_l[rec] = l[k];
-            }
-        }
-        }
-        // publish the record, then count the arrival (acquire-release at GPU scope)
-        asm volatile("fence.acq_rel.gpu;" ::: "memory");
-        __syncwarp();
-        int arrived = 0;
-        int32_t *cnt = a.counters + ((size_t)cur.b * a.Hkv + cur.g) * a.HS + cur.hs;
-        if (lane == 0)
-            asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], 1;" : "=r"(arrived) : "l"(cnt) : "memory");
-        arrived = __shfl_sync(0xffffffffu, arrived, 0);
-        if (arrived != cur.nchunks - 1)
-            continue;
-
-        // ---- last arrival for (b, g, hs): merge every chunk
-        asm volatile("fence.acq_rel.gpu;" ::: "memory");
-        const int nch = cur.nchunks, nwc = cur.nwc;
-        const float *Uv = a.Uv + (size_t)cur.g * DD * kHeadDim;
-        T *out = static_cast<T *>(a.out);
-#pragma unroll 1
-        for (int k = 0; k < GH; ++k) {
-            const size_t rec0 = ((size_t)cur.b * a.Hq + h0 + k) * a.maxc;
-            float M = -INFINITY;
-            for (int c0 = 0; c0 < nch; c0 += 32)
-                if (c0 + lane < nch)
-                    M = fmaxf(M, __ldcg(a.rec_m + rec0 + c0 + lane));
-#pragma unroll
-            for (int off = 16; off; off >>= 1)
-                M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-            float lsum = 0.f, o0 = 0.f, o1 = 0.f, gd0 = 0.f, gd1 = 0.f;
-            for (int c0 = 0; c0 < nch; c0 += 32) {
-                float f = 0.f;
-                if (c0 + lane < nch) {
-                    f = exp2f(__ldcg(a.rec_m + rec0 + c0 + lane) - M);
-                    lsum = fmaf(f, __ldcg(a.rec_l + rec0 + c0 + lane), lsum);
-                }
-                const int jn = min(32, nch - c0);
-#pragma unroll 4
-                for (int j = 0; j < jn; ++j) {
-                    const float fj = __shfl_sync(0xffffffffu, f, j);
-                    const int cc = c0 + j;
-                    const float *ra = a.rec_acc + (rec0 + cc) * kHeadDim;
-                    if (cc < nwc) {
-                        const float2 v = __ldcg(reinterpret_cast<const float2 *>(ra) + lane);
-                        o0 = fmaf(fj, v.x, o0);
-                        o1 = fmaf(fj, v.y, o1);
-                    } else {
-                        if (lane < DD)
-                            gd0 = fmaf(fj, __ldcg(ra + lane), gd0);
-                        if (lane + 32 < DD)
-                            gd1 = fmaf(fj, __ldcg(ra + lane + 32), gd1);
-                    }
+                if (lane == 0) {
+                    a.rec_m[rec] = m[k];
+                    a.rec_l[rec] = l[k];
                 }
             }
-#pragma unroll
-            for (int off = 16; off; off >>= 1)
-                lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
-            if (lane < DD)
-                sc.qt[0][lane] = gd0;
-            if (lane + 32 < DD)
-                sc.qt[0][lane + 32] = gd1;
-            __syncwarp();
-#pragma unroll 4
-            for (int cc = 0; cc < DD; ++cc) {
-                const float gv = sc.qt[0][cc];
-                const float2 u2 = __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
-                o0 = fmaf(gv, u2.x, o0);
-                o1 = fmaf(gv, u2.y, o1);
-            }
-            __syncwarp();
-            const float inv = 1.f / lsum;
-            T *orow = out + ((size_t)cur.b * a.Hq + h0 + k) * kHeadDim;
-            orow[2 * lane] = from_f32<T>(o0 * inv);
-            orow[2 * lane + 1] = from_f32<T>(o1 * inv);
         }
-        if (lane == 0)
-            *cnt = 0;  // ready for the next call
     }
 
     if (!alive) {
@@ -857,14 +1122,44 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         for (int r = consumed + 1; r < issued; ++r)
             mbar_wait(&my_bars[r % kStages], (unsigned)((r / kStages) & 1), a.status);
     }
-    // the last warp to leave resets the item counter for the next call
-    if (lane == 0) {
-        if (atomicAdd(a.sched + 1, 1) == nwarps_total - 1) {
-            a.sched[0] = 0;
-            a.sched[1] = 0;
+
+    // ---- merge.  Groups (index b * per_chunk + gh) whose chunks this CTA
+    // covered completely are merged here; a group shared with other CTAs is
+    // merged by the CTA whose atomic completes its chunk count.
+    __threadfence();  // this thread's records are visible GPU-wide before any count below
+    __syncthreads();
+    if (lo < hi) {
+        auto group_of = [&](int it) {
+            const int b = seq_of(it);
+            return b * per_chunk + (it - s_pre[b] * per_chunk) / (s_pre[b + 1] - s_pre[b]);
+        };
+        const int ga = group_of(lo), gb = group_of(hi - 1);
+        for (int gi = ga + warp; gi <= gb; gi += kDecWarps) {
+            const int b = gi / per_chunk, gh = gi % per_chunk;
+            const int nch = s_pre[b + 1] - s_pre[b];
+            if (nch == 0)
+                continue;
+            const int base = s_pre[b] * per_chunk + gh * nch;
+            const int done = min(hi, base + nch) - max(lo, base);
+            if (done <= 0)
+                continue;
+            if (done < nch) {
+                int old = 0;
+                if (lane == 0)
+                    old = atomicAdd(a.counters + gi, done);
+                old = __shfl_sync(0xffffffffu, old, 0);
+                if (old + done != nch)
+                    continue;
+                __threadfence();  // the other CTAs' records of this group
+            }
+            const int nwc = (min(s_len[b], w) + cw - 1) / cw;
+            const int g = gh / a.HS, h0 = g * a.G + (gh % a.HS) * a.GH;
+            for (int k = 0; k < GH; ++k)
+                combine_row<T, DD>(a, b, h0 + k, g, nwc, nch, lane);
         }
     }
 }
+
 
 // --------------------------------------------------------------------- launch
 
@@ -882,19 +1177,20 @@ DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int
 }
 
 template <typename T, int DD, int GH>
-static cudaError_t decode_t(const DecodeArgs &a, cudaStream_t s)
+static cudaError_t decode_t(const DecodeArgs &a0, cudaStream_t s)
 {
     auto kern = decode_kernel<T, DD, GH>;
     CUtensorMap m_wk{}, m_wv{}, m_pk{}, m_pv{};
     if (decode_uses_mma<T, DD>()) {
-        constexpr int tps_w = kHalf / (kHeadDim * 2), tps_d = kHalf / (DD * 2);
-        const int pr = tps_d < kPage ? tps_d : kPage;
-        const unsigned long long ring_rows = (unsigned long long)a.B * a.Hkv * a.w;
-        const unsigned long long pool_rows = (unsigned long long)(a.num_pages > 0 ? a.num_pages : 1) * a.Hkv * kPage;
-        if (!make_tma_2d_bf16(&m_wk, a.win_k, ring_rows, kHeadDim, tps_w) ||
-            !make_tma_2d_bf16(&m_wv, a.win_v, ring_rows, kHeadDim, tps_w) ||
-            !make_tma_2d_bf16(&m_pk, a.pool_kd, pool_rows, DD, pr) ||
-            !make_tma_2d_bf16(&m_pv, a.pool_vd, pool_rows, DD, pr))
+        constexpr int tps_w = tps_ring<T>(), tps_d = tps_page<T, DD>();
+        // one page box: min(64, tps_d) tokens = that many * DD / 64 lines of 128 bytes
+        const int pr = (tps_d < kPage ? tps_d : kPage) * DD / kHeadDim;
+        const unsigned long long ring_rows = (unsigned long long)a0.B * a0.Hkv * a0.w;
+        const unsigned long long pool_lines = (unsigned long long)(a0.num_pages > 0 ? a0.num_pages : 1) * a0.Hkv * DD;
+        if (!make_tma_2d_bf16(&m_wk, a0.win_k, ring_rows, kHeadDim, tps_w) ||
+            !make_tma_2d_bf16(&m_wv, a0.win_v, ring_rows, kHeadDim, tps_w) ||
+            !make_tma_2d_bf16(&m_pk, a0.pool_kd, pool_lines, kHeadDim, pr) ||
+            !make_tma_2d_bf16(&m_pv, a0.pool_vd, pool_lines, kHeadDim, pr))
             return cudaErrorInvalidValue;
     }
     // one-time set-up per instantiation (kept out of the launch path so launches
@@ -902,15 +1198,36 @@ static cudaError_t decode_t(const DecodeArgs &a, cudaStream_t s)
     static int sms = 0;
     if (sms == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)decode_smem_bytes<GH>(DAR_DECODE_MAX_BATCH));
+                                             (int)decode_smem_bytes(DAR_DECODE_MAX_BATCH));
         if (e != cudaSuccess)
             return e;
-        int dev = 0;
+        int dev = 0, n = 0;
         cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        sms = n;
     }
-    kern<<<sms, kDecThreads, decode_smem_bytes<GH>(a.B), s>>>(m_wk, m_wv, m_pk, m_pv, a);
-    return cudaGetLastError();
+    const DecodeArgs &a = a0;
+    const int rows = a.B * a.Hq;
+    const int prep_blocks = min(2 * sms, max(1, (rows + kPrepThreads / 32 - 1) / (kPrepThreads / 32)));
+    // both kernels use programmatic launch: prep computes q~ while the kernel
+    // before it finishes (and waits for it before exiting); the stream kernel
+    // sets up while prep drains
+    cudaLaunchAttribute pdl[1];
+    pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    pdl[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.stream = s;
+    cfg.attrs = pdl;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(prep_blocks);
+    cfg.blockDim = dim3(kPrepThreads);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, decode_prep_kernel<T, DD>, a);
+    if (e != cudaSuccess)
+        return e;
+    cfg.gridDim = dim3(sms);
+    cfg.blockDim = dim3(kDecThreads);
+    cfg.dynamicSmemBytes = decode_smem_bytes(a.B);
+    return cudaLaunchKernelEx(&cfg, kern, m_wk, m_wv, m_pk, m_pv, a);
 }
 
 template <typename T, int DD>

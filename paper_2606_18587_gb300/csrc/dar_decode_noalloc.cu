@@ -53,13 +53,7 @@ extern "C" dar_status dar_attn_decode_noalloc(const dar_cache *cache, int32_t Hq
         dar::set_last_error(msg);
         return DAR_ERR_CAPACITY;
     }
-    // The array keeps whatever the previous call left; the decode kernel needs
-    // its counters at zero, so clear the region this call uses.
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const cudaError_t e = cudaMemsetAsync(g_scratch_ptr[dev], 0, need, s);
-    if (e != cudaSuccess) {
-        dar::set_last_error(cudaGetErrorString(e));
-        return DAR_ERR_CUDA;
-    }
+    // The array keeps whatever the previous call left; the decode kernels
+    // rewrite every byte of it they read, so it needs no clearing.
     return dar_attn_decode(cache, Hq, q, Uk, Uv, scale, out, g_scratch_ptr[dev], need, stream);
 }

@@ -31,9 +31,9 @@ struct DecodeArgs {
     const int32_t *seq_lens;
     int32_t *status;
     const float *Uk, *Uv;  // [Hkv][dd][64]
-    float *rec_m, *rec_l, *rec_acc;  // split-K partial results
-    int32_t *counters;               // per (b, g, head slice) arrival counts
-    int32_t *sched;                  // [2] item counter, exited-warp counter
+    float *rec_m, *rec_l, *rec_acc;  // split-K partial results [B][Hq][maxc] (acc: x 64)
+    float *qt;                       // [B][Hq][dd] q~ = q Uk^T
+    int32_t *counters;               // [B][Hkv][HS] chunks finished per shared group
     int B, Hq, Hkv, G, GH, HS, w, maxp, num_pages, maxc, cw, cd;
     float qscale;  // scale * log2(e)
 };
@@ -63,7 +63,7 @@ cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s);
 
 // Split-K geometry of the decode kernel (shared by workspace sizing and launch).
 struct DecodeGeometry {
-    int cw, cd, maxc, GH, HS;
+    int cw, cd, maxc, GH, HS;  // minimum chunk sizes (tokens), chunks per head at that size, head grouping
 };
 DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int maxp);
 

@@ -129,8 +129,16 @@ __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
-// Order generic-proxy shared-memory writes before later async-proxy reads
-// (the tensor core reading operands written with st.shared).
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialisation may start while the previous kernel on its stream still runs;
+// grid_dep_wait() returns once that kernel has finished and its memory
+// operations are visible.  grid_dep_launch() lets the next such kernel start.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Order generic-proxy shared-memory accesses before later async-proxy accesses
+// (the tensor core reading operands written with st.shared, or a TMA copy
+// overwriting bytes the generic proxy wrote).
 __device__ __forceinline__ void fence_proxy_async_smem()
 {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

@@ -191,11 +191,11 @@ def dar_decode_workspace_bytes(cache: DarCache, Hq: int) -> int:
 
 
 def decode_workspace(cache: DarCache, Hq: int):
-    """A zero-filled workspace of the size dar_attn_decode needs."""
+    """A workspace of the size dar_attn_decode needs (no initialisation needed)."""
     nbytes = dar_decode_workspace_bytes(cache, Hq)
     if nbytes == 0:
         raise DarError(DAR_ERR_INVALID_ARG, dar_last_error() or "bad cache/Hq")
-    return torch.zeros(nbytes, dtype=torch.uint8, device=cache.win_k.device)
+    return torch.empty(nbytes, dtype=torch.uint8, device=cache.win_k.device)
 
 
 def dar_attn_decode(cache: DarCache, q, Uk, Uv, workspace, scale=0.0, out=None, stream=None):
