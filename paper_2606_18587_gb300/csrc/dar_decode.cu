@@ -402,105 +402,73 @@ __device__ __forceinline__ float reduce_scatter(const float (&o)[DD], int lane)
 }
 
 // Per-sequence tables of one decode call, built by every CTA of the stream
-// kernel into its shared memory (kSeqPerThread sequences per thread, one
-// block-wide scan): s_len[b] = validated length (-1 if beyond the cache's
-// capacity), s_pre[b] = chunks of the sequences before b (s_pre[B] = all),
-// and the chunk sizes (cw, cd) = f * (minimum sizes), f chosen so that the
-// grid gets about kItemsPerWarp items per warp.  Larger chunks only lower the
-// chunk counts, so the workspace sized for the minimum chunks always fits.
-constexpr int kSeqPerThread = DAR_DECODE_MAX_BATCH / kDecThreads;
-
-__device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, int *s_len, long long *s_red,
-                                             int *s_scan, int *s_f)
+// kernel into its shared memory: s_len[b] = validated length (-1 if beyond
+// the cache's capacity), s_pre[b] = chunks of the sequences before b
+// (s_pre[B] = all), and the chunk sizes (cw, cd) = f * (minimum sizes), f
+// chosen so that the grid gets about kItemsPerWarp items per warp.  Larger
+// chunks only lower the chunk counts, so the workspace sized for the minimum
+// chunks always fits.  The CTA loads the lengths; warp 0 (a contiguous run of
+// sequences per lane) reduces and scans them.
+__device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, int *s_len, int *s_f)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int B = a.B, w = a.w;
-    int Ls[kSeqPerThread];
-#pragma unroll
-    for (int k = 0; k < kSeqPerThread; ++k) {
-        const int b = threadIdx.x * kSeqPerThread + k;
-        Ls[k] = b < B ? a.seq_lens[b] : 0;
-    }
-    long long units = 0;
-#pragma unroll
-    for (int k = 0; k < kSeqPerThread; ++k) {
-        const int b = threadIdx.x * kSeqPerThread + k;
-        int L = Ls[k];
-        if (b < B && (L < 0 || (long long)L - w > (long long)a.maxp * kPage)) {
+    for (int b = threadIdx.x; b < B; b += blockDim.x) {
+        int L = a.seq_lens[b];
+        if (L < 0 || (long long)L - w > (long long)a.maxp * kPage) {
             if (blockIdx.x == 0)
                 report(a.status, DAR_ERR_CAPACITY);
             L = -1;
         }
-        Ls[k] = L;
-        if (b < B)
-            s_len[b] = L;
-        const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
-        units += (nwin + a.cw - 1) / a.cw + (ndist + a.cd - 1) / a.cd;
+        s_len[b] = L;
     }
-#pragma unroll
-    for (int off = 16; off; off >>= 1)
-        units += __shfl_xor_sync(0xffffffffu, units, off);
-    if (lane == 0)
-        s_red[warp] = units;
     __syncthreads();
     if (warp == 0) {
-        units = lane < kDecWarps ? s_red[lane] : 0;
+        const int per = (B + 31) / 32;
+        const int b0 = min(B, lane * per), b1 = min(B, b0 + per);
+        long long units = 0;
+        for (int b = b0; b < b1; ++b) {
+            const int L = s_len[b];
+            const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
+            units += (nwin + a.cw - 1) / a.cw + (ndist + a.cd - 1) / a.cd;
+        }
 #pragma unroll
         for (int off = 16; off; off >>= 1)
             units += __shfl_xor_sync(0xffffffffu, units, off);
-        if (lane == 0) {
-            const long long target = (long long)gridDim.x * kDecWarps * kItemsPerWarp;
-            long long f = (units * a.Hkv * a.HS + target - 1) / target;
-            const long long fmax = (long long)(64 * kPage) / a.cd;  // a page chunk spans at most 64 pages
-            f = f > fmax ? fmax : f;
-            f = f > kMaxChunkScale ? kMaxChunkScale : f;
-            *s_f = f < 1 ? 1 : (int)f;
+        const long long target = (long long)gridDim.x * kDecWarps * kItemsPerWarp;
+        long long f = (units * a.Hkv * a.HS + target - 1) / target;
+        const long long fmax = (long long)(64 * kPage) / a.cd;  // a page chunk spans at most 64 pages
+        f = f > fmax ? fmax : f;
+        f = f > kMaxChunkScale ? kMaxChunkScale : f;
+        f = f < 1 ? 1 : f;
+        const int cw = a.cw * (int)f, cd = a.cd * (int)f;
+        int mine = 0;
+        for (int b = b0; b < b1; ++b) {
+            const int L = s_len[b];
+            const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
+            mine += (nwin + cw - 1) / cw + (ndist + cd - 1) / cd;
         }
-    }
-    __syncthreads();
-    const int cw = a.cw * *s_f, cd = a.cd * *s_f;
-    int cnt[kSeqPerThread], mine = 0;
-#pragma unroll
-    for (int k = 0; k < kSeqPerThread; ++k) {
-        const int L = Ls[k];
-        const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
-        cnt[k] = (nwin + cw - 1) / cw + (ndist + cd - 1) / cd;
-        mine += cnt[k];
-    }
-    int incl = mine;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, off);
-        if (lane >= off)
-            incl += y;
-    }
-    if (lane == 31)
-        s_scan[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {
-        int v = lane < kDecWarps ? s_scan[lane] : 0;
+        int incl = mine;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, v, off);
+            const int y = __shfl_up_sync(0xffffffffu, incl, off);
             if (lane >= off)
-                v += y;
+                incl += y;
         }
-        if (lane < kDecWarps)
-            s_scan[lane] = v;  // inclusive over warps
-    }
-    __syncthreads();
-    int run = incl - mine + (warp > 0 ? s_scan[warp - 1] : 0);
-#pragma unroll
-    for (int k = 0; k < kSeqPerThread; ++k) {
-        const int b = threadIdx.x * kSeqPerThread + k;
-        if (b < B)
+        int run = incl - mine;
+        for (int b = b0; b < b1; ++b) {
+            const int L = s_len[b];
+            const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
             s_pre[b] = run;
-        run += cnt[k];
+            run += (nwin + cw - 1) / cw + (ndist + cd - 1) / cd;
+        }
+        if (lane == 31)
+            s_pre[B] = incl;  // all chunks
+        if (lane == 0)
+            *s_f = (int)f;
     }
-    if (threadIdx.x == kDecThreads - 1)
-        s_pre[B] = run;  // all chunks
     __syncthreads();
-    return make_int2(cw, cd);
+    return make_int2(a.cw * *s_f, a.cd * *s_f);
 }
 
 // One (b, h) output row from its chunk records, by one warp:
@@ -515,6 +483,13 @@ __device__ __forceinline__ void combine_row(const DecodeArgs &a, int b, int h, i
 {
     const size_t rec0 = ((size_t)b * a.Hq + h) * a.maxc;
     const int jmax = min(nch, kCombChunks);
+    // Uv rows in flight with the records (small d_down only: registers)
+    constexpr int UVP = DD <= 32 ? DD : 1;
+    const float *Uv = a.Uv + (size_t)g * DD * kHeadDim;
+    float2 uv[UVP];
+#pragma unroll
+    for (int cc = 0; cc < UVP; ++cc)
+        uv[cc] = __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
     float mj = -INFINITY, lj = 0.f;
     if (lane < jmax) {
         mj = __ldcg(a.rec_m + rec0 + lane);
@@ -573,11 +548,11 @@ __device__ __forceinline__ void combine_row(const DecodeArgs &a, int b, int h, i
     for (int off = 16; off; off >>= 1)
         lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
     // lift the global part once: o += gd Uv[g]   (gd[c] sits in lane c / 2)
-    const float *Uv = a.Uv + (size_t)g * DD * kHeadDim;
 #pragma unroll
     for (int cc = 0; cc < DD; ++cc) {
         const float gv = __shfl_sync(0xffffffffu, (cc & 1) ? gd1 : gd0, cc >> 1);
-        const float2 u2 = __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
+        const float2 u2 = UVP == DD ? uv[cc < UVP ? cc : 0]
+                                    : __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
         o0 = fmaf(gv, u2.x, o0);
         o1 = fmaf(gv, u2.y, o1);
     }
@@ -615,8 +590,7 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     int4 *meta = reinterpret_cast<int4 *>(bars + kDecWarps * kStages);
     int *s_pre = reinterpret_cast<int *>(meta + kDecWarps * kStages);  // [B + 1]
     int *s_len = s_pre + a.B + 1;                                      // [B]
-    __shared__ long long s_red[kDecWarps];
-    __shared__ int s_scan[kDecWarps], s_f;
+    __shared__ int s_f;
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     unsigned char *my_slots = slots + (size_t)warp * kStages * kSlotBytes;
@@ -638,10 +612,18 @@ __global__ void __launch_bounds__(kDecThreads, 1)
             sm100::prefetch_tensormap(&tm_pv);
         }
     }
+    // The block table is not written by the cache append: warm L2 with this
+    // CTA's share of it while the kernels before finish.
+    {
+        const size_t lines = ((size_t)a.B * a.maxp * sizeof(int32_t) + 127) / 128;
+        const size_t l0 = lines * blockIdx.x / gridDim.x, l1 = lines * (blockIdx.x + 1) / gridDim.x;
+        for (size_t i = l0 + threadIdx.x; i < l1; i += blockDim.x)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<const char *>(a.block_table) + i * 128));
+    }
     // everything below reads the cache and q~ (the prep kernel waited for the
     // kernel before it, so both are final)
     sm100::grid_dep_wait();
-    const int2 chunk = build_tables(a, s_pre, s_len, s_red, s_scan, &s_f);
+    const int2 chunk = build_tables(a, s_pre, s_len, &s_f);
     const int cw = chunk.x, cd = chunk.y;
     if (blockIdx.x == 0) {  // sequences with nothing to attend to get a zero output
         T *out = static_cast<T *>(a.out);
@@ -1115,6 +1097,7 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                 }
             }
         }
+
     }
 
     if (!alive) {
@@ -1124,9 +1107,11 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     }
 
     // ---- merge.  Groups (index b * per_chunk + gh) whose chunks this CTA
-    // covered completely are merged here; a group shared with other CTAs is
-    // merged by the CTA whose atomic completes its chunk count.
-    __threadfence();  // this thread's records are visible GPU-wide before any count below
+    // covered completely are merged as soon as every warp is done; a group
+    // shared with other CTAs is merged by the CTA whose atomic completes its
+    // chunk count.  Each warp releases its records GPU-wide as it finishes, so
+    // that fence overlaps the other warps' streaming.
+    __threadfence();
     __syncthreads();
     if (lo < hi) {
         auto group_of = [&](int it) {
