@@ -1,23 +1,27 @@
 // dar_prefill_tc.cu -- causal DAR attention forward (bf16) on the 5th-generation
-// tensor cores: tcgen05.mma with operands in shared memory (staged by TMA) and
-// fp32 accumulators in tensor memory (TMEM).
+// tensor cores: tcgen05.mma with operands staged by TMA in shared memory (or,
+// for P, held in tensor memory) and fp32 accumulators in tensor memory (TMEM).
 //
 // One CTA = 128 query rows of one head; key tiles of 64, visited from the
 // diagonal down to key 0.  Per key tile (Eq. 3: local iff i - j < w):
 //   local part   S_loc  = Q  K^T       (M128 N64 K64)   O_loc  += P_loc  V    (N64)
 //   global part  S_glob = Q~ (K^D)^T   (M128 N64 Kdd)   O_glob += P_glob V^D  (Ndd)
 // with q~ = q Uk^T (W_up absorbed into the query, exact by linearity of
-// Eq. 2).  A tile issues only the parts it needs; a band tile (both kinds)
-// selects per element.  One online softmax over both parts (Eq. 4), with the
-// running max raised lazily (only when it grows by more than 2^8), and the
-// epilogue lifts the global part once:  o = (O_loc + O_glob Uv) / l.
+// Eq. 2).  A tile that holds both kinds (the window edge crosses it) is run
+// as two virtual tiles, each with the other kind masked out.  One online
+// softmax over every virtual tile (Eq. 4), with the running max raised lazily
+// (only when it grows by more than 2^8), and the epilogue lifts the global
+// part once:  o = (O_loc + O_glob Uv) / l.
 //
 // Warp roles (192 threads): warp 0 issues TMA loads, warp 1 allocates TMEM and
 // issues the MMAs (one thread), warps 2-5 own one query row per thread
-// (TMEM lane = row) for q~, the softmax and the epilogue.  256 TMEM columns
-// and ~100 KB of shared memory per CTA let two CTAs share an SM, so one CTA's
-// softmax overlaps the other's MMA and load waits.  Every wait is bounded; on
-// a timeout the CTA flags *status and exits.
+// (TMEM lane = row) for q~, the softmax and the epilogue.  The softmax writes
+// P (bf16) into TMEM with tcgen05.st and the PV products take it from there
+// as their A operand, so P never touches shared memory.  Two S buffers (when
+// d_down <= 32) let S(t+1) run while the softmax works on S(t).  256 TMEM
+// columns and ~80 KB of shared memory per CTA let two CTAs share an SM, so
+// one CTA's softmax overlaps the other's MMA and load waits.  Every wait is
+// bounded; on a timeout the CTA flags *status and exits.
 #include <cuda.h>
 
 #include "dar_common.cuh"
@@ -32,30 +36,44 @@ using namespace sm100;
 constexpr int BM = 128, BN = 64;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t COL_SL = 0, COL_SG = 64, COL_OL = 128, COL_OG = 192;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p stays below 2^8 between rescales
 
 constexpr uint32_t align_up(uint32_t x, uint32_t a) { return (x + a - 1) / a * a; }
 
-// Shared-memory layout (offsets from a 1024-byte aligned base).
+// Tensor-memory columns of one CTA (256 of the SM's 512, two CTAs per SM):
+// S buffers (fp32, BN columns each; two when they fit, so S(t+1) can be
+// computed while the softmax still reads S(t)), O_loc (64), P (bf16 pairs,
+// BN / 2 columns; the A operand of the PV products), O_glob (DP).
+template <int DP>
+struct Tmem {
+    static constexpr int NSB = DP <= 32 ? 2 : 1;
+    static constexpr uint32_t S = 0;
+    static constexpr uint32_t OL = NSB * BN;
+    static constexpr uint32_t P = 192;
+    static constexpr uint32_t OG = NSB == 2 ? 224 : 128;
+    static_assert(OL + 64 <= P && P + BN / 2 <= (NSB == 2 ? OG : 256) && (NSB == 1 || OG + DP <= kTmemCols),
+                  "tensor-memory columns overlap");
+};
+
+// Shared-memory layout (offsets from a 1024-byte aligned base).  A stage holds
+// the operands of one virtual tile: K and V (local) or K^D and V^D (global).
 template <int DP>
 struct Layout {
-    static constexpr int NS = 2;                          // K/V stages
+    static constexpr int NS = 3;                          // K/V stages
     static constexpr uint32_t Q = 0;                      // [128][64] bf16, 128B swizzle
     static constexpr uint32_t QT = BM * 64 * 2;           // [128][DP] bf16
     static constexpr uint32_t STG = align_up(QT + BM * DP * 2, 1024);
     static constexpr uint32_t K_OFF = 0;                  // [64][64]
     static constexpr uint32_t V_OFF = BN * 64 * 2;        // [64][64]
-    static constexpr uint32_t KD_OFF = 2 * BN * 64 * 2;   // [64][DP]
-    static constexpr uint32_t VD_OFF = KD_OFF + BN * DP * 2;
-    static constexpr uint32_t STAGE = align_up(VD_OFF + BN * DP * 2, 1024);
-    static constexpr uint32_t PL = STG + NS * STAGE;      // P_loc  [128][64] bf16 (one 128B-swizzle atom wide)
-    static constexpr uint32_t PG = PL + BM * BN * 2;      // P_glob
-    static constexpr uint32_t UK = PG + BM * BN * 2;      // fp32 [DP][64]
+    static constexpr uint32_t KD_OFF = 0;                 // [64][DP]
+    static constexpr uint32_t VD_OFF = align_up(BN * DP * 2, 1024);
+    static constexpr uint32_t STAGE = align_up(2 * BN * 64 * 2, 1024);
+    static constexpr uint32_t UK = STG + NS * STAGE;      // fp32 [DP][64]
     static constexpr uint32_t UV = UK + DP * 64 * 4;
     static constexpr uint32_t BAR = UV + DP * 64 * 4;
     static constexpr uint32_t TOTAL = BAR + 256;
     static_assert(STAGE % 1024 == 0 && STG % 1024 == 0, "operand tiles must stay 1024-byte aligned");
+    static_assert(VD_OFF + BN * DP * 2 <= STAGE, "a stage holds either part");
 };
 
 template <int DP>
@@ -131,6 +149,42 @@ __device__ __forceinline__ uint4 ld_swz(const unsigned char *base, int r, int c)
     return *reinterpret_cast<const uint4 *>(base + (size_t)r * RB + phys * 16);
 }
 
+// Virtual tiles: a key tile whose pairs are all local or all global is one
+// virtual tile; a band tile (the window edge crosses it) is two, its local
+// part then its global part, each with the other part masked out.  All roles
+// walk the same sequence, from the diagonal down to key 0.
+struct VTile {
+    int kt;    // key tile index (keys kt*BN .. kt*BN+BN-1)
+    bool loc;  // local part (Q K^T, V) or global part (Q~ K^D^T, V^D)
+    bool band; // the key tile also has the other part
+};
+
+__device__ __forceinline__ VTile vt_first(int i0, int i_last, int w)
+{
+    const int kt = i_last / BN;
+    const TileKind k = tile_kind(i0, i_last, kt * BN, w);
+    return VTile{kt, k.loc, k.loc && k.glob};
+}
+
+__device__ __forceinline__ VTile vt_next(VTile v, int i0, int i_last, int w)
+{
+    if (v.band && v.loc)
+        return VTile{v.kt, false, true};
+    const int kt = v.kt - 1;
+    if (kt < 0)
+        return VTile{-1, false, false};
+    const TileKind k = tile_kind(i0, i_last, kt * BN, w);
+    return VTile{kt, k.loc, k.loc && k.glob};
+}
+
+__device__ __forceinline__ int vt_count(int i0, int i_last, int w)
+{
+    int n = 0;
+    for (VTile v = vt_first(i0, i_last, w); v.kt >= 0; v = vt_next(v, i0, i_last, w))
+        ++n;
+    return n;
+}
+
 template <int DP>
 __global__ void __launch_bounds__(kThreads, 2)
     prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -138,20 +192,22 @@ __global__ void __launch_bounds__(kThreads, 2)
                       const __grid_constant__ CUtensorMap tmVD, PrefillArgs a)
 {
     using Ly = Layout<DP>;
+    using Tm = Tmem<DP>;
     constexpr int NS = Ly::NS;
+    constexpr int NSB = Tm::NSB;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + Ly::BAR);
-    uint64_t *full = bars;            // [NS] TMA -> MMA
-    uint64_t *empty = bars + NS;      // [NS] MMA -> TMA
-    uint64_t *q_full = bars + 2 * NS; // Q landed
-    uint64_t *qt_ready = q_full + 1;  // q~ written, O zeroed (128 arrivals)
-    uint64_t *s_full = q_full + 2;    // S of a tile computed
-    uint64_t *s_free = q_full + 3;    // S read into registers (128 arrivals)
-    uint64_t *p_full = q_full + 4;    // P written (128 arrivals)
-    uint64_t *pv_done = q_full + 5;   // PV of a tile finished
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_full + 6);
+    uint64_t *full = bars;                 // [NS] TMA -> MMA
+    uint64_t *empty = bars + NS;           // [NS] MMA -> TMA
+    uint64_t *s_full = bars + 2 * NS;      // [NSB] S of a virtual tile computed
+    uint64_t *s_free = s_full + NSB;       // [NSB] S read into registers (128 arrivals)
+    uint64_t *q_full = s_free + NSB;       // Q landed
+    uint64_t *qt_ready = q_full + 1;       // q~ written, O zeroed (128 arrivals)
+    uint64_t *p_full = q_full + 2;         // P written to TMEM (128 arrivals)
+    uint64_t *pv_done = q_full + 3;        // PV of a virtual tile finished
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_full + 4);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -160,17 +216,19 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int qt = nqt - 1 - (int)blockIdx.y;  // longest rows first
     const int bh = blockIdx.x, b = bh / a.Hq, h = bh % a.Hq, g = h / (a.Hq / a.Hkv);
     const int i0 = qt * BM, i_last = min(i0 + BM, N) - 1;
-    const int T = i_last / BN + 1;  // key tiles kt = T-1-t, t = 0..T-1
+    const int VT = vt_count(i0, i_last, w);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
+        for (int s = 0; s < NSB; ++s) {
+            mbar_init(&s_full[s], 1);
+            mbar_init(&s_free[s], 128);
+        }
         mbar_init(q_full, 1);
         mbar_init(qt_ready, 128);
-        mbar_init(s_full, 1);
-        mbar_init(s_free, 128);
         mbar_init(p_full, 128);
         mbar_init(pv_done, 1);
         *abort_flag = 0;
@@ -195,21 +253,19 @@ __global__ void __launch_bounds__(kThreads, 2)
             prefetch_tensormap(&tmVD);
             mbar_expect_tx(q_full, BM * 64 * 2);
             tma_load_2d(sm + Ly::Q, &tmQ, 0, (b * a.Hq + h) * N + i0, q_full);
-            for (int t = 0; t < T; ++t) {
+            VTile vt = vt_first(i0, i_last, w);
+            for (int t = 0; t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
                 const int s = t % NS;
                 if (t >= NS && !mbar_wait(&empty[s], ((t / NS) - 1) & 1, abort_flag))
                     break;
-                const int j0 = (T - 1 - t) * BN;
-                const TileKind k = tile_kind(i0, i_last, j0, w);
-                const unsigned bytes = (k.loc ? 2 * BN * 64 * 2 : 0) + (k.glob ? 2 * BN * DP * 2 : 0);
                 unsigned char *st = sm + Ly::STG + s * Ly::STAGE;
-                const int krow = (b * a.Hkv + g) * N + j0;
-                mbar_expect_tx(&full[s], bytes);
-                if (k.loc) {
+                const int krow = (b * a.Hkv + g) * N + vt.kt * BN;
+                if (vt.loc) {
+                    mbar_expect_tx(&full[s], 2 * BN * 64 * 2);
                     tma_load_2d(st + Ly::K_OFF, &tmK, 0, krow, &full[s]);
                     tma_load_2d(st + Ly::V_OFF, &tmV, 0, krow, &full[s]);
-                }
-                if (k.glob) {
+                } else {
+                    mbar_expect_tx(&full[s], 2 * BN * DP * 2);
                     tma_load_2d(st + Ly::KD_OFF, &tmKD, 0, krow, &full[s]);
                     tma_load_2d(st + Ly::VD_OFF, &tmVD, 0, krow, &full[s]);
                 }
@@ -222,62 +278,64 @@ __global__ void __launch_bounds__(kThreads, 2)
             constexpr uint32_t idPV = idesc_bf16(BM, 64, true);
             constexpr uint32_t idPVg = idesc_bf16(BM, DP, true);
             const uint32_t sQ = smem_u32(sm + Ly::Q), sQT = smem_u32(sm + Ly::QT);
-            const uint32_t sPL = smem_u32(sm + Ly::PL), sPG = smem_u32(sm + Ly::PG);
             bool ok = mbar_wait(qt_ready, 0, abort_flag);
             tc_fence_after();
-            auto issue_S = [&](int t) -> bool {
-                const int s = t % NS;
+            auto issue_S = [&](int t, VTile vt) -> bool {
+                const int s = t % NS, sb = t % NSB;
                 if (!mbar_wait(&full[s], (t / NS) & 1, abort_flag))
                     return false;
-                if (t > 0 && !mbar_wait(s_free, (t - 1) & 1, abort_flag))
+                if (t >= NSB && !mbar_wait(&s_free[sb], ((t / NSB) - 1) & 1, abort_flag))
                     return false;
                 tc_fence_after();
-                const TileKind k = tile_kind(i0, i_last, (T - 1 - t) * BN, w);
                 const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
-                if (k.loc)
+                const uint32_t dS = tmem + Tm::S + sb * BN;
+                if (vt.loc)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        mma_f16_ss(tmem + COL_SL, smem_desc(sQ + kk * 32, 16, 1024, kSw128),
+                        mma_f16_ss(dS, smem_desc(sQ + kk * 32, 16, 1024, kSw128),
                                    smem_desc(st + Ly::K_OFF + kk * 32, 16, 1024, kSw128), idS, kk > 0);
-                if (k.glob)
+                else
 #pragma unroll
                     for (int kk = 0; kk < DP / 16; ++kk)
-                        mma_f16_ss(tmem + COL_SG, smem_desc(sQT + kk * 32, 16, 8 * DP * 2, dp_swizzle<DP>()),
+                        mma_f16_ss(dS, smem_desc(sQT + kk * 32, 16, 8 * DP * 2, dp_swizzle<DP>()),
                                    smem_desc(st + Ly::KD_OFF + kk * 32, 16, 8 * DP * 2, dp_swizzle<DP>()), idS,
                                    kk > 0);
-                mma_commit(s_full);
+                mma_commit(&s_full[sb]);
                 return true;
             };
-            auto issue_PV = [&](int t) -> bool {
+            auto issue_PV = [&](int t, VTile vt) -> bool {
                 const int s = t % NS;
                 if (!mbar_wait(p_full, t & 1, abort_flag))
                     return false;
                 tc_fence_after();
-                const TileKind k = tile_kind(i0, i_last, (T - 1 - t) * BN, w);
                 const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
 #pragma unroll
-                for (int kk = 0; kk < BN / 16; ++kk) {
-                    const uint32_t aoff = kk * 32;
-                    if (k.loc)
-                        mma_f16_ss(tmem + COL_OL, smem_desc(sPL + aoff, 16, 1024, kSw128),
-                                   smem_desc(st + Ly::V_OFF + kk * 16 * 128, 16, 1024, kSw128), idPV, true);
-                    if (k.glob)
-                        mma_f16_ss(tmem + COL_OG, smem_desc(sPG + aoff, 16, 1024, kSw128),
-                                   smem_desc(st + Ly::VD_OFF + kk * 16 * DP * 2, 16, 8 * DP * 2,
-                                             dp_swizzle<DP>()),
+                for (int kk = 0; kk < BN / 16; ++kk) {  // P (TMEM, 8 columns per 16 keys) times V / V^D
+                    const uint32_t aP = tmem + Tm::P + kk * 8;
+                    if (vt.loc)
+                        mma_f16_ts(tmem + Tm::OL, aP, smem_desc(st + Ly::V_OFF + kk * 16 * 128, 16, 1024, kSw128),
+                                   idPV, true);
+                    else
+                        mma_f16_ts(tmem + Tm::OG, aP,
+                                   smem_desc(st + Ly::VD_OFF + kk * 16 * DP * 2, 16, 8 * DP * 2, dp_swizzle<DP>()),
                                    idPVg, true);
                 }
                 mma_commit(pv_done);
                 mma_commit(&empty[s]);
                 return true;
             };
-            // S(t) is issued as soon as the softmax has read S(t-1), so it
-            // overlaps the softmax of tile t-1; PV(t-1) follows once P(t-1) is written
-            for (int t = 0; ok && t <= T; ++t) {
-                if (t < T)
-                    ok = issue_S(t);
-                if (ok && t > 0)
-                    ok = issue_PV(t - 1);
+            // S(t) is issued as soon as its K tile and an S buffer are free, so
+            // it overlaps the softmax of t-1; PV(t-1) follows once P(t-1) is in TMEM
+            VTile vs = vt_first(i0, i_last, w), vp = vs;
+            for (int t = 0; ok && t <= VT; ++t) {
+                if (t < VT) {
+                    ok = issue_S(t, vs);
+                    vs = vt_next(vs, i0, i_last, w);
+                }
+                if (ok && t > 0) {
+                    ok = issue_PV(t - 1, vp);
+                    vp = vt_next(vp, i0, i_last, w);
+                }
             }
         }
     } else {
@@ -343,22 +401,25 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int e = 0; e < 16; ++e)
                 z[e] = 0u;
 #pragma unroll
-            for (int c = 0; c < 64 + DP; c += 16)
-                tmem_st16(tl + COL_OL + c, z);
+            for (int c = 0; c < 64; c += 16)
+                tmem_st16(tl + Tm::OL + c, z);
+#pragma unroll
+            for (int c = 0; c < DP; c += 16)
+                tmem_st16(tl + Tm::OG + c, z);
             tmem_wait_st();
         }
-        fence_proxy_async_smem();
+        fence_proxy_async_smem();  // q~ (generic stores) before the MMAs read it
         tc_fence_before();
         mbar_arrive(qt_ready);
 
         const float c2 = a.qscale;  // softmax scale * log2(e)
         float m_used = -INFINITY, l = 0.f;
-        int pv_waited = -1;  // highest tile whose PV completion has been observed
-        for (int t = 0; ok && t < T; ++t) {
-            const int j0 = (T - 1 - t) * BN;
-            const TileKind k = tile_kind(i0, i_last, j0, w);
-            const bool band = k.loc && k.glob;
-            if (!wait_uniform(s_full, t & 1)) {
+        int pv_waited = -1;  // highest virtual tile whose PV completion has been observed
+        VTile vt = vt_first(i0, i_last, w);
+        for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
+            const int j0 = vt.kt * BN;
+            const int sb = t % NSB;
+            if (!wait_uniform(&s_full[sb], (t / NSB) & 1)) {
                 ok = false;
                 break;
             }
@@ -367,27 +428,22 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int c = 0; c < BN; c += 32) {
                 uint32_t r[32];
-                tmem_ld32(tl + (k.loc ? COL_SL : COL_SG) + c, r);
-                if (band) {
-                    uint32_t r2[32];
-                    tmem_ld32(tl + COL_SG + c, r2);
+                tmem_ld32(tl + Tm::S + sb * BN + c, r);
 #pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        s[c + e] = (i - (j0 + c + e) < w) ? __uint_as_float(r[e]) : __uint_as_float(r2[e]);
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        s[c + e] = __uint_as_float(r[e]);
-                }
+                for (int e = 0; e < 32; ++e)
+                    s[c + e] = __uint_as_float(r[e]);
             }
             tc_fence_before();
-            mbar_arrive(s_free);
-            // causal mask (tiles reaching past row i0) and rows past the end
-            if (j0 + BN - 1 > i0 || i >= N) {
+            mbar_arrive(&s_free[sb]);
+            // masks: causal (tiles reaching past row i0), the other part of a
+            // band tile, rows past the end
+            if (j0 + BN - 1 > i0 || vt.band || i >= N) {
 #pragma unroll
-                for (int e = 0; e < BN; ++e)
-                    if (j0 + e > i || i >= N)
-                        s[e] = -INFINITY;
+                for (int e = 0; e < BN; ++e) {
+                    const int j = j0 + e;
+                    const bool keep = j <= i && i < N && (!vt.band || ((i - j < w) == vt.loc));
+                    s[e] = keep ? s[e] : -INFINITY;
+                }
             }
             const float mt = tree_max(s) * c2;
             // raise the running max only when it grows by more than the threshold
@@ -405,13 +461,22 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tc_fence_after();
                 }
 #pragma unroll
-                for (int c = 0; c < 64 + DP; c += 16) {
+                for (int c = 0; c < 64; c += 16) {
                     uint32_t r[16];
-                    tmem_ld16(tl + COL_OL + c, r);
+                    tmem_ld16(tl + Tm::OL + c, r);
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
                         r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-                    tmem_st16(tl + COL_OL + c, r);
+                    tmem_st16(tl + Tm::OL + c, r);
+                }
+#pragma unroll
+                for (int c = 0; c < DP; c += 16) {
+                    uint32_t r[16];
+                    tmem_ld16(tl + Tm::OG + c, r);
+#pragma unroll
+                    for (int e = 0; e < 16; ++e)
+                        r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+                    tmem_st16(tl + Tm::OG + c, r);
                 }
                 tmem_wait_st();
             }
@@ -420,11 +485,17 @@ __global__ void __launch_bounds__(kThreads, 2)
                 m_used = mt;
             // P = 2^(s * c2 - m); masked entries (s = -inf) give 0
             const float mneg = m_used == -INFINITY ? 0.f : -m_used;
+            uint32_t pk[BN / 2];
+            float ls = 0.f;
 #pragma unroll
-            for (int e = 0; e < BN; ++e)
-                s[e] = ex2_approx(fmaf(s[e], c2, mneg));
-            l += tree_sum(s);
-            // the PV of the previous tile must be done reading the P buffers
+            for (int e = 0; e < BN; e += 2) {
+                const float p0 = ex2_approx(fmaf(s[e], c2, mneg));
+                const float p1 = ex2_approx(fmaf(s[e + 1], c2, mneg));
+                ls += p0 + p1;
+                pk[e / 2] = pack_bf16(p0, p1);
+            }
+            l += ls;
+            // the PV of the previous virtual tile must be done reading P
             if (t > 0 && pv_waited < t - 1) {
                 if (!wait_uniform(pv_done, (t - 1) & 1)) {
                     ok = false;
@@ -433,39 +504,21 @@ __global__ void __launch_bounds__(kThreads, 2)
                 pv_waited = t - 1;
                 tc_fence_after();
             }
-#pragma unroll
-            for (int c = 0; c < BN / 8; ++c) {
-                float vl[8], vg[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int j = j0 + 8 * c + e;
-                    const bool is_loc = band ? (i - j < w) : k.loc;
-                    vl[e] = is_loc ? s[8 * c + e] : 0.f;
-                    vg[e] = is_loc ? 0.f : s[8 * c + e];
-                }
-                if (k.loc)
-                    st_swz<128>(sm + Ly::PL, row, c,
-                                make_uint4(pack_bf16(vl[0], vl[1]), pack_bf16(vl[2], vl[3]),
-                                           pack_bf16(vl[4], vl[5]), pack_bf16(vl[6], vl[7])));
-                if (k.glob)
-                    st_swz<128>(sm + Ly::PG, row, c,
-                                make_uint4(pack_bf16(vg[0], vg[1]), pack_bf16(vg[2], vg[3]),
-                                           pack_bf16(vg[4], vg[5]), pack_bf16(vg[6], vg[7])));
-            }
-            fence_proxy_async_smem();
+            tmem_st16(tl + Tm::P, *reinterpret_cast<const uint32_t(*)[16]>(&pk[0]));
+            tmem_st16(tl + Tm::P + 16, *reinterpret_cast<const uint32_t(*)[16]>(&pk[16]));
+            tmem_wait_st();
             tc_fence_before();
             mbar_arrive(p_full);
         }
 
         // ---- epilogue: o = (O_loc + O_glob Uv) / l
-        if (ok && wait_uniform(pv_done, (T - 1) & 1)) {
+        if (ok && wait_uniform(pv_done, (VT - 1) & 1)) {
             tc_fence_after();
             float og[DP];
 #pragma unroll
             for (int c = 0; c < DP; c += 16) {
                 uint32_t r[16];
-                tmem_ld16(tl + COL_OG + c, r);
-                tmem_wait_ld();
+                tmem_ld16(tl + Tm::OG + c, r);
 #pragma unroll
                 for (int e = 0; e < 16; ++e)
                     og[c + e] = __uint_as_float(r[e]);
@@ -475,8 +528,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int c = 0; c < 64; c += 16) {
                 uint32_t r[16];
-                tmem_ld16(tl + COL_OL + c, r);
-                tmem_wait_ld();
+                tmem_ld16(tl + Tm::OL + c, r);
                 float o[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
