@@ -15,10 +15,11 @@
 //
 // Warp roles (192 threads): warp 0 issues TMA loads, warp 1 allocates TMEM and
 // issues the MMAs (one thread), warps 2-5 own one query row per thread
-// (TMEM lane = row) for q~, the softmax and the epilogue.  The softmax writes
+// (TMEM lane = row) for the softmax and the epilogue.  q~ is computed by a
+// pre-pass into the first d_down entries of each output row and loaded with Q.  The softmax writes
 // P (bf16) into TMEM with tcgen05.st and the PV products take it from there
 // as their A operand, so P never touches shared memory.  Two S buffers (when
-// d_down <= 32) let S(t+1) run while the softmax works on S(t).  256 TMEM
+// d_down <= 32) let S run two virtual tiles ahead of the softmax.  256 TMEM
 // columns and ~80 KB of shared memory per CTA let two CTAs share an SM, so
 // one CTA's softmax overlaps the other's MMA and load waits.  Every wait is
 // bounded; on a timeout the CTA flags *status and exits.
@@ -41,18 +42,17 @@ constexpr float kRescaleThreshold = 8.0f;  // log2 units: p stays below 2^8 betw
 constexpr uint32_t align_up(uint32_t x, uint32_t a) { return (x + a - 1) / a * a; }
 
 // Tensor-memory columns of one CTA (256 of the SM's 512, two CTAs per SM):
-// S buffers (fp32, BN columns each; two when they fit, so S(t+1) can be
-// computed while the softmax still reads S(t)), O_loc (64), P (bf16 pairs,
-// BN / 2 columns; the A operand of the PV products), O_glob (DP).
+// S buffers (fp32, BN columns each; two when they fit, so S runs two virtual
+// tiles ahead of the softmax), O_loc (64), O_glob (DP) and P (bf16 pairs,
+// BN / 2 columns; the A operand of the PV products).
 template <int DP>
 struct Tmem {
     static constexpr int NSB = DP <= 32 ? 2 : 1;
-    static constexpr uint32_t S = 0;
+    static constexpr uint32_t S = 0;  // buffer b at S + b * BN
     static constexpr uint32_t OL = NSB * BN;
-    static constexpr uint32_t P = 192;
-    static constexpr uint32_t OG = NSB == 2 ? 224 : 128;
-    static_assert(OL + 64 <= P && P + BN / 2 <= (NSB == 2 ? OG : 256) && (NSB == 1 || OG + DP <= kTmemCols),
-                  "tensor-memory columns overlap");
+    static constexpr uint32_t OG = OL + 64;
+    static constexpr uint32_t P = kTmemCols - BN / 2;
+    static_assert(OG + DP <= P, "tensor-memory columns overlap");
 };
 
 // Shared-memory layout (offsets from a 1024-byte aligned base).  A stage holds
@@ -61,15 +61,14 @@ template <int DP>
 struct Layout {
     static constexpr int NS = 3;                          // K/V stages
     static constexpr uint32_t Q = 0;                      // [128][64] bf16, 128B swizzle
-    static constexpr uint32_t QT = BM * 64 * 2;           // [128][DP] bf16
+    static constexpr uint32_t QT = BM * 64 * 2;           // [128][DP] bf16 (q~, loaded by TMA)
     static constexpr uint32_t STG = align_up(QT + BM * DP * 2, 1024);
     static constexpr uint32_t K_OFF = 0;                  // [64][64]
     static constexpr uint32_t V_OFF = BN * 64 * 2;        // [64][64]
     static constexpr uint32_t KD_OFF = 0;                 // [64][DP]
     static constexpr uint32_t VD_OFF = align_up(BN * DP * 2, 1024);
     static constexpr uint32_t STAGE = align_up(2 * BN * 64 * 2, 1024);
-    static constexpr uint32_t UK = STG + NS * STAGE;      // fp32 [DP][64]
-    static constexpr uint32_t UV = UK + DP * 64 * 4;
+    static constexpr uint32_t UV = STG + NS * STAGE;      // fp32 [DP][64]
     static constexpr uint32_t BAR = UV + DP * 64 * 4;
     static constexpr uint32_t TOTAL = BAR + 256;
     static_assert(STAGE % 1024 == 0 && STG % 1024 == 0, "operand tiles must stay 1024-byte aligned");
@@ -108,6 +107,31 @@ __device__ __forceinline__ float tree_max(const float (&v)[N])
         for (int e = 0; e < n; ++e)
             t[e] = fmaxf(t[e], t[e + n]);
     return t[0];
+}
+
+__device__ __forceinline__ float max3(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// Maximum of N values with the 3-input max.f32: four independent running
+// maxima, two new values per step each.
+template <int N>
+__device__ __forceinline__ float tree_max3(const float (&v)[N])
+{
+    float m[4] = {v[0], v[1], v[2], v[3]};
+#pragma unroll
+    for (int e = 4; e + 8 <= N; e += 8)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            m[k] = max3(m[k], v[e + 2 * k], v[e + 2 * k + 1]);
+    constexpr int R = 4 + (N - 4) / 8 * 8;
+#pragma unroll
+    for (int e = R; e < N; ++e)
+        m[e & 3] = fmaxf(m[e & 3], v[e]);
+    return max3(m[0], m[1], fmaxf(m[2], m[3]));
 }
 
 template <int N>
@@ -187,9 +211,10 @@ __device__ __forceinline__ int vt_count(int i0, int i_last, int w)
 
 template <int DP>
 __global__ void __launch_bounds__(kThreads, 2)
-    prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                      const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKD,
-                      const __grid_constant__ CUtensorMap tmVD, PrefillArgs a)
+    prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQT,
+                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                      const __grid_constant__ CUtensorMap tmKD, const __grid_constant__ CUtensorMap tmVD,
+                      PrefillArgs a)
 {
     using Ly = Layout<DP>;
     using Tm = Tmem<DP>;
@@ -202,9 +227,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint64_t *full = bars;                 // [NS] TMA -> MMA
     uint64_t *empty = bars + NS;           // [NS] MMA -> TMA
     uint64_t *s_full = bars + 2 * NS;      // [NSB] S of a virtual tile computed
-    uint64_t *s_free = s_full + NSB;       // [NSB] S read into registers (128 arrivals)
-    uint64_t *q_full = s_free + NSB;       // Q landed
-    uint64_t *qt_ready = q_full + 1;       // q~ written, O zeroed (128 arrivals)
+    uint64_t *q_full = s_full + NSB;       // Q and q~ landed
+    uint64_t *qt_ready = q_full + 1;       // O zeroed (128 arrivals)
     uint64_t *p_full = q_full + 2;         // P written to TMEM (128 arrivals)
     uint64_t *pv_done = q_full + 3;        // PV of a virtual tile finished
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_full + 4);
@@ -223,10 +247,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        for (int s = 0; s < NSB; ++s) {
-            mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], 128);
-        }
+        for (int b2 = 0; b2 < NSB; ++b2)
+            mbar_init(&s_full[b2], 1);
         mbar_init(q_full, 1);
         mbar_init(qt_ready, 128);
         mbar_init(p_full, 128);
@@ -247,12 +269,14 @@ __global__ void __launch_bounds__(kThreads, 2)
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             prefetch_tensormap(&tmQ);
+            prefetch_tensormap(&tmQT);
             prefetch_tensormap(&tmK);
             prefetch_tensormap(&tmV);
             prefetch_tensormap(&tmKD);
             prefetch_tensormap(&tmVD);
-            mbar_expect_tx(q_full, BM * 64 * 2);
+            mbar_expect_tx(q_full, BM * 64 * 2 + BM * DP * 2);
             tma_load_2d(sm + Ly::Q, &tmQ, 0, (b * a.Hq + h) * N + i0, q_full);
+            tma_load_2d(sm + Ly::QT, &tmQT, 0, (b * a.Hq + h) * N + i0, q_full);
             VTile vt = vt_first(i0, i_last, w);
             for (int t = 0; t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
                 const int s = t % NS;
@@ -284,8 +308,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                 const int s = t % NS, sb = t % NSB;
                 if (!mbar_wait(&full[s], (t / NS) & 1, abort_flag))
                     return false;
-                if (t >= NSB && !mbar_wait(&s_free[sb], ((t / NSB) - 1) & 1, abort_flag))
-                    return false;
                 tc_fence_after();
                 const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
                 const uint32_t dS = tmem + Tm::S + sb * BN;
@@ -309,9 +331,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                     return false;
                 tc_fence_after();
                 const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
+                const uint32_t P = tmem + Tm::P;
 #pragma unroll
                 for (int kk = 0; kk < BN / 16; ++kk) {  // P (TMEM, 8 columns per 16 keys) times V / V^D
-                    const uint32_t aP = tmem + Tm::P + kk * 8;
+                    const uint32_t aP = P + kk * 8;
                     if (vt.loc)
                         mma_f16_ts(tmem + Tm::OL, aP, smem_desc(st + Ly::V_OFF + kk * 16 * 128, 16, 1024, kSw128),
                                    idPV, true);
@@ -324,17 +347,19 @@ __global__ void __launch_bounds__(kThreads, 2)
                 mma_commit(&empty[s]);
                 return true;
             };
-            // S(t) is issued as soon as its K tile and an S buffer are free, so
-            // it overlaps the softmax of t-1; PV(t-1) follows once P(t-1) is in TMEM
+            // S runs NSB virtual tiles ahead: S(t + NSB) reuses the buffer of S(t),
+            // which P(t) being written proves the softmax has read
             VTile vs = vt_first(i0, i_last, w), vp = vs;
-            for (int t = 0; ok && t <= VT; ++t) {
-                if (t < VT) {
-                    ok = issue_S(t, vs);
+            for (int t = 0; ok && t < NSB && t < VT; ++t) {
+                ok = issue_S(t, vs);
+                vs = vt_next(vs, i0, i_last, w);
+            }
+            for (int t = 0; ok && t < VT; ++t) {
+                ok = issue_PV(t, vp);
+                vp = vt_next(vp, i0, i_last, w);
+                if (ok && t + NSB < VT) {
+                    ok = issue_S(t + NSB, vs);
                     vs = vt_next(vs, i0, i_last, w);
-                }
-                if (ok && t > 0) {
-                    ok = issue_PV(t - 1, vp);
-                    vp = vt_next(vp, i0, i_last, w);
                 }
             }
         }
@@ -345,13 +370,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int i = i0 + row;
         const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
         const int stid = threadIdx.x - 64;  // 0..127
-        float *sUk = reinterpret_cast<float *>(sm + Ly::UK);
         float *sUv = reinterpret_cast<float *>(sm + Ly::UV);
         for (int idx = stid; idx < DP * 64; idx += 128) {
             const int c = idx / 64, t = idx % 64;
-            const bool in = c < a.dd;
-            sUk[idx] = in ? a.Uk[((size_t)g * a.dd + c) * 64 + t] : 0.f;
-            sUv[idx] = in ? a.Uv[((size_t)g * a.dd + c) * 64 + t] : 0.f;
+            sUv[idx] = c < a.dd ? a.Uv[((size_t)g * a.dd + c) * 64 + t] : 0.f;
         }
         asm volatile("bar.sync 1, 128;" ::: "memory");
         // tcgen05.ld/st are warp-collective: every branch around them is warp-uniform
@@ -360,41 +382,6 @@ __global__ void __launch_bounds__(kThreads, 2)
             return __all_sync(0xffffffffu, r) != 0;
         };
         bool ok = wait_uniform(q_full, 0);
-
-        // q~ row = q Uk^T  (fp32, rounded once to bf16 for the MMA)
-        {
-            float q[64];
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                const uint4 v = ld_swz<128>(sm + Ly::Q, row, c);
-                q[8 * c + 0] = bf16lo(v.x);
-                q[8 * c + 1] = bf16hi(v.x);
-                q[8 * c + 2] = bf16lo(v.y);
-                q[8 * c + 3] = bf16hi(v.y);
-                q[8 * c + 4] = bf16lo(v.z);
-                q[8 * c + 5] = bf16hi(v.z);
-                q[8 * c + 6] = bf16lo(v.w);
-                q[8 * c + 7] = bf16hi(v.w);
-            }
-#pragma unroll 1
-            for (int c8 = 0; c8 < DP / 8; ++c8) {
-                float o[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float *u = sUk + (c8 * 8 + e) * 64;
-                    float a0 = 0.f, a1 = 0.f;
-#pragma unroll
-                    for (int t = 0; t < 64; t += 2) {
-                        a0 = fmaf(q[t], u[t], a0);
-                        a1 = fmaf(q[t + 1], u[t + 1], a1);
-                    }
-                    o[e] = a0 + a1;
-                }
-                st_swz<DP * 2>(sm + Ly::QT, row, c8,
-                               make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]),
-                                          pack_bf16(o[6], o[7])));
-            }
-        }
         {  // zero the accumulators
             uint32_t z[16];
 #pragma unroll
@@ -408,7 +395,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                 tmem_st16(tl + Tm::OG + c, z);
             tmem_wait_st();
         }
-        fence_proxy_async_smem();  // q~ (generic stores) before the MMAs read it
         tc_fence_before();
         mbar_arrive(qt_ready);
 
@@ -425,16 +411,15 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             tc_fence_after();
             float s[BN];
+            {
+                uint32_t r[BN];  // both halves in flight, one wait
+                tmem_ld32_nowait(tl + Tm::S + sb * BN, *reinterpret_cast<uint32_t(*)[32]>(&r[0]));
+                tmem_ld32_nowait(tl + Tm::S + sb * BN + 32, *reinterpret_cast<uint32_t(*)[32]>(&r[32]));
+                tmem_wait_ld_regs(r);
 #pragma unroll
-            for (int c = 0; c < BN; c += 32) {
-                uint32_t r[32];
-                tmem_ld32(tl + Tm::S + sb * BN + c, r);
-#pragma unroll
-                for (int e = 0; e < 32; ++e)
-                    s[c + e] = __uint_as_float(r[e]);
+                for (int e = 0; e < BN; ++e)
+                    s[e] = __uint_as_float(r[e]);
             }
-            tc_fence_before();
-            mbar_arrive(&s_free[sb]);
             // masks: causal (tiles reaching past row i0), the other part of a
             // band tile, rows past the end
             if (j0 + BN - 1 > i0 || vt.band || i >= N) {
@@ -445,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     s[e] = keep ? s[e] : -INFINITY;
                 }
             }
-            const float mt = tree_max(s) * c2;
+            const float mt = tree_max3(s) * c2;
             // raise the running max only when it grows by more than the threshold
             const bool raise = mt > m_used + kRescaleThreshold;
             const bool scale_o = raise && m_used != -INFINITY;
@@ -478,12 +463,12 @@ __global__ void __launch_bounds__(kThreads, 2)
                         r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
                     tmem_st16(tl + Tm::OG + c, r);
                 }
-                tmem_wait_st();
             }
             l *= alpha;
             if (raise)
                 m_used = mt;
-            // P = 2^(s * c2 - m); masked entries (s = -inf) give 0
+            // P = 2^(s * c2 - m) (masked entries give 0); the PV of the previous
+            // virtual tile must be done reading the P columns
             const float mneg = m_used == -INFINITY ? 0.f : -m_used;
             uint32_t pk[BN / 2];
             float ls = 0.f;
@@ -495,7 +480,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                 pk[e / 2] = pack_bf16(p0, p1);
             }
             l += ls;
-            // the PV of the previous virtual tile must be done reading P
             if (t > 0 && pv_waited < t - 1) {
                 if (!wait_uniform(pv_done, (t - 1) & 1)) {
                     ok = false;
@@ -512,6 +496,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
 
         // ---- epilogue: o = (O_loc + O_glob Uv) / l
+        // every PV before the last has been waited for (before writing P)
         if (ok && wait_uniform(pv_done, (VT - 1) & 1)) {
             tc_fence_after();
             float og[DP];
@@ -531,13 +516,23 @@ __global__ void __launch_bounds__(kThreads, 2)
                 tmem_ld16(tl + Tm::OL + c, r);
                 float o[16];
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    float acc = __uint_as_float(r[e]);
+                for (int e = 0; e < 16; ++e)
+                    o[e] = __uint_as_float(r[e]);
 #pragma unroll
-                    for (int kk = 0; kk < DP; ++kk)
-                        acc = fmaf(og[kk], sUv[kk * 64 + c + e], acc);
-                    o[e] = acc * inv;
+                for (int kk = 0; kk < DP; ++kk) {
+                    const float4 *u4 = reinterpret_cast<const float4 *>(sUv + kk * 64 + c);
+#pragma unroll
+                    for (int e4 = 0; e4 < 4; ++e4) {
+                        const float4 u = u4[e4];
+                        o[4 * e4 + 0] = fmaf(og[kk], u.x, o[4 * e4 + 0]);
+                        o[4 * e4 + 1] = fmaf(og[kk], u.y, o[4 * e4 + 1]);
+                        o[4 * e4 + 2] = fmaf(og[kk], u.z, o[4 * e4 + 2]);
+                        o[4 * e4 + 3] = fmaf(og[kk], u.w, o[4 * e4 + 3]);
+                    }
                 }
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                    o[e] *= inv;
                 if (i < N) {
                     uint4 *dst = reinterpret_cast<uint4 *>(orow + c);
                     dst[0] = make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]),
@@ -583,15 +578,16 @@ static EncodeTiledFn encode_fn()
     return fn;
 }
 
-// 2-D bf16 tensor [rows][cols] (row pitch = cols), box [box_rows][cols].
+// 2-D bf16 tensor [rows][cols] with a row pitch of `pitch` elements (0: cols),
+// box [box_rows][cols].
 static bool make_map(CUtensorMap *m, const void *base, unsigned long long rows, int cols, int box_rows,
-                     CUtensorMapSwizzle sw)
+                     CUtensorMapSwizzle sw, int pitch = 0)
 {
     EncodeTiledFn fn = encode_fn();
     if (!fn)
         return false;
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    cuuint64_t strides[1] = {(cuuint64_t)(pitch > 0 ? pitch : cols) * 2};
     cuuint32_t box[2] = {(cuuint32_t)cols, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
@@ -602,12 +598,14 @@ static bool make_map(CUtensorMap *m, const void *base, unsigned long long rows, 
 template <int DP>
 static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
 {
-    CUtensorMap mq, mk, mv, mkd, mvd;
+    CUtensorMap mq, mqt, mk, mv, mkd, mvd;
     const CUtensorMapSwizzle swd = DP == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
                                    : DP == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
                                               : CU_TENSOR_MAP_SWIZZLE_128B;
     const unsigned long long rq = (unsigned long long)a.B * a.Hq * a.N, rk = (unsigned long long)a.B * a.Hkv * a.N;
+    // q~ sits in the first DP entries of each output row (written by the pre-pass)
     if (!make_map(&mq, a.q, rq, 64, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&mqt, a.out, rq, DP, BM, swd, 64) ||
         !make_map(&mk, a.k, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&mv, a.v, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) || !make_map(&mkd, a.kd, rk, DP, BN, swd) ||
         !make_map(&mvd, a.vd, rk, DP, BN, swd))
@@ -622,7 +620,72 @@ static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
         configured = true;
     }
     dim3 grid(a.B * a.Hq, (a.N + BM - 1) / BM);
-    kern<<<grid, kThreads, smem, s>>>(mq, mk, mv, mkd, mvd, a);
+    kern<<<grid, kThreads, smem, s>>>(mq, mqt, mk, mv, mkd, mvd, a);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- q~ pre-pass
+
+// q~ = q Uk^T for every query row (fp32 chains, rounded once to bf16), written
+// into the first DP entries of the row's output slot (entries dd..DP-1 zero):
+// the CTA that owns a row reads its q~ before it writes the row's output.
+// grid (ceil(N / 128), B * Hq), 128 threads, one row per thread.
+template <int DP>
+__global__ void __launch_bounds__(128) qtilde_kernel(const bf16 *__restrict__ q, const float *__restrict__ Uk,
+                                                     bf16 *__restrict__ out, int Hq, int G, int dd, int N)
+{
+    __shared__ __align__(16) float sUk[DP * 64];
+    const int bh = blockIdx.y, g = (bh % Hq) / G;
+    for (int i = threadIdx.x; i < DP * 64; i += blockDim.x)
+        sUk[i] = i / 64 < dd ? Uk[((size_t)g * dd + i / 64) * 64 + i % 64] : 0.f;
+    __syncthreads();
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= N)
+        return;
+    const size_t row = (size_t)bh * N + j;
+    float x[64];
+    const uint4 *q4 = reinterpret_cast<const uint4 *>(q + row * 64);
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        const uint4 v = q4[c];
+        x[8 * c + 0] = bf16lo(v.x);
+        x[8 * c + 1] = bf16hi(v.x);
+        x[8 * c + 2] = bf16lo(v.y);
+        x[8 * c + 3] = bf16hi(v.y);
+        x[8 * c + 4] = bf16lo(v.z);
+        x[8 * c + 5] = bf16hi(v.z);
+        x[8 * c + 6] = bf16lo(v.w);
+        x[8 * c + 7] = bf16hi(v.w);
+    }
+    uint4 *o4 = reinterpret_cast<uint4 *>(out + row * 64);
+#pragma unroll 1
+    for (int c8 = 0; c8 < DP / 8; ++c8) {
+        float o[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float4 *u4 = reinterpret_cast<const float4 *>(sUk + (c8 * 8 + e) * 64);
+            float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+            for (int t4 = 0; t4 < 16; ++t4) {
+                const float4 u = u4[t4];
+                a0 = fmaf(x[4 * t4 + 0], u.x, a0);
+                a1 = fmaf(x[4 * t4 + 1], u.y, a1);
+                a0 = fmaf(x[4 * t4 + 2], u.z, a0);
+                a1 = fmaf(x[4 * t4 + 3], u.w, a1);
+            }
+            o[e] = a0 + a1;
+        }
+        o4[c8] = make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]),
+                            pack_bf16(o[6], o[7]));
+    }
+}
+
+template <int DP>
+static cudaError_t launch_qtilde(const PrefillArgs &a, cudaStream_t s)
+{
+    dim3 grid((a.N + 127) / 128, a.B * a.Hq);
+    qtilde_kernel<DP><<<grid, 128, 0, s>>>(static_cast<const bf16 *>(a.q), a.Uk, static_cast<bf16 *>(a.out), a.Hq,
+                                           a.Hq / a.Hkv, a.dd, a.N);
     return cudaGetLastError();
 }
 
@@ -641,10 +704,11 @@ cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s)
 {
     if (a.B == 0 || a.N == 0)
         return cudaSuccess;
+    cudaError_t e;
     switch (a.kd_stride) {
-    case 16: return tcp::launch_dp<16>(a, s);
-    case 32: return tcp::launch_dp<32>(a, s);
-    case 64: return tcp::launch_dp<64>(a, s);
+    case 16: e = tcp::launch_qtilde<16>(a, s); return e != cudaSuccess ? e : tcp::launch_dp<16>(a, s);
+    case 32: e = tcp::launch_qtilde<32>(a, s); return e != cudaSuccess ? e : tcp::launch_dp<32>(a, s);
+    case 64: e = tcp::launch_qtilde<64>(a, s); return e != cudaSuccess ? e : tcp::launch_dp<64>(a, s);
     default: return cudaErrorInvalidValue;
     }
 }
