@@ -34,6 +34,15 @@ sys.path.insert(0, ROOT)
 METRIC = "decode GB/s & prefill TFLOP/s of DAR attention, % of GB300 roofline (1 GPU)"
 # kernels of one timed step: the cache append, then the decode's prep and stream kernels
 LAUNCHES_PER_STEP = 3
+# DRAM bytes (read + write) of one decode_kernel<bf16,16,1> launch on the
+# decode-160M workload, from an ncu capture of `python bench.py --only decode`
+# (dram__bytes_read.sum + dram__bytes_write.sum); None whenever that kernel
+# has changed since the capture.
+DECODE_TRAFFIC_BYTES = 113_094_656 + 3_339_008
+# multi-function-unit ex2 throughput per SM and the maximum SM clock (the
+# prefill's exponential roofline)
+MUFU_EX2_PER_CLK = 16
+SM_MAX_MHZ = 2070.0
 
 
 def load_peaks():
@@ -190,6 +199,47 @@ def graph_kernel_times(torch, dar, wls, knew, vnew, outs, R, K, stream):
 
 # ----------------------------------------------------------------------------- GPU arm
 
+def prefill_section(args, torch, W, I, dev, stream, tc_peak, peak_src):
+    """Time the 410M-like prefill (B = --prefill-batch, 8 by default) and
+    return its JSON object."""
+    K, Wm = args.steps, args.warmup
+    pcfg = I.PREFILL_410M
+    if args.prefill_batch != pcfg.B:
+        pcfg = I.Prefill(f"{pcfg.name} (B={args.prefill_batch})", pcfg.seed, args.prefill_batch, pcfg.Hq, pcfg.Hkv,
+                         pcfg.N, pcfg.d, pcfg.dd, pcfg.w, pcfg.dtype)
+    pw = W.PrefillWorkload(pcfg)
+    flops = W.prefill_flops(pcfg)
+    for _ in range(max(3, Wm)):
+        pw.run()
+    torch.cuda.synchronize()
+    pk = max(3, min(K, 10))
+    pev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(pk)]
+    for a, b in pev:
+        a.record(stream)
+        pw.run()
+        b.record(stream)
+    torch.cuda.synchronize()
+    p_ms = float(np.mean([a.elapsed_time(b) for a, b in pev]))
+    p_tflops = flops / (p_ms * 1e-3) / 1e12
+    # The prefill is bound by the exponentials of the softmax (one per causal
+    # (query, key) pair), not by its small contractions: 16 ex2 per clock per
+    # SM on the multi-function units, at the maximum SM clock.
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    exps = W.prefill_exps(pcfg)
+    exp_rate = exps / (p_ms * 1e-3) / 1e9
+    exp_peak = sms * MUFU_EX2_PER_CLK * SM_MAX_MHZ * 1e6 / 1e9
+    prefill = {"workload": pcfg.name, "tflops": round(p_tflops, 2), "ms": round(p_ms, 4),
+               "flops_per_call": flops, "exps_per_call": exps,
+               "roofline": {"bound": "alu", "achieved": round(exp_rate, 1), "peak": round(exp_peak, 1),
+                            "unit": "Gexp/s", "frac": round(exp_rate / exp_peak, 4), "traffic": None,
+                            "peak_source": f"{sms} SMs x {MUFU_EX2_PER_CLK} ex2/clk x {SM_MAX_MHZ:.0f} MHz (nominal)"},
+               "tensor": {"achieved": round(p_tflops, 2), "peak": tc_peak, "unit": "TFLOP/s",
+                          "frac": round(p_tflops / tc_peak, 4), "peak_source": f"{peak_src} bf16 dense (burst)"}}
+
+    return prefill
+
+
+
 def run_ours(args, world, rank, local):
     import torch
     from paper_2606_18587_gb300 import dar
@@ -200,6 +250,11 @@ def run_ours(args, world, rank, local):
     dev = torch.device("cuda", local)
     init_dist(world, "nccl")
     hbm_peak, tc_peak, tc_sus, peak_src = load_peaks()
+    if args.only == "prefill":  # profiling aid: the prefill alone
+        pre = prefill_section(args, torch, W, I, dev, torch.cuda.current_stream(), tc_peak, peak_src)
+        if rank == 0:
+            print(json.dumps({"metric": "prefill (profiling run)", "prefill": pre}), flush=True)
+        return
     cfg = I.DECODE_160M
     K, Wm = args.steps, args.warmup
 
@@ -319,27 +374,7 @@ def run_ours(args, world, rank, local):
     h2d = (knew[0].numel() + vnew[0].numel() + wls[0].q.numel()) * knew[0].element_size()
     d2h = outs[0].numel() * outs[0].element_size()
 
-    # ---- prefill (410M-like) on the same GPU
-    pcfg = I.PREFILL_410M
-    pw = W.PrefillWorkload(pcfg)
-    flops = W.prefill_flops(pcfg)
-    for _ in range(max(3, Wm)):
-        pw.run()
-    torch.cuda.synchronize()
-    pk = max(3, min(K, 10))
-    pev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(pk)]
-    for a, b in pev:
-        a.record(stream)
-        pw.run()
-        b.record(stream)
-    torch.cuda.synchronize()
-    p_ms = float(np.mean([a.elapsed_time(b) for a, b in pev]))
-    p_tflops = flops / (p_ms * 1e-3) / 1e12
-    prefill = {"workload": pcfg.name, "tflops": round(p_tflops, 2), "ms": round(p_ms, 4),
-               "flops_per_call": flops, "exps_per_call": W.prefill_exps(pcfg),
-               "roofline": {"bound": "tensor", "achieved": round(p_tflops, 2), "peak": tc_peak, "unit": "TFLOP/s",
-                            "frac": round(p_tflops / tc_peak, 4), "traffic": None,
-                            "peak_source": f"{peak_src} bf16 dense (burst)"}}
+    prefill = None if args.only == "decode" else prefill_section(args, torch, W, I, dev, stream, tc_peak, peak_src)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -359,7 +394,7 @@ def run_ours(args, world, rank, local):
             "e2e": {"value": round(e2e_val, 2), "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": LAUNCHES_PER_STEP * steps_done,
             "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
-                         "frac": round(dec_gbs / hbm_peak, 4), "traffic": None,
+                         "frac": round(dec_gbs / hbm_peak, 4), "traffic": DECODE_TRAFFIC_BYTES,
                          "kernel": "dar_attn_decode (decode_prep_kernel + decode_kernel<bf16,16,1>)",
                          "bytes_per_launch": int(np.mean(dec_bytes)),
                          "us_per_launch": round(1e3 * float(np.mean(dec_ms)), 3),
@@ -416,6 +451,9 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for the CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--only", choices=["all", "decode", "prefill"], default="all",
+                    help="profiling aid: run only the decode step or only the prefill")
+    ap.add_argument("--prefill-batch", type=int, default=8, help="batch of the prefill workload")
     ap.add_argument("--soak-seconds", type=float, default=1.0,
                     help="untimed replays of the step graph just before the timed region (clock sampling)")
     args = ap.parse_args()
