@@ -11,7 +11,7 @@
  *   Eq. 3  k_j, v_j = full if i - j < w, lifted otherwise
  *   Eq. 4  o_i = softmax(q_i K_i^T / sqrt(d_k)) V_i   (one softmax over all j <= i)
  *
- * Readings of the paper that this file encodes (each is listed in the design doc):
+ * Readings of the paper that this file encodes:
  *   - the projections act per KV head on that head's key/value vectors
  *     (W_down = Dk or Dv, W_up = Uk or Uv), with separate matrices for K and V;
  *   - the query/key inputs are already position-encoded (no RoPE here);
