@@ -426,7 +426,8 @@ __device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, in
     if (warp == 0) {
         const int per = (B + 31) / 32;
         const int b0 = min(B, lane * per), b1 = min(B, b0 + per);
-        long long units = 0;
+        // items at the minimum chunk sizes: at most B * Hq * maxc < 2^31 (checked at the boundary)
+        int units = 0;
         for (int b = b0; b < b1; ++b) {
             const int L = s_len[b];
             const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
@@ -435,13 +436,12 @@ __device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, in
 #pragma unroll
         for (int off = 16; off; off >>= 1)
             units += __shfl_xor_sync(0xffffffffu, units, off);
-        const long long target = (long long)gridDim.x * kDecWarps * kItemsPerWarp;
-        long long f = (units * a.Hkv * a.HS + target - 1) / target;
-        const long long fmax = (long long)(64 * kPage) / a.cd;  // a page chunk spans at most 64 pages
-        f = f > fmax ? fmax : f;
-        f = f > kMaxChunkScale ? kMaxChunkScale : f;
-        f = f < 1 ? 1 : f;
-        const int cw = a.cw * (int)f, cd = a.cd * (int)f;
+        const int target = gridDim.x * kDecWarps * kItemsPerWarp;
+        int f = (int)(((unsigned)(units * a.Hkv * a.HS) + target - 1) / (unsigned)target);
+        const int fmax = 64 * kPage / a.cd;  // a page chunk spans at most 64 pages
+        f = min(f, min(fmax, kMaxChunkScale));
+        f = max(f, 1);
+        const int cw = a.cw * f, cd = a.cd * f;
         int mine = 0;
         for (int b = b0; b < b1; ++b) {
             const int L = s_len[b];
@@ -465,7 +465,7 @@ __device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, in
         if (lane == 31)
             s_pre[B] = incl;  // all chunks
         if (lane == 0)
-            *s_f = (int)f;
+            *s_f = f;
     }
     __syncthreads();
     return make_int2(a.cw * *s_f, a.cd * *s_f);
@@ -642,6 +642,8 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     const T *pk = static_cast<const T *>(a.pool_kd);
     const T *pv = static_cast<const T *>(a.pool_vd);
     bool alive = true;
+    // cache pages are read once per call: first out of L2
+    const uint64_t pol = sm100::l2_evict_first_policy();
 
     // ---- issue side.  Items are ordered by sequence, then (KV head, slice)
     // group, then chunk; CTA k owns the contiguous range [lo, hi) and hands it
@@ -745,14 +747,14 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                 const int y = (iss.b * a.Hkv + iss.g) * w + tb;
                 if constexpr (kMma) {  // whole boxes of TPS_W rows, 128-byte swizzle
                     mbar_expect_tx(bar, 2 * TPS_W * kHeadDim * ES + hdr_bytes);
-                    sm100::tma_load_2d_u(smem_u32(dst), &tm_wk, 0, y, bar);
-                    sm100::tma_load_2d_u(smem_u32(dst + kHalf), &tm_wv, 0, y, bar);
+                    sm100::tma_load_2d_hint(smem_u32(dst), &tm_wk, 0, y, bar, pol);
+                    sm100::tma_load_2d_hint(smem_u32(dst + kHalf), &tm_wv, 0, y, bar, pol);
                 } else {
                     const unsigned bytes = (unsigned)(te - tb) * kHeadDim * ES;
                     const size_t off = (size_t)y * kHeadDim;
                     mbar_expect_tx(bar, 2 * bytes + hdr_bytes);
-                    bulk_g2s(dst, wk + off, bytes, bar);
-                    bulk_g2s(dst + kHalf, wv + off, bytes, bar);
+                    sm100::bulk_g2s_hint(dst, wk + off, bytes, bar, pol);
+                    sm100::bulk_g2s_hint(dst + kHalf, wv + off, bytes, bar, pol);
                 }
                 if (hdr_bytes)
                     bulk_g2s(my_hdrs + slot * kHdrBytes, hsrc, hdr_bytes, bar);
@@ -788,13 +790,13 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                         const size_t doff = (size_t)(ptb - tb) * DD * ES;
                         if constexpr (kMma) {  // page (id, g) = DD lines of 128 bytes
                             const int y = (id[j] * a.Hkv + iss.g) * DD + (ptb % kPage) * DD / kHeadDim;
-                            sm100::tma_load_2d_u(smem_u32(dst + doff), &tm_pk, 0, y, bar);
-                            sm100::tma_load_2d_u(smem_u32(dst + kHalf + doff), &tm_pv, 0, y, bar);
+                            sm100::tma_load_2d_hint(smem_u32(dst + doff), &tm_pk, 0, y, bar, pol);
+                            sm100::tma_load_2d_hint(smem_u32(dst + kHalf + doff), &tm_pv, 0, y, bar, pol);
                         } else {
                             const unsigned bytes = (unsigned)(pte - ptb) * DD * ES;
                             const size_t src = (((size_t)id[j] * a.Hkv + iss.g) * kPage + (ptb % kPage)) * DD;
-                            bulk_g2s(dst + doff, pk + src, bytes, bar);
-                            bulk_g2s(dst + kHalf + doff, pv + src, bytes, bar);
+                            sm100::bulk_g2s_hint(dst + doff, pk + src, bytes, bar, pol);
+                            sm100::bulk_g2s_hint(dst + kHalf + doff, pv + src, bytes, bar, pol);
                         }
                     }
                 }
