@@ -91,22 +91,22 @@ dar_status check_cache(const dar_cache *c)
 }
 
 struct DecodeLayout {
-    size_t m, l, acc, qt, counters, total;
+    size_t qt, counters, rec, total;
 };
 
-// Workspace of dar_attn_decode: split-K records for the smallest chunks, the
-// absorbed queries and one counter per (sequence, KV head, head slice) group.
-// Every call rewrites what it reads.
+// Workspace of dar_attn_decode: the absorbed queries, one counter per
+// (sequence, KV head, head slice) group plus the pool's claim counter, and the
+// split-K records of every range the stream kernel can run (one per warp,
+// then the pool chunks).  Every call rewrites what it reads.
 DecodeLayout decode_layout(const dar_cache *c, int Hq, const dar::DecodeGeometry &gm)
 {
     DecodeLayout L;
-    const size_t recs = (size_t)c->B * Hq * gm.maxc;
-    L.m = 0;
-    L.l = L.m + align256(recs * sizeof(float));
-    L.acc = L.l + align256(recs * sizeof(float));
-    L.qt = L.acc + align256(recs * dar::kHeadDim * sizeof(float));
+    L.qt = 0;
     L.counters = L.qt + align256((size_t)c->B * Hq * c->d_down * sizeof(float));
-    L.total = L.counters + align256((size_t)c->B * c->Hkv * gm.HS * sizeof(int32_t));
+    L.rec = L.counters + align256(((size_t)c->B * c->Hkv * gm.HS + 1) * sizeof(int32_t));
+    const size_t ranges = (size_t)dar::kMaxDecodeCtas * dar::kDecodeWarpsPerCta + dar::kDecodePoolChunks;
+    const size_t recs = ranges * 4 * gm.GH;
+    L.total = L.rec + align256(recs * dar::kRecFloats * sizeof(float));
     return L;
 }
 
@@ -207,9 +207,9 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
     dar::DecodeGeometry gm = dar::decode_geometry(cache->dtype, Hq, cache->Hkv, cache->d_down,
                                                   cache->w, cache->max_pages_per_seq);
     DecodeLayout L = decode_layout(cache, Hq, gm);
-    if ((double)cache->B * Hq * gm.maxc >= 2147483647.0)
-        return fail(DAR_ERR_UNSUPPORTED, "B * Hq * chunks = %.0f exceeds the int32 record index",
-                    (double)cache->B * Hq * gm.maxc);
+    if ((double)cache->B * Hq * gm.sph >= 2147483647.0)
+        return fail(DAR_ERR_UNSUPPORTED, "B * Hq * stages = %.0f exceeds the int32 stage index",
+                    (double)cache->B * Hq * gm.sph);
     if (workspace_bytes < L.total)
         return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
     char *ws = static_cast<char *>(workspace);
@@ -225,9 +225,7 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
     a.status = cache->status;
     a.Uk = Uk;
     a.Uv = Uv;
-    a.rec_m = reinterpret_cast<float *>(ws + L.m);
-    a.rec_l = reinterpret_cast<float *>(ws + L.l);
-    a.rec_acc = reinterpret_cast<float *>(ws + L.acc);
+    a.rec = reinterpret_cast<float *>(ws + L.rec);
     a.qt = reinterpret_cast<float *>(ws + L.qt);
     a.counters = reinterpret_cast<int32_t *>(ws + L.counters);
     a.B = cache->B;
@@ -239,9 +237,6 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
     a.w = cache->w;
     a.maxp = cache->max_pages_per_seq;
     a.num_pages = cache->num_pages;
-    a.maxc = gm.maxc;
-    a.cw = gm.cw;
-    a.cd = gm.cd;
     a.qscale = default_scale(scale, cache->d) * kLog2e;
     return from_cuda(dar::launch_decode(cache->dtype, cache->d_down, a,
                                         static_cast<cudaStream_t>(stream)),

@@ -8,19 +8,25 @@
 //           exact by linearity of Eq. 2) and zeroed group counters.  Neither
 //           needs the cache, so this overlaps the kernel before it (normally
 //           the cache append); it waits for that kernel before exiting.
-//  stream   split-K over the sequence.  Every CTA builds the per-sequence
-//           tables (lengths, chunk sizes, chunk counts) in shared memory.
-//           Work items are (sequence b, KV head g, head slice hs, chunk c),
-//           ordered by sequence, group (g, hs) and chunk; chunks 0..nwc-1
-//           cover the ring (full d = 64 keys/values), the rest the pages
-//           (d_down vectors, page aligned).  CTA k owns a contiguous range of
-//           items and its warps take them in order from a shared-memory
-//           counter.  Each item leaves one partial result (running max m, sum
-//           l, unnormalised acc) per head in the workspace.  At its end a CTA
-//           merges the groups it covered completely -- one softmax over all
-//           chunks (Eq. 4), the global part lifted once with Uv,
-//           o = (acc_local + acc_global Uv) / l -- and a group shared with
-//           other CTAs is merged by the CTA that completes its chunk count.
+//  stream   split-K over the sequence, balanced per warp (stream-K).  The
+//           work of a group (sequence b, KV head g, head slice hs) is a run
+//           of stages -- the ring's tokens (full d = 64 keys/values) in
+//           stages of TPS_W tokens, then the pages' tokens (d_down vectors,
+//           page aligned) in stages of TPS_D tokens -- and the groups are laid
+//           end to end, ordered by sequence then group.  Every CTA builds the
+//           per-sequence stage counts and their prefix sums in shared memory.
+//           The first 3/4 of the S stages are split evenly over the NW warps
+//           of the grid (warp k owns [Ss k / NW, Ss (k + 1) / NW)); the rest
+//           is a pool of small chunks that warps claim with an atomic counter
+//           once their own range is done, so that SMs the memory system serves
+//           faster take more of it.  A range cuts groups into parts; within a
+//           part, the ring stages and the page stages each leave one partial
+//           result per head (running max m, sum l, unnormalised acc) in the
+//           range's record slots.  When a part ends, a group that lies inside
+//           the range is merged at once; a group spread over several ranges
+//           is merged by the warp whose atomic completes its stage count.
+//           The merge is one softmax over all parts (Eq. 4) with the global
+//           part lifted once by Uv: o = (acc_local + acc_global Uv) / l.
 //
 // Streaming: every warp owns a ring of kStages shared-memory slots of
 // kSlotBytes (keys in the first half, values in the second) plus a small
@@ -28,11 +34,12 @@
 // 128-byte lines into 128-byte-swizzled tiles for the tensor-core consumer --
 // pages of d_down < 64 are viewed as lines holding 64 / d_down tokens, since
 // boxes of short rows stream markedly slower -- and 1-D bulk copies otherwise;
-// completion counted on the slot's mbarrier) and, with the first stage of an
-// item, copies the item's query rows (q for the ring, q~ for the pages) into
-// the slot's header.  The warp consumes slots in order and refills each one
-// as soon as it has been read, across item boundaries, so it keeps up to
-// kStages * kSlotBytes of cache in flight while it computes.
+// completion counted on the slot's mbarrier) and, with the first stage of a
+// segment, copies the segment's query rows (q for the ring, q~ for the pages)
+// into the slot's header.  The warp consumes slots in order and refills each
+// one as soon as it has been read, across segment boundaries, so it keeps up
+// to kStages * kSlotBytes of cache in flight while it computes.  Cache bytes
+// are loaded with an evict-first L2 policy: they are read once per call.
 //
 // Compute (bf16, d_down >= 16): the two small contractions of a stage run on
 // the tensor cores with warp-level mma.sync m16n8k16 (bf16 in, fp32 out): the
@@ -43,7 +50,7 @@
 // serves a single query head, page stages instead give each lane whole tokens
 // on the CUDA cores (the tensor-core tile would be 15/16 idle).  Other cases
 // (fp32 storage, d_down = 8) use the CUDA cores with LPT lanes per token row.
-// One online softmax (log2 domain) covers an item.
+// One online softmax (log2 domain) covers a segment.
 #include <type_traits>
 
 #include "dar_common.cuh"
@@ -52,15 +59,12 @@
 
 namespace dar {
 
-constexpr int kDecWarps = 8;
+constexpr int kDecWarps = kDecodeWarpsPerCta;
 constexpr int kDecThreads = kDecWarps * 32;
 constexpr int kStages = 3;
 constexpr int kSlotBytes = 8192;
 constexpr int kHalf = kSlotBytes / 2;
 constexpr int kHdrBytes = 1024;     // per slot: up to 4 query rows of 64 fp32
-constexpr int kItemStages = 2;      // stages per minimum-size chunk
-constexpr int kMaxChunkScale = 32;  // chunks grow to at most 32x the minimum
-constexpr int kItemsPerWarp = 6;    // chunk sizes aim at about this many items per warp
 constexpr int kPrepThreads = 256;   // prep block size
 
 static_assert(DAR_DECODE_MAX_BATCH % kDecThreads == 0, "stream threads hold whole groups of sequences");
@@ -103,18 +107,42 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, int32_
     return false;
 }
 
-// A work item: chunk c of (sequence b, KV head g, head slice hs).
-struct Item {
-    int it;  // -1 = none
-    int b, g, h0, window, t0, t1, nst, rec0;
-    int2 pid;  // lane j: ids of the item's pages j and 32 + j
-};
+// Stage metadata a slot carries from the issuing lane to the consumer:
+//   x: group index (b * Hkv * HS + g * HS + hs); y: flags | page mask << 24;
+//   z: valid tokens in the stage.
+constexpr int kMetaRing = 1 << 16;      // a ring stage (else a page stage)
+constexpr int kMetaSegStart = 1 << 17;  // first stage of a segment: query rows in the header
+constexpr int kMetaSegEnd = 1 << 18;    // last stage of a segment: write its records
+constexpr int kMetaPartEnd = 1 << 19;   // last stage of the warp's part of the group
+constexpr int kMetaShared = 1 << 20;    // the group has parts in other warps
+constexpr int kMetaSlot1 = 1 << 21;     // record slot 1 (else 0)
 
-// Stage metadata a slot carries from the issuing lane to the consumer.
-//   x: record index of the item's first head; y: stage | ring << 16 |
-//   last << 17 | page mask << 24; z: valid tokens in the stage.
-constexpr int kMetaRing = 1 << 16;
-constexpr int kMetaLast = 1 << 17;
+// Stages of one group of a sequence of validated length L (-1 or 0: none).
+struct SeqStages {
+    int nwin, ndist;  // ring tokens, page tokens
+    int r, n;         // ring stages, all stages
+};
+template <int TPS_W, int TPS_D>
+__device__ __forceinline__ SeqStages seq_stages(int L, int w)
+{
+    SeqStages q;
+    q.nwin = L > 0 ? min(L, w) : 0;
+    q.ndist = L > 0 ? L - q.nwin : 0;
+    q.r = (q.nwin + TPS_W - 1) / TPS_W;
+    q.n = q.r + (q.ndist + TPS_D - 1) / TPS_D;
+    return q;
+}
+
+// Partial results: record (range, slot, type, head) at
+// rec + (((range * 2 + slot) * 2 + type) * GH + head) * kRecFloats, holding
+// acc[64] (type 0, ring) or acc[d_down] (type 1, pages), then m and l.
+// Slot 0 belongs to a part whose group began before the range, slot 1 to any
+// other part (a group that lies inside the range is merged at once and reuses
+// slot 1 before the range's last part writes it).
+__device__ __forceinline__ float *rec_ptr(float *rec, int range, int slot, int type, int k, int GH)
+{
+    return rec + (size_t)(((range * 2 + slot) * 2 + type) * GH + k) * kRecFloats;
+}
 
 // Dynamic shared memory of the stream kernel for a batch of B sequences:
 // alignment slack, slots, headers, barriers, stage metadata, the tables.
@@ -167,8 +195,8 @@ __global__ void __launch_bounds__(kPrepThreads) decode_prep_kernel(DecodeArgs a)
                 a.qt[(size_t)row * DD + c] = (p[0] + p[1]) + (p[2] + p[3]);
         }
     }
-    const int ngroups = a.B * a.Hkv * a.HS;
-    for (int i = blockIdx.x * kPrepThreads + threadIdx.x; i < ngroups; i += gridDim.x * kPrepThreads)
+    const int ngroups = a.B * a.Hkv * a.HS;  // group counters, then the pool's claim counter
+    for (int i = blockIdx.x * kPrepThreads + threadIdx.x; i <= ngroups; i += gridDim.x * kPrepThreads)
         a.counters[i] = 0;
     sm100::grid_dep_wait();
 }
@@ -403,13 +431,11 @@ __device__ __forceinline__ float reduce_scatter(const float (&o)[DD], int lane)
 
 // Per-sequence tables of one decode call, built by every CTA of the stream
 // kernel into its shared memory: s_len[b] = validated length (-1 if beyond
-// the cache's capacity), s_pre[b] = chunks of the sequences before b
-// (s_pre[B] = all), and the chunk sizes (cw, cd) = f * (minimum sizes), f
-// chosen so that the grid gets about kItemsPerWarp items per warp.  Larger
-// chunks only lower the chunk counts, so the workspace sized for the minimum
-// chunks always fits.  The CTA loads the lengths; warp 0 (a contiguous run of
-// sequences per lane) reduces and scans them.
-__device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, int *s_len, int *s_f)
+// the cache's capacity) and s_pre[b] = stages per group of the sequences
+// before b (s_pre[B] = all).  The CTA loads the lengths; warp 0 (a contiguous
+// run of sequences per lane) scans the stage counts.
+template <int TPS_W, int TPS_D>
+__device__ __forceinline__ void build_tables(const DecodeArgs &a, int *s_pre, int *s_len)
 {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int B = a.B, w = a.w;
@@ -426,28 +452,9 @@ __device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, in
     if (warp == 0) {
         const int per = (B + 31) / 32;
         const int b0 = min(B, lane * per), b1 = min(B, b0 + per);
-        // items at the minimum chunk sizes: at most B * Hq * maxc < 2^31 (checked at the boundary)
-        int units = 0;
-        for (int b = b0; b < b1; ++b) {
-            const int L = s_len[b];
-            const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
-            units += (nwin + a.cw - 1) / a.cw + (ndist + a.cd - 1) / a.cd;
-        }
-#pragma unroll
-        for (int off = 16; off; off >>= 1)
-            units += __shfl_xor_sync(0xffffffffu, units, off);
-        const int target = gridDim.x * kDecWarps * kItemsPerWarp;
-        int f = (int)(((unsigned)(units * a.Hkv * a.HS) + target - 1) / (unsigned)target);
-        const int fmax = 64 * kPage / a.cd;  // a page chunk spans at most 64 pages
-        f = min(f, min(fmax, kMaxChunkScale));
-        f = max(f, 1);
-        const int cw = a.cw * f, cd = a.cd * f;
         int mine = 0;
-        for (int b = b0; b < b1; ++b) {
-            const int L = s_len[b];
-            const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
-            mine += (nwin + cw - 1) / cw + (ndist + cd - 1) / cd;
-        }
+        for (int b = b0; b < b1; ++b)
+            mine += seq_stages<TPS_W, TPS_D>(s_len[b], w).n;
         int incl = mine;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
@@ -457,32 +464,75 @@ __device__ __forceinline__ int2 build_tables(const DecodeArgs &a, int *s_pre, in
         }
         int run = incl - mine;
         for (int b = b0; b < b1; ++b) {
-            const int L = s_len[b];
-            const int nwin = L > 0 ? min(L, w) : 0, ndist = L > 0 ? L - nwin : 0;
             s_pre[b] = run;
-            run += (nwin + cw - 1) / cw + (ndist + cd - 1) / cd;
+            run += seq_stages<TPS_W, TPS_D>(s_len[b], w).n;
         }
         if (lane == 31)
-            s_pre[B] = incl;  // all chunks
-        if (lane == 0)
-            *s_f = f;
+            s_pre[B] = incl;
     }
     __syncthreads();
-    return make_int2(a.cw * *s_f, a.cd * *s_f);
 }
 
-// One (b, h) output row from its chunk records, by one warp:
-// o = (sum_c f_c acc_c[local] + (sum_c f_c acc_c[global]) Uv) / sum_c f_c l_c,
-// f_c = 2^(m_c - max m) (Eq. 4: one softmax over all chunks).  Lane j holds
-// chunk j's (m, l); lane i holds entries 2i, 2i+1 of every chunk's acc.  The
-// loads of the first kCombChunks chunks are issued together.
-constexpr int kCombChunks = 32;
+// The split of the S stages into ranges.  The first Ss stages are divided
+// evenly over the NW warps of the grid (range k < NW = [lo(k), lo(k + 1)),
+// lo(k) = floor(Ss k / NW)); the rest form a pool of NC chunks of C stages
+// (range NW + u = chunk u), which warps that have finished their own range
+// claim one at a time, so that SMs served faster by the memory system take
+// more of them.  Range ids index the record slots.
+struct Split {
+    int S, Ss, NW, C, NC;
+    int q0, r0;  // Ss = q0 NW + r0, so that floor(Ss k / NW) = q0 k + floor(r0 k / NW) in 32 bits
+    __device__ __forceinline__ int lo(int k) const
+    {
+        return k <= NW ? q0 * k + (r0 * k) / NW : min(S, Ss + (k - NW) * C);
+    }
+    __device__ __forceinline__ int owner(int t) const  // the range holding stage t
+    {
+        if (t >= Ss)
+            return NW + (t - Ss) / C;
+        // the last k with lo(k) <= t: a float estimate, then exact steps
+        int k = min(NW - 1, (int)((float)t * (float)NW / (float)Ss));
+        while (k > 0 && lo(k) > t)
+            --k;
+        while (k + 1 < NW && lo(k + 1) <= t)
+            ++k;
+        return k;
+    }
+};
+constexpr int kPoolPercent = 0;                               // share of the stages in the pool
+constexpr int kMaxPoolChunks = kMaxDecodeCtas * kDecWarps * 2;  // pool chunks the records hold
+static_assert(kMaxPoolChunks == kDecodePoolChunks, "record slots of the pool");
 
-template <typename T, int DD>
-__device__ __forceinline__ void combine_row(const DecodeArgs &a, int b, int h, int g, int nwc, int nch, int lane)
+__device__ __forceinline__ Split make_split(int S, int NW)
 {
-    const size_t rec0 = ((size_t)b * a.Hq + h) * a.maxc;
-    const int jmax = min(nch, kCombChunks);
+    Split sp;
+    sp.S = S;
+    sp.NW = NW;
+    const int P = (int)((long long)S * kPoolPercent / 100);
+    sp.C = max(1, (P + kMaxPoolChunks - 1) / kMaxPoolChunks);
+    sp.NC = (P + sp.C - 1) / sp.C;
+    sp.Ss = S - P;
+    sp.q0 = sp.Ss / NW;
+    sp.r0 = sp.Ss - sp.q0 * NW;
+    return sp;
+}
+
+// Merge of group `gid` from the records of every warp part, by one warp:
+// one softmax over all parts (Eq. 4), o = (sum_p f_p acc_p[ring] +
+// (sum_p f_p acc_p[pages]) Uv) / sum_p f_p l_p, f_p = 2^(m_p - max m).  Lane i
+// reads candidate i of a batch of 32 (range wa + i / 2, type i % 2); lane j
+// holds entries 2j, 2j + 1 of the output row.
+template <typename T, int DD, int GH, int TPS_W, int TPS_D>
+__device__ __noinline__ void combine_group(const DecodeArgs &a, const int *s_pre, const int *s_len, int gid,
+                                           Split sp, int lane)
+{
+    const int per_chunk = a.Hkv * a.HS;
+    const int b = gid / per_chunk, gh = gid - b * per_chunk;
+    const int g = gh / a.HS, h0 = g * a.G + (gh - g * a.HS) * GH;
+    const SeqStages sq = seq_stages<TPS_W, TPS_D>(s_len[b], a.w);
+    const int G0 = s_pre[b] * per_chunk + gh * sq.n, G1 = G0 + sq.n, GR = G0 + sq.r;
+    const int wa = sp.owner(G0);
+    const int ncand = 2 * (sp.owner(G1 - 1) - wa + 1);
     // Uv rows in flight with the records (small d_down only: registers)
     constexpr int UVP = DD <= 32 ? DD : 1;
     const float *Uv = a.Uv + (size_t)g * DD * kHeadDim;
@@ -490,83 +540,119 @@ __device__ __forceinline__ void combine_row(const DecodeArgs &a, int b, int h, i
 #pragma unroll
     for (int cc = 0; cc < UVP; ++cc)
         uv[cc] = __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
-    float mj = -INFINITY, lj = 0.f;
-    if (lane < jmax) {
-        mj = __ldcg(a.rec_m + rec0 + lane);
-        lj = __ldcg(a.rec_l + rec0 + lane);
-    }
-    float2 av[kCombChunks];
+    for (int k = 0; k < GH; ++k) {
+        // candidate c0 + lane: its record index, or -1 if the part has no such segment
+        auto cand = [&](int c0) {
+            const int i = c0 + lane;
+            if (i >= ncand)
+                return -1;
+            const int wk = wa + (i >> 1), type = i & 1;
+            const int rlo = sp.lo(wk);
+            const int lo = max(rlo, G0), hi = min(sp.lo(wk + 1), G1);
+            const bool has = type == 0 ? lo < min(hi, GR) : max(lo, GR) < hi;
+            if (!has)
+                return -1;
+            const int slot = G0 < rlo ? 0 : 1;
+            return ((wk * 2 + slot) * 2 + type) * GH + k;
+        };
+        auto acc_of = [&](int rj, int j) {  // lane's entry pair of record rj (candidate j: even ring, odd pages)
+            return rj >= 0 && ((j & 1) == 0 || 2 * lane < DD)
+                       ? __ldcg(reinterpret_cast<const float2 *>(a.rec + (size_t)rj * kRecFloats) + lane)
+                       : make_float2(0.f, 0.f);
+        };
+        // (m, l) by lane; the entries of the first kPre candidates are loaded
+        // with them, before the max is known (later candidates, groups over
+        // more than kPre / 2 ranges, follow one at a time)
+        constexpr int kPre = 16;
+        float2 v[kPre];
+        int r0 = -1;
+        float m0 = -INFINITY, l0 = 0.f, M = -INFINITY;
+        for (int c0 = 0; c0 < ncand; c0 += 32) {
+            const int r = cand(c0);
+            float mr = -INFINITY, lr = 0.f;
+            if (r >= 0) {
+                const float2 ml = __ldcg(reinterpret_cast<const float2 *>(a.rec + (size_t)r * kRecFloats + kHeadDim));
+                mr = ml.x;
+                lr = ml.y;
+            }
+            if (c0 == 0) {
+                r0 = r;
+                m0 = mr;
+                l0 = lr;
 #pragma unroll
-    for (int j = 0; j < kCombChunks; ++j)
-        av[j] = j < jmax ? __ldcg(reinterpret_cast<const float2 *>(a.rec_acc + (rec0 + j) * kHeadDim) + lane)
-                         : make_float2(0.f, 0.f);
-    // entries past a page chunk's d_down values are never combined: they may hold anything
-    float M = mj;
-    for (int c0 = kCombChunks; c0 < nch; c0 += 32)
-        if (c0 + lane < nch)
-            M = fmaxf(M, __ldcg(a.rec_m + rec0 + c0 + lane));
+                for (int j = 0; j < kPre; ++j)
+                    v[j] = acc_of(__shfl_sync(0xffffffffu, r, j), j);
+            }
+            M = fmaxf(M, mr);
+        }
 #pragma unroll
-    for (int off = 16; off; off >>= 1)
-        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    float o0 = 0.f, o1 = 0.f, gd0 = 0.f, gd1 = 0.f;
-    const float f0 = lane < jmax ? exp2f(mj - M) : 0.f;
-    float lsum = f0 * lj;
+        for (int off = 16; off; off >>= 1)
+            M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        float o0 = 0.f, o1 = 0.f, gd0 = 0.f, gd1 = 0.f, lsum = 0.f;
+        auto add = [&](float fj, float2 x, int j) {
+            if ((j & 1) == 0) {
+                o0 = fmaf(fj, x.x, o0);
+                o1 = fmaf(fj, x.y, o1);
+            } else {
+                gd0 = fmaf(fj, x.x, gd0);
+                gd1 = fmaf(fj, x.y, gd1);
+            }
+        };
+        for (int c0 = 0; c0 < ncand; c0 += 32) {
+            int r = r0;
+            float mr = m0, lr = l0;
+            if (c0 > 0) {
+                r = cand(c0);
+                mr = -INFINITY;
+                lr = 0.f;
+                if (r >= 0) {
+                    const float2 ml =
+                        __ldcg(reinterpret_cast<const float2 *>(a.rec + (size_t)r * kRecFloats + kHeadDim));
+                    mr = ml.x;
+                    lr = ml.y;
+                }
+            }
+            const float f = r >= 0 ? exp2f(mr - M) : 0.f;
+            lsum = fmaf(f, lr, lsum);
+            int j0 = 0;
+            if (c0 == 0) {
 #pragma unroll
-    for (int j = 0; j < kCombChunks; ++j) {
-        const float fj = __shfl_sync(0xffffffffu, f0, j);
-        if (j < jmax) {
-            if (j < nwc) {
-                o0 = fmaf(fj, av[j].x, o0);
-                o1 = fmaf(fj, av[j].y, o1);
-            } else if (2 * lane < DD) {
-                gd0 = fmaf(fj, av[j].x, gd0);
-                gd1 = fmaf(fj, av[j].y, gd1);
+                for (int j = 0; j < kPre; ++j)
+                    add(__shfl_sync(0xffffffffu, f, j), v[j], j);
+                j0 = kPre;
+            }
+            const unsigned live = __ballot_sync(0xffffffffu, r >= 0);
+            for (int j = j0; j < 32; ++j) {
+                if (!((live >> j) & 1u))
+                    continue;
+                const float fj = __shfl_sync(0xffffffffu, f, j);
+                add(fj, acc_of(__shfl_sync(0xffffffffu, r, j), j), j);
             }
         }
-    }
-    for (int c0 = kCombChunks; c0 < nch; c0 += 32) {  // long sequences with small chunks
-        float f = 0.f;
-        if (c0 + lane < nch) {
-            f = exp2f(__ldcg(a.rec_m + rec0 + c0 + lane) - M);
-            lsum = fmaf(f, __ldcg(a.rec_l + rec0 + c0 + lane), lsum);
-        }
-        const int jn = min(32, nch - c0);
-        for (int j = 0; j < jn; ++j) {
-            const float fj = __shfl_sync(0xffffffffu, f, j);
-            const int cc = c0 + j;
-            const float2 v = __ldcg(reinterpret_cast<const float2 *>(a.rec_acc + (rec0 + cc) * kHeadDim) + lane);
-            if (cc < nwc) {
-                o0 = fmaf(fj, v.x, o0);
-                o1 = fmaf(fj, v.y, o1);
-            } else if (2 * lane < DD) {
-                gd0 = fmaf(fj, v.x, gd0);
-                gd1 = fmaf(fj, v.y, gd1);
-            }
-        }
-    }
 #pragma unroll
-    for (int off = 16; off; off >>= 1)
-        lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
-    // lift the global part once: o += gd Uv[g]   (gd[c] sits in lane c / 2)
+        for (int off = 16; off; off >>= 1)
+            lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+        // lift the global part once: o += gd Uv[g]   (gd[c] sits in lane c / 2)
 #pragma unroll
-    for (int cc = 0; cc < DD; ++cc) {
-        const float gv = __shfl_sync(0xffffffffu, (cc & 1) ? gd1 : gd0, cc >> 1);
-        const float2 u2 = UVP == DD ? uv[cc < UVP ? cc : 0]
-                                    : __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
-        o0 = fmaf(gv, u2.x, o0);
-        o1 = fmaf(gv, u2.y, o1);
+        for (int cc = 0; cc < DD; ++cc) {
+            const float gv = __shfl_sync(0xffffffffu, (cc & 1) ? gd1 : gd0, cc >> 1);
+            const float2 u2 = UVP == DD ? uv[cc < UVP ? cc : 0]
+                                        : __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
+            o0 = fmaf(gv, u2.x, o0);
+            o1 = fmaf(gv, u2.y, o1);
+        }
+        const float inv = 1.f / lsum;
+        T *orow = static_cast<T *>(a.out) + ((size_t)b * a.Hq + h0 + k) * kHeadDim;
+        orow[2 * lane] = from_f32<T>(o0 * inv);
+        orow[2 * lane + 1] = from_f32<T>(o1 * inv);
     }
-    const float inv = 1.f / lsum;
-    T *orow = static_cast<T *>(a.out) + ((size_t)b * a.Hq + h) * kHeadDim;
-    orow[2 * lane] = from_f32<T>(o0 * inv);
-    orow[2 * lane + 1] = from_f32<T>(o1 * inv);
 }
 
 template <typename T, int DD, int GH>
 __global__ void __launch_bounds__(kDecThreads, 1)
     decode_kernel(const __grid_constant__ CUtensorMap tm_wk, const __grid_constant__ CUtensorMap tm_wv,
                   const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv,
-                  DecodeArgs a)
+                  const __grid_constant__ DecodeArgs a)
 {
     constexpr int E = Granule<T>::kElems;
     constexpr int ES = sizeof(T);
@@ -590,18 +676,14 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     int4 *meta = reinterpret_cast<int4 *>(bars + kDecWarps * kStages);
     int *s_pre = reinterpret_cast<int *>(meta + kDecWarps * kStages);  // [B + 1]
     int *s_len = s_pre + a.B + 1;                                      // [B]
-    __shared__ int s_f;
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     unsigned char *my_slots = slots + (size_t)warp * kStages * kSlotBytes;
     unsigned char *my_hdrs = hdrs + (size_t)warp * kStages * kHdrBytes;
     uint64_t *my_bars = bars + warp * kStages;
     int4 *my_meta = meta + warp * kStages;
-    __shared__ int s_next;  // this CTA's item counter
     if (lane < kStages)
         mbar_init(&my_bars[lane], 1);
-    if (threadIdx.x == 0)
-        s_next = 0;
     sm100::mbar_init_fence();
     __syncthreads();
     if constexpr (kMma) {
@@ -623,8 +705,7 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     // everything below reads the cache and q~ (the prep kernel waited for the
     // kernel before it, so both are final)
     sm100::grid_dep_wait();
-    const int2 chunk = build_tables(a, s_pre, s_len, &s_f);
-    const int cw = chunk.x, cd = chunk.y;
+    build_tables<TPS_W, TPS_D>(a, s_pre, s_len);
     if (blockIdx.x == 0) {  // sequences with nothing to attend to get a zero output
         T *out = static_cast<T *>(a.out);
         for (int b = warp; b < a.B; b += kDecWarps) {
@@ -641,110 +722,130 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     const T *wv = static_cast<const T *>(a.win_v);
     const T *pk = static_cast<const T *>(a.pool_kd);
     const T *pv = static_cast<const T *>(a.pool_vd);
-    bool alive = true;
     // cache pages are read once per call: first out of L2
     const uint64_t pol = sm100::l2_evict_first_policy();
+    bool alive = true;
 
-    // ---- issue side.  Items are ordered by sequence, then (KV head, slice)
-    // group, then chunk; CTA k owns the contiguous range [lo, hi) and hands it
-    // to its warps in order from a shared-memory counter.  An item is decoded
-    // from the tables; the block-table ids of its pages are loaded two items
-    // before they are used (`iss` is being copied in, `nxt` and `nn` follow).
+    // ---- the range being issued (first this warp's own, then pool chunks)
+    // and the walk over it: sequence wb, group wgh of the sequence, stage wj
+    // of the group (the ring's sq.r stages, then the pages')
     const int per_chunk = a.Hkv * a.HS;
-    const int items = s_pre[a.B] * per_chunk;
-    const int lo = (int)((long long)blockIdx.x * items / gridDim.x);
-    const int hi = (int)((long long)(blockIdx.x + 1) * items / gridDim.x);
-    auto seq_of = [&](int it) {  // the sequence whose items include `it`
-        int lb = 0, hb = a.B;
+    const Split sp = make_split(s_pre[a.B] * per_chunk, gridDim.x * kDecWarps);
+    int32_t *pool_next = a.counters + a.B * per_chunk;  // the pool's claim counter
+    int rid = blockIdx.x * kDecWarps + warp;
+    int lo = sp.lo(rid), hi = sp.lo(rid + 1);
+    int iss_s = lo;  // next stage to issue
+    int wb = 0, wgh = 0, wj = 0;
+    SeqStages sq = {0, 0, 0, 1};
+    auto begin_range = [&]() {  // the walk's position at stage lo
+        int lb = 0, hb = a.B;   // the last sequence whose first stage is <= lo
         while (hb - lb > 1) {
             const int mid = (lb + hb) >> 1;
-            if (s_pre[mid] * per_chunk <= it)
+            if (s_pre[mid] * per_chunk <= lo)
                 lb = mid;
             else
                 hb = mid;
         }
-        return lb;
+        wb = lb;
+        sq = seq_stages<TPS_W, TPS_D>(s_len[wb], w);
+        const int r0 = lo - s_pre[wb] * per_chunk;
+        wgh = r0 / sq.n;
+        wj = r0 - wgh * sq.n;
     };
-    auto fetch_item = [&](int it) {
-        Item I;
-        I.it = -1;
-        I.b = I.g = I.h0 = I.window = I.t0 = I.t1 = I.nst = I.rec0 = 0;
-        I.pid = make_int2(-1, -1);
-        if (it < hi) {
-            const int b = seq_of(it);
-            const int nch = s_pre[b + 1] - s_pre[b];
-            const int r = it - s_pre[b] * per_chunk;
-            const int gh = r / nch, c = r % nch;
-            const int L = s_len[b], nwin = min(L, w), ndist = L - nwin;
-            const int nwc = (nwin + cw - 1) / cw;
-            I.it = it;
-            I.b = b;
-            I.g = gh / a.HS;
-            I.h0 = I.g * a.G + (gh % a.HS) * a.GH;
-            if (c < nwc) {
-                I.window = 1;
-                I.t0 = c * cw;
-                I.t1 = min(nwin, I.t0 + cw);
-                I.nst = (I.t1 - I.t0 + TPS_W - 1) / TPS_W;
-            } else {
-                I.t0 = (c - nwc) * cd;
-                I.t1 = min(ndist, I.t0 + cd);
-                I.nst = (I.t1 - I.t0 + TPS_D - 1) / TPS_D;
-                const int p0 = I.t0 / kPage, np = (I.t1 - 1) / kPage - p0 + 1;
-                const int32_t *bt = a.block_table + (size_t)b * a.maxp + p0;
-                if (lane < np)
-                    I.pid.x = __ldg(bt + lane);
-                if (lane + 32 < np)
-                    I.pid.y = __ldg(bt + lane + 32);
-            }
-            I.rec0 = (b * a.Hq + I.h0) * a.maxc + c;
-        }
-        return I;
+    // block-table window: lane j holds the ids of pages pw0 + j and pw0 + 32 + j of sequence pwb
+    int pwb = -1, pw0 = 0;
+    int2 pid = make_int2(-1, -1);
+    auto load_window = [&](int b, int p0) {
+        pwb = b;
+        pw0 = p0;
+        const int32_t *bt = a.block_table + (size_t)b * a.maxp;
+        pid.x = p0 + lane < a.maxp ? __ldg(bt + p0 + lane) : -1;
+        pid.y = p0 + 32 + lane < a.maxp ? __ldg(bt + p0 + 32 + lane) : -1;
     };
-    auto next_index = [&]() {
-        int v = 0;
+    auto page_id = [&](int p) {  // page p of sequence pwb, inside the window
+        const int j = p - pw0;
+        const int x = __shfl_sync(0xffffffffu, pid.x, j & 31);
+        const int y = __shfl_sync(0xffffffffu, pid.y, j & 31);
+        return j < 32 ? x : y;
+    };
+    auto window_for_range = [&]() {  // a range that opens in a page run: fetch its ids now
+        if (wj >= sq.r)
+            load_window(wb, (wj - sq.r) * TPS_D / kPage);
+    };
+    // pool claims: lane 0 asks for the next chunk while issuing the last stages
+    // of a range (two stages ahead), and the warp moves on to the claimed
+    // chunk as soon as that range's last stage is issued
+    int claim = 0;
+    bool asked = false, pool_done = sp.NC == 0;
+    auto ask = [&]() {
         if (lane == 0)
-            v = lo + atomicAdd(&s_next, 1);
-        return __shfl_sync(0xffffffffu, v, 0);
+            claim = atomicAdd(pool_next, 1);
+        asked = true;
     };
-    Item iss = fetch_item(next_index());
-    Item nxt = iss.it >= 0 ? fetch_item(next_index()) : fetch_item(hi);
-    Item nn = nxt.it >= 0 ? fetch_item(next_index()) : fetch_item(hi);
+    int ask_at = max(lo, hi - 2);
+    auto next_range = [&]() {
+        if (pool_done)
+            return;
+        if (!asked)
+            ask();
+        const int c = __shfl_sync(0xffffffffu, claim, 0);
+        asked = false;
+        if (c >= sp.NC) {
+            pool_done = true;
+            return;
+        }
+        rid = sp.NW + c;
+        lo = sp.lo(rid);
+        hi = sp.lo(rid + 1);
+        iss_s = lo;
+        ask_at = max(lo, hi - 2);
+        begin_range();
+        window_for_range();
+    };
+    if (lo < hi) {
+        begin_range();
+        window_for_range();
+    } else {
+        next_range();  // no own stages (tiny workloads): straight to the pool
+    }
 
-    int iss_s = 0;
     int issued = 0, consumed = 0;    // stages issued / consumed by this warp
     int iss_slot = 0, con_slot = 0;  // ring positions
     unsigned con_phase = 0;          // parity of the consumer's current pass over the ring
-    auto page_id = [&](int j) {      // page j (0..63) of the item being issued
-        const int x = __shfl_sync(0xffffffffu, iss.pid.x, j & 31);
-        const int y = __shfl_sync(0xffffffffu, iss.pid.y, j & 31);
-        return j < 32 ? x : y;
-    };
 
-    auto issue_one = [&]() {  // copy the next stage of `iss` into its slot
+    auto issue_one = [&]() {  // copy stage iss_s into its slot
         const int slot = iss_slot;
         iss_slot = iss_slot + 1 == kStages ? 0 : iss_slot + 1;
         unsigned char *dst = my_slots + (size_t)slot * kSlotBytes;
         uint64_t *bar = &my_bars[slot];
-        const int s = iss_s;
-        const int info = s | (s + 1 == iss.nst ? kMetaLast : 0);
-        // the item's query rows travel with its first stage
+        const bool ring = wj < sq.r;
+        const int G0 = iss_s - wj, G1 = G0 + sq.n;
+        const bool seg_start = iss_s == lo || wj == 0 || wj == sq.r;
+        const bool seg_end = iss_s == hi - 1 || wj == sq.n - 1 || wj == sq.r - 1;
+        const bool part_end = iss_s == hi - 1 || wj == sq.n - 1;
+        int flags = (ring ? kMetaRing : 0) | (seg_start ? kMetaSegStart : 0) | (seg_end ? kMetaSegEnd : 0) |
+                    (part_end ? kMetaPartEnd : 0) | (G0 < lo || G1 > hi ? kMetaShared : 0) |
+                    (G0 < lo ? 0 : kMetaSlot1);
+        const int g = wgh / a.HS;
+        const int h0 = g * a.G + (wgh - g * a.HS) * GH;
+        const int gid = wb * per_chunk + wgh;
+        // a segment's query rows travel with its first stage
         unsigned hdr_bytes = 0;
         const void *hsrc = nullptr;
-        if (s == 0) {
-            if (iss.window) {
+        if (seg_start) {
+            if (ring) {
                 hdr_bytes = GH * kHeadDim * ES;
-                hsrc = qg + ((size_t)iss.b * a.Hq + iss.h0) * kHeadDim;
+                hsrc = qg + ((size_t)wb * a.Hq + h0) * kHeadDim;
             } else {
                 hdr_bytes = GH * DD * 4;
-                hsrc = a.qt + ((size_t)iss.b * a.Hq + iss.h0) * DD;
+                hsrc = a.qt + ((size_t)wb * a.Hq + h0) * DD;
             }
         }
-        if (iss.window) {
-            const int tb = iss.t0 + s * TPS_W, te = min(iss.t1, tb + TPS_W);
+        if (ring) {
+            const int tb = wj * TPS_W, te = min(sq.nwin, tb + TPS_W);
             if (lane == 0) {
-                my_meta[slot] = make_int4(iss.rec0, info | kMetaRing | (0xff << 24), te - tb, 0);
-                const int y = (iss.b * a.Hkv + iss.g) * w + tb;
+                my_meta[slot] = make_int4(gid, flags | (0xff << 24), te - tb, rid);
+                const int y = (wb * a.Hkv + g) * w + tb;
                 if constexpr (kMma) {  // whole boxes of TPS_W rows, 128-byte swizzle
                     mbar_expect_tx(bar, 2 * TPS_W * kHeadDim * ES + hdr_bytes);
                     sm100::tma_load_2d_hint(smem_u32(dst), &tm_wk, 0, y, bar, pol);
@@ -760,15 +861,17 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                     bulk_g2s(my_hdrs + slot * kHdrBytes, hsrc, hdr_bytes, bar);
             }
         } else {
-            const int tb = iss.t0 + s * TPS_D, te = min(iss.t1, tb + TPS_D);
-            const int pfirst = tb / kPage - iss.t0 / kPage;  // index within the item's pages
+            const int tb = (wj - sq.r) * TPS_D, te = min(sq.ndist, tb + TPS_D);
+            const int pfirst = tb / kPage;
+            if (pwb != wb || pfirst < pw0 || pfirst + PPS > pw0 + 64)
+                load_window(wb, pfirst);
             int id[PPS];
             unsigned mask = 0, total = 0;
 #pragma unroll
             for (int j = 0; j < PPS; ++j) {
                 id[j] = page_id(pfirst + j);
-                const int ptb = max(tb, (tb / kPage + j) * kPage);
-                const int pte = min(te, (tb / kPage + j + 1) * kPage);
+                const int ptb = max(tb, (pfirst + j) * kPage);
+                const int pte = min(te, (pfirst + j + 1) * kPage);
                 if (pte > ptb) {
                     if (id[j] >= 0 && id[j] < a.num_pages) {
                         mask |= 1u << j;
@@ -780,21 +883,21 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                 }
             }
             if (lane == 0) {
-                my_meta[slot] = make_int4(iss.rec0, info | (int)(mask << 24), te - tb, 0);
+                my_meta[slot] = make_int4(gid, flags | (int)(mask << 24), te - tb, rid);
                 mbar_expect_tx(bar, 2 * total + hdr_bytes);
 #pragma unroll
                 for (int j = 0; j < PPS; ++j) {
                     if ((mask >> j) & 1u) {
-                        const int ptb = max(tb, (tb / kPage + j) * kPage);
-                        const int pte = min(te, (tb / kPage + j + 1) * kPage);
+                        const int ptb = max(tb, (pfirst + j) * kPage);
+                        const int pte = min(te, (pfirst + j + 1) * kPage);
                         const size_t doff = (size_t)(ptb - tb) * DD * ES;
                         if constexpr (kMma) {  // page (id, g) = DD lines of 128 bytes
-                            const int y = (id[j] * a.Hkv + iss.g) * DD + (ptb % kPage) * DD / kHeadDim;
+                            const int y = (id[j] * a.Hkv + g) * DD + (ptb % kPage) * DD / kHeadDim;
                             sm100::tma_load_2d_hint(smem_u32(dst + doff), &tm_pk, 0, y, bar, pol);
                             sm100::tma_load_2d_hint(smem_u32(dst + kHalf + doff), &tm_pv, 0, y, bar, pol);
                         } else {
                             const unsigned bytes = (unsigned)(pte - ptb) * DD * ES;
-                            const size_t src = (((size_t)id[j] * a.Hkv + iss.g) * kPage + (ptb % kPage)) * DD;
+                            const size_t src = (((size_t)id[j] * a.Hkv + g) * kPage + (ptb % kPage)) * DD;
                             sm100::bulk_g2s_hint(dst + doff, pk + src, bytes, bar, pol);
                             sm100::bulk_g2s_hint(dst + kHalf + doff, pv + src, bytes, bar, pol);
                         }
@@ -806,17 +909,22 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         }
         __syncwarp();
         ++issued;
-        if (++iss_s == iss.nst) {  // move on to the next item
-            iss = nxt;
-            iss_s = 0;
-            if (iss.it >= 0) {
-                nxt = nn;
-                nn = nxt.it >= 0 ? fetch_item(next_index()) : fetch_item(hi);
+        if (iss_s == ask_at && !pool_done && !asked)
+            ask();  // the pool chunk after this range
+        // step the walk to the next stage of the range, or to the next range
+        if (++iss_s == hi) {
+            next_range();
+        } else if (++wj == sq.n) {
+            wj = 0;
+            if (++wgh == per_chunk) {
+                wgh = 0;
+                do {
+                    ++wb;
+                } while (s_pre[wb + 1] == s_pre[wb]);  // sequences without stages
+                sq = seq_stages<TPS_W, TPS_D>(s_len[wb], w);
             }
         }
     };
-    while (issued - consumed < kStages && iss.it >= 0)
-        issue_one();
 
     // ---- consume side
     // tensor-core consumer state: A fragments of q (ring) or q~ (pages), output
@@ -838,7 +946,125 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         for (int e = 0; e < E; ++e)
             acc[k][e] = qr[k][e] = 0.f;
     }
-    while (consumed < issued) {
+    int4 pend = make_int4(0, 0, 0, 0);  // metadata of the last stage consumed, if it ends a segment
+    // Shared parts finished by this warp: lane i holds the group and stage
+    // count of the i-th.  Their counts are added together (after one fence)
+    // when the warp runs out of work, so the streaming never waits on them; a
+    // count that completes its group's stages makes this warp merge the group.
+    int pg = 0, pp = 0, npend = 0;
+    auto flush = [&]() {
+        if (npend == 0)
+            return;
+        __threadfence();  // this warp's records, GPU-wide, before its counts
+        bool fin = false;
+        if (lane < npend) {
+            const int old = atomicAdd(a.counters + pg, pp);
+            fin = old + pp == seq_stages<TPS_W, TPS_D>(s_len[pg / per_chunk], w).n;
+        }
+        unsigned fm = __ballot_sync(0xffffffffu, fin);
+        if (fm)
+            __threadfence();  // the other parts' records
+        while (fm) {
+            const int j = __ffs(fm) - 1;
+            fm &= fm - 1;
+            combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, __shfl_sync(0xffffffffu, pg, j), sp, lane);
+        }
+        npend = 0;
+    };
+    for (;;) {
+        // refill first, so that the copies run while a finished segment is written
+        while (issued - consumed < kStages && iss_s < hi)
+            issue_one();
+        if (pend.y & kMetaSegEnd) {
+            // ---- segment done: write the partial result (m, l, acc) of every head
+            const bool win = (pend.y & kMetaRing) != 0;
+            float *rec0 = rec_ptr(a.rec, pend.w, (pend.y & kMetaSlot1) ? 1 : 0, win ? 0 : 1, 0, GH);
+            if (kLanePages && !win) {
+                if constexpr (kLanePages) {
+#pragma unroll
+                    for (int off = 16; off; off >>= 1)
+                        lp += __shfl_xor_sync(0xffffffffu, lp, off);
+                    const float tot = reduce_scatter<DD>(ol, lane);
+                    constexpr int LPE = 32 / DD;  // lanes holding each entry
+                    if (lane % LPE == 0)
+                        rec0[lane / LPE] = tot;
+                    if (lane == 0)
+                        *reinterpret_cast<float2 *>(rec0 + kHeadDim) = make_float2(mm, lp);
+                }
+            } else if constexpr (kMma) {
+                lp += __shfl_xor_sync(0xffffffffu, lp, 1);
+                lp += __shfl_xor_sync(0xffffffffu, lp, 2);
+                const int g = lane >> 2, c = lane & 3;
+                if (g < GH) {
+                    float *ra = rec0 + (size_t)g * kRecFloats;
+                    if (win) {
+#pragma unroll
+                        for (int d = 0; d < 8; ++d)
+                            *reinterpret_cast<float2 *>(ra + 8 * d + 2 * c) = make_float2(ow[d][0], ow[d][1]);
+                    } else {
+#pragma unroll
+                        for (int d = 0; d < NDD; ++d)
+                            *reinterpret_cast<float2 *>(ra + 8 * d + 2 * c) = make_float2(od[d][0], od[d][1]);
+                    }
+                    if (c == 0)
+                        *reinterpret_cast<float2 *>(ra + kHeadDim) = make_float2(mm, lp);
+                }
+            } else {
+                const int LPTc = (win ? kHeadDim : DD) / E;
+                for (int off = LPTc; off < 32; off <<= 1) {
+#pragma unroll
+                    for (int k = 0; k < GH; ++k) {
+                        const float mo = __shfl_xor_sync(0xffffffffu, m[k], off);
+                        const float lo2 = __shfl_xor_sync(0xffffffffu, l[k], off);
+                        const float mn = fmaxf(m[k], mo);
+                        const float fa = (m[k] == -INFINITY) ? 0.f : exp2f(m[k] - mn);
+                        const float fb = (mo == -INFINITY) ? 0.f : exp2f(mo - mn);
+                        l[k] = l[k] * fa + lo2 * fb;
+#pragma unroll
+                        for (int e = 0; e < E; ++e) {
+                            const float ao = __shfl_xor_sync(0xffffffffu, acc[k][e], off);
+                            acc[k][e] = acc[k][e] * fa + ao * fb;
+                        }
+                        m[k] = mn;
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < GH; ++k) {
+                    float *ra = rec0 + (size_t)k * kRecFloats;
+                    if (lane < LPTc) {
+                        float4 *dstv = reinterpret_cast<float4 *>(ra + lane * E);
+#pragma unroll
+                        for (int e4 = 0; e4 < E / 4; ++e4)
+                            dstv[e4] = make_float4(acc[k][4 * e4], acc[k][4 * e4 + 1], acc[k][4 * e4 + 2],
+                                                   acc[k][4 * e4 + 3]);
+                    }
+                    if (lane == 0)
+                        *reinterpret_cast<float2 *>(ra + kHeadDim) = make_float2(m[k], l[k]);
+                }
+            }
+            if (pend.y & kMetaPartEnd) {
+                // ---- the range's part of the group is done
+                if (pend.y & kMetaShared) {  // counted later, with the warp's other shared parts
+                    const int gid = pend.x;
+                    const int b = gid / per_chunk, gh = gid - b * per_chunk;
+                    const SeqStages gq = seq_stages<TPS_W, TPS_D>(s_len[b], w);
+                    const int G0 = s_pre[b] * per_chunk + gh * gq.n;
+                    if (lane == npend) {
+                        pg = gid;
+                        pp = min(sp.lo(pend.w + 1), G0 + gq.n) - max(sp.lo(pend.w), G0);
+                    }
+                    if (++npend == 32)
+                        flush();
+                } else {
+                    __syncwarp();  // this warp's own records, read back by other lanes
+                    combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, pend.x, sp, lane);
+                }
+            }
+        }
+        pend.y = 0;
+        if (consumed == issued)
+            break;
+
         const int slot = con_slot;
         const unsigned parity = con_phase;
         if (!mbar_wait(&my_bars[slot], parity, a.status)) {
@@ -847,14 +1073,12 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         }
         __syncwarp();
         const int4 md = my_meta[slot];
-        const int s = md.y & 0xffff;
         const bool win = (md.y & kMetaRing) != 0;
-        const bool last = (md.y & kMetaLast) != 0;
         const unsigned pmask = ((unsigned)md.y >> 24) & 0xffu;
         const int ntok = md.z;
         const unsigned char *hdr = my_hdrs + slot * kHdrBytes;
-        if (s == 0) {
-            // ---- new item: its query rows arrived in this slot's header
+        if (md.y & kMetaSegStart) {
+            // ---- new segment: its query rows arrived in this slot's header
             if constexpr (kMma) {
                 const int g = lane >> 2, c = lane & 3;
                 if (win) {
@@ -1021,129 +1245,15 @@ __global__ void __launch_bounds__(kDecThreads, 1)
             con_slot = 0;
             con_phase ^= 1u;
         }
-        if (iss.it >= 0)
-            issue_one();  // refill the slot just read
-
-        if (!last)
-            continue;
-
-        // ---- item done: write the partial result (m, l, acc) of every head
-        const size_t rec0 = (size_t)md.x;
-        if (kLanePages && !win) {
-            if constexpr (kLanePages) {
-#pragma unroll
-                for (int off = 16; off; off >>= 1)
-                    lp += __shfl_xor_sync(0xffffffffu, lp, off);
-                const float tot = reduce_scatter<DD>(ol, lane);
-                constexpr int LPE = 32 / DD;  // lanes holding each entry
-                if (lane % LPE == 0)
-                    a.rec_acc[rec0 * kHeadDim + lane / LPE] = tot;
-                if (lane == 0) {
-                    a.rec_m[rec0] = mm;
-                    a.rec_l[rec0] = lp;
-                }
-            }
-        } else if constexpr (kMma) {
-            lp += __shfl_xor_sync(0xffffffffu, lp, 1);
-            lp += __shfl_xor_sync(0xffffffffu, lp, 2);
-            const int g = lane >> 2, c = lane & 3;
-            if (g < GH) {
-                const size_t rec = rec0 + (size_t)g * a.maxc;
-                float *ra = a.rec_acc + rec * kHeadDim;
-                if (win) {
-#pragma unroll
-                    for (int d = 0; d < 8; ++d)
-                        *reinterpret_cast<float2 *>(ra + 8 * d + 2 * c) = make_float2(ow[d][0], ow[d][1]);
-                } else {
-#pragma unroll
-                    for (int d = 0; d < NDD; ++d)
-                        *reinterpret_cast<float2 *>(ra + 8 * d + 2 * c) = make_float2(od[d][0], od[d][1]);
-                }
-                if (c == 0) {
-                    a.rec_m[rec] = mm;
-                    a.rec_l[rec] = lp;
-                }
-            }
-        } else {
-            const int LPTc = (win ? kHeadDim : DD) / E;
-            for (int off = LPTc; off < 32; off <<= 1) {
-#pragma unroll
-                for (int k = 0; k < GH; ++k) {
-                    const float mo = __shfl_xor_sync(0xffffffffu, m[k], off);
-                    const float lo = __shfl_xor_sync(0xffffffffu, l[k], off);
-                    const float mn = fmaxf(m[k], mo);
-                    const float fa = (m[k] == -INFINITY) ? 0.f : exp2f(m[k] - mn);
-                    const float fb = (mo == -INFINITY) ? 0.f : exp2f(mo - mn);
-                    l[k] = l[k] * fa + lo * fb;
-#pragma unroll
-                    for (int e = 0; e < E; ++e) {
-                        const float ao = __shfl_xor_sync(0xffffffffu, acc[k][e], off);
-                        acc[k][e] = acc[k][e] * fa + ao * fb;
-                    }
-                    m[k] = mn;
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < GH; ++k) {
-                const size_t rec = rec0 + (size_t)k * a.maxc;
-                if (lane < LPTc) {
-                    float4 *dstv = reinterpret_cast<float4 *>(a.rec_acc + rec * kHeadDim + lane * E);
-#pragma unroll
-                    for (int e4 = 0; e4 < E / 4; ++e4)
-                        dstv[e4] = make_float4(acc[k][4 * e4], acc[k][4 * e4 + 1], acc[k][4 * e4 + 2],
-                                               acc[k][4 * e4 + 3]);
-                }
-                if (lane == 0) {
-                    a.rec_m[rec] = m[k];
-                    a.rec_l[rec] = l[k];
-                }
-            }
-        }
-
+        pend = md;
     }
 
+    if (alive)
+        flush();
     if (!alive) {
         // a wait gave up: let this warp's copies still in flight land (bounded) before leaving
         for (int r = consumed + 1; r < issued; ++r)
             mbar_wait(&my_bars[r % kStages], (unsigned)((r / kStages) & 1), a.status);
-    }
-
-    // ---- merge.  Groups (index b * per_chunk + gh) whose chunks this CTA
-    // covered completely are merged as soon as every warp is done; a group
-    // shared with other CTAs is merged by the CTA whose atomic completes its
-    // chunk count.  Each warp releases its records GPU-wide as it finishes, so
-    // that fence overlaps the other warps' streaming.
-    __threadfence();
-    __syncthreads();
-    if (lo < hi) {
-        auto group_of = [&](int it) {
-            const int b = seq_of(it);
-            return b * per_chunk + (it - s_pre[b] * per_chunk) / (s_pre[b + 1] - s_pre[b]);
-        };
-        const int ga = group_of(lo), gb = group_of(hi - 1);
-        for (int gi = ga + warp; gi <= gb; gi += kDecWarps) {
-            const int b = gi / per_chunk, gh = gi % per_chunk;
-            const int nch = s_pre[b + 1] - s_pre[b];
-            if (nch == 0)
-                continue;
-            const int base = s_pre[b] * per_chunk + gh * nch;
-            const int done = min(hi, base + nch) - max(lo, base);
-            if (done <= 0)
-                continue;
-            if (done < nch) {
-                int old = 0;
-                if (lane == 0)
-                    old = atomicAdd(a.counters + gi, done);
-                old = __shfl_sync(0xffffffffu, old, 0);
-                if (old + done != nch)
-                    continue;
-                __threadfence();  // the other CTAs' records of this group
-            }
-            const int nwc = (min(s_len[b], w) + cw - 1) / cw;
-            const int g = gh / a.HS, h0 = g * a.G + (gh % a.HS) * a.GH;
-            for (int k = 0; k < GH; ++k)
-                combine_row<T, DD>(a, b, h0 + k, g, nwc, nch, lane);
-        }
     }
 }
 
@@ -1154,9 +1264,8 @@ DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int
 {
     DecodeGeometry gm;
     const int esz = dt == DAR_F32 ? 4 : 2;
-    gm.cw = kItemStages * (kHalf / (kHeadDim * esz));
-    gm.cd = kItemStages * (kHalf / (dd * esz));
-    gm.maxc = (w + gm.cw - 1) / gm.cw + (maxp * kPage + gm.cd - 1) / gm.cd;
+    const long long tw = kHalf / (kHeadDim * esz), td = kHalf / (dd * esz);
+    gm.sph = (w + tw - 1) / tw + ((long long)maxp * kPage + td - 1) / td;
     const int G = Hq / Hkv;
     gm.GH = (G % 4 == 0) ? 4 : (G % 2 == 0) ? 2 : 1;
     gm.HS = G / gm.GH;
@@ -1164,7 +1273,7 @@ DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int
 }
 
 template <typename T, int DD, int GH>
-static cudaError_t decode_t(const DecodeArgs &a0, cudaStream_t s)
+static cudaError_t decode_t(const DecodeArgs &a, cudaStream_t s)
 {
     auto kern = decode_kernel<T, DD, GH>;
     CUtensorMap m_wk{}, m_wv{}, m_pk{}, m_pv{};
@@ -1172,18 +1281,18 @@ static cudaError_t decode_t(const DecodeArgs &a0, cudaStream_t s)
         constexpr int tps_w = tps_ring<T>(), tps_d = tps_page<T, DD>();
         // one page box: min(64, tps_d) tokens = that many * DD / 64 lines of 128 bytes
         const int pr = (tps_d < kPage ? tps_d : kPage) * DD / kHeadDim;
-        const unsigned long long ring_rows = (unsigned long long)a0.B * a0.Hkv * a0.w;
-        const unsigned long long pool_lines = (unsigned long long)(a0.num_pages > 0 ? a0.num_pages : 1) * a0.Hkv * DD;
-        if (!make_tma_2d_bf16(&m_wk, a0.win_k, ring_rows, kHeadDim, tps_w) ||
-            !make_tma_2d_bf16(&m_wv, a0.win_v, ring_rows, kHeadDim, tps_w) ||
-            !make_tma_2d_bf16(&m_pk, a0.pool_kd, pool_lines, kHeadDim, pr) ||
-            !make_tma_2d_bf16(&m_pv, a0.pool_vd, pool_lines, kHeadDim, pr))
+        const unsigned long long ring_rows = (unsigned long long)a.B * a.Hkv * a.w;
+        const unsigned long long pool_lines = (unsigned long long)(a.num_pages > 0 ? a.num_pages : 1) * a.Hkv * DD;
+        if (!make_tma_2d_bf16(&m_wk, a.win_k, ring_rows, kHeadDim, tps_w) ||
+            !make_tma_2d_bf16(&m_wv, a.win_v, ring_rows, kHeadDim, tps_w) ||
+            !make_tma_2d_bf16(&m_pk, a.pool_kd, pool_lines, kHeadDim, pr) ||
+            !make_tma_2d_bf16(&m_pv, a.pool_vd, pool_lines, kHeadDim, pr))
             return cudaErrorInvalidValue;
     }
     // one-time set-up per instantiation (kept out of the launch path so launches
     // stay cheap and can be captured in a CUDA graph)
-    static int sms = 0;
-    if (sms == 0) {
+    static int ctas = 0;
+    if (ctas == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)decode_smem_bytes(DAR_DECODE_MAX_BATCH));
         if (e != cudaSuccess)
@@ -1191,11 +1300,10 @@ static cudaError_t decode_t(const DecodeArgs &a0, cudaStream_t s)
         int dev = 0, n = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        sms = n;
+        ctas = n < kMaxDecodeCtas ? n : kMaxDecodeCtas;  // the workspace holds records for this many
     }
-    const DecodeArgs &a = a0;
     const int rows = a.B * a.Hq;
-    const int prep_blocks = min(2 * sms, max(1, (rows + kPrepThreads / 32 - 1) / (kPrepThreads / 32)));
+    const int prep_blocks = min(2 * ctas, max(1, (rows + kPrepThreads / 32 - 1) / (kPrepThreads / 32)));
     // both kernels use programmatic launch: prep computes q~ while the kernel
     // before it finishes (and waits for it before exiting); the stream kernel
     // sets up while prep drains
@@ -1211,7 +1319,8 @@ static cudaError_t decode_t(const DecodeArgs &a0, cudaStream_t s)
     cudaError_t e = cudaLaunchKernelEx(&cfg, decode_prep_kernel<T, DD>, a);
     if (e != cudaSuccess)
         return e;
-    cfg.gridDim = dim3(sms);
+    // one CTA per SM (the records of the workspace are sized for kMaxDecodeCtas)
+    cfg.gridDim = dim3(ctas);
     cfg.blockDim = dim3(kDecThreads);
     cfg.dynamicSmemBytes = decode_smem_bytes(a.B);
     return cudaLaunchKernelEx(&cfg, kern, m_wk, m_wv, m_pk, m_pv, a);

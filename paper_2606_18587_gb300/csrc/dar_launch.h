@@ -31,10 +31,10 @@ struct DecodeArgs {
     const int32_t *seq_lens;
     int32_t *status;
     const float *Uk, *Uv;  // [Hkv][dd][64]
-    float *rec_m, *rec_l, *rec_acc;  // split-K partial results [B][Hq][maxc] (acc: x 64)
-    float *qt;                       // [B][Hq][dd] q~ = q Uk^T
-    int32_t *counters;               // [B][Hkv][HS] chunks finished per shared group
-    int B, Hq, Hkv, G, GH, HS, w, maxp, num_pages, maxc, cw, cd;
+    float *rec;         // split-K partial results, kRecFloats per (warp, slot, type, head)
+    float *qt;          // [B][Hq][dd] q~ = q Uk^T
+    int32_t *counters;  // [B][Hkv][HS] finished stages per group, then the pool's claim counter
+    int B, Hq, Hkv, G, GH, HS, w, maxp, num_pages;
     float qscale;  // scale * log2(e)
 };
 
@@ -63,8 +63,18 @@ cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s);
 
 // Split-K geometry of the decode kernel (shared by workspace sizing and launch).
 struct DecodeGeometry {
-    int cw, cd, maxc, GH, HS;  // minimum chunk sizes (tokens), chunks per head at that size, head grouping
+    long long sph;  // stages per (sequence, query head) at full capacity
+    int GH, HS;     // query heads per group, groups per KV head
 };
+// The decode stream kernel runs one CTA of kDecodeWarpsPerCta warps per SM, at
+// most kMaxDecodeCtas CTAs.  Its stages fall into ranges -- one per warp, then
+// up to kDecodePoolChunks pool chunks -- and each range owns 2 slots x 2 types
+// x GH records of kRecFloats floats (acc[64], m, l, padding to 16 bytes) in
+// the workspace.
+constexpr int kDecodeWarpsPerCta = 8;
+constexpr int kMaxDecodeCtas = 160;
+constexpr int kDecodePoolChunks = 2 * kMaxDecodeCtas * kDecodeWarpsPerCta;  // ranges beyond the warps' own
+constexpr int kRecFloats = 68;
 DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int maxp);
 
 // 2-D tensor map of a bf16 row-major [rows][cols] array (cols * 2 = 16, 32, 64

@@ -37,12 +37,12 @@ def test_noalloc_matches_workspace_decode_twice():
 
 
 def test_noalloc_refuses_shapes_beyond_its_scratch():
-    # 64 sequences x 32 heads with room for 32768 tokens each needs far more
-    # than the built-in scratch; nothing may be launched
-    cache = dar.DarCache(64, 8, 16, 256, 512, 64, dtype=torch.bfloat16)
-    assert dar.dar_decode_workspace_bytes(cache, 32) > (8 << 20)
-    q = torch.zeros((64, 32, 64), dtype=torch.bfloat16, device="cuda")
-    U = torch.zeros((8, 16, 64), dtype=torch.float32, device="cuda")
+    # 512 sequences x 64 query heads with d_down = 64: the absorbed queries
+    # alone (512 * 64 * 64 fp32) exceed the built-in scratch; nothing may be launched
+    cache = dar.DarCache(512, 8, 64, 16, 1, dtype=torch.bfloat16)
+    assert dar.dar_decode_workspace_bytes(cache, 64) > (8 << 20)
+    q = torch.zeros((512, 64, 64), dtype=torch.bfloat16, device="cuda")
+    U = torch.zeros((8, 64, 64), dtype=torch.float32, device="cuda")
     out = torch.full_like(q, 7.0)
     with pytest.raises(dar.DarError) as e:
         dar.dar_attn_decode_noalloc(cache, q, U, U, out=out)
