@@ -145,11 +145,12 @@ __device__ __forceinline__ float *rec_ptr(float *rec, int range, int slot, int t
 }
 
 // Dynamic shared memory of the stream kernel for a batch of B sequences:
-// alignment slack, slots, headers, barriers, stage metadata, the tables.
+// alignment slack, slots, headers, barriers, stage metadata, merge barriers,
+// the tables.
 constexpr size_t decode_smem_bytes(int B)
 {
     return 1024 + (size_t)kDecWarps * kStages * (kSlotBytes + kHdrBytes + sizeof(uint64_t) + sizeof(int4)) +
-           (size_t)(2 * B + 1) * sizeof(int);
+           (size_t)kDecWarps * sizeof(uint64_t) + (size_t)(2 * B + 1) * sizeof(int);
 }
 
 // --------------------------------------------------------------------- prep
@@ -517,14 +518,17 @@ __device__ __forceinline__ Split make_split(int S, int NW)
     return sp;
 }
 
-// Merge of group `gid` from the records of every warp part, by one warp:
-// one softmax over all parts (Eq. 4), o = (sum_p f_p acc_p[ring] +
-// (sum_p f_p acc_p[pages]) Uv) / sum_p f_p l_p, f_p = 2^(m_p - max m).  Lane i
-// reads candidate i of a batch of 32 (range wa + i / 2, type i % 2); lane j
-// holds entries 2j, 2j + 1 of the output row.
+// Merge of group `gid` from the records of all its parts, by one warp: one
+// softmax over all parts (Eq. 4), o = (sum_p f_p acc_p[ring] + (sum_p f_p
+// acc_p[pages]) Uv) / sum_p f_p l_p, f_p = 2^(m_p - max m).  With `rows` (the
+// warp's idle slots, at the end of its streaming) the records are pulled into
+// shared memory by bulk copies, all in flight at once (completion counted on
+// `mbar`, whose phase `mphase` tracks); without it (a group that lies inside
+// one range: two records at most) they are read in place.  Lane j holds
+// entries 2j, 2j + 1 of the output row.
 template <typename T, int DD, int GH, int TPS_W, int TPS_D>
 __device__ __noinline__ void combine_group(const DecodeArgs &a, const int *s_pre, const int *s_len, int gid,
-                                           Split sp, int lane)
+                                           Split sp, int lane, float *rows, uint64_t *mbar, unsigned *mphase)
 {
     const int per_chunk = a.Hkv * a.HS;
     const int b = gid / per_chunk, gh = gid - b * per_chunk;
@@ -540,94 +544,91 @@ __device__ __noinline__ void combine_group(const DecodeArgs &a, const int *s_pre
 #pragma unroll
     for (int cc = 0; cc < UVP; ++cc)
         uv[cc] = __ldg(reinterpret_cast<const float2 *>(Uv + (size_t)cc * kHeadDim) + lane);
+    // records in shared memory are final once the barrier completes; in place,
+    // they are read from L2 (another SM's L1 copy could be stale)
+    auto ld2 = [&](const float *p) {
+        return rows ? *reinterpret_cast<const float2 *>(p) : __ldcg(reinterpret_cast<const float2 *>(p));
+    };
     for (int k = 0; k < GH; ++k) {
-        // candidate c0 + lane: its record index, or -1 if the part has no such segment
-        auto cand = [&](int c0) {
-            const int i = c0 + lane;
-            if (i >= ncand)
-                return -1;
-            const int wk = wa + (i >> 1), type = i & 1;
-            const int rlo = sp.lo(wk);
-            const int lo = max(rlo, G0), hi = min(sp.lo(wk + 1), G1);
-            const bool has = type == 0 ? lo < min(hi, GR) : max(lo, GR) < hi;
-            if (!has)
-                return -1;
-            const int slot = G0 < rlo ? 0 : 1;
-            return ((wk * 2 + slot) * 2 + type) * GH + k;
-        };
-        auto acc_of = [&](int rj, int j) {  // lane's entry pair of record rj (candidate j: even ring, odd pages)
-            return rj >= 0 && ((j & 1) == 0 || 2 * lane < DD)
-                       ? __ldcg(reinterpret_cast<const float2 *>(a.rec + (size_t)rj * kRecFloats) + lane)
-                       : make_float2(0.f, 0.f);
-        };
-        // (m, l) by lane; the entries of the first kPre candidates are loaded
-        // with them, before the max is known (later candidates, groups over
-        // more than kPre / 2 ranges, follow one at a time)
-        constexpr int kPre = 16;
-        float2 v[kPre];
-        int r0 = -1;
-        float m0 = -INFINITY, l0 = 0.f, M = -INFINITY;
+        float M = -INFINITY, lsum = 0.f, o0 = 0.f, o1 = 0.f, gd0 = 0.f, gd1 = 0.f;
+        // rounds of 32 candidates: candidate c0 + lane is (range wa + (c0 + lane) / 2,
+        // type lane % 2); one online softmax runs over the rounds
         for (int c0 = 0; c0 < ncand; c0 += 32) {
-            const int r = cand(c0);
+            int r = -1;
+            if (c0 + lane < ncand) {
+                const int wk = wa + ((c0 + lane) >> 1);
+                const int rlo = sp.lo(wk);
+                const int lo = max(rlo, G0), hi = min(sp.lo(wk + 1), G1);
+                if ((lane & 1) == 0 ? lo < min(hi, GR) : max(lo, GR) < hi)
+                    r = ((wk * 2 + (G0 < rlo ? 0 : 1)) * 2 + (lane & 1)) * GH + k;
+            }
+            const unsigned live = __ballot_sync(0xffffffffu, r >= 0);
+            // this lane's record: pulled into shared memory by bulk copies (all
+            // in flight at once), or read where it is
+            const float *mine = a.rec + (size_t)(r >= 0 ? r : 0) * kRecFloats;
+            if (rows) {
+                if (lane == 0)
+                    mbar_expect_tx(mbar, (unsigned)__popc(live) * kRecFloats * 4);
+                __syncwarp();
+                if (r >= 0)
+                    bulk_g2s(rows + lane * kRecFloats, mine, kRecFloats * 4, mbar);
+                mbar_wait(mbar, *mphase, a.status);
+                *mphase ^= 1u;
+                mine = rows + lane * kRecFloats;
+            }
             float mr = -INFINITY, lr = 0.f;
             if (r >= 0) {
-                const float2 ml = __ldcg(reinterpret_cast<const float2 *>(a.rec + (size_t)r * kRecFloats + kHeadDim));
+                const float2 ml = ld2(mine + kHeadDim);
                 mr = ml.x;
                 lr = ml.y;
             }
-            if (c0 == 0) {
-                r0 = r;
-                m0 = mr;
-                l0 = lr;
+            float mx = mr;
 #pragma unroll
-                for (int j = 0; j < kPre; ++j)
-                    v[j] = acc_of(__shfl_sync(0xffffffffu, r, j), j);
-            }
-            M = fmaxf(M, mr);
-        }
-#pragma unroll
-        for (int off = 16; off; off >>= 1)
-            M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-        float o0 = 0.f, o1 = 0.f, gd0 = 0.f, gd1 = 0.f, lsum = 0.f;
-        auto add = [&](float fj, float2 x, int j) {
-            if ((j & 1) == 0) {
-                o0 = fmaf(fj, x.x, o0);
-                o1 = fmaf(fj, x.y, o1);
-            } else {
-                gd0 = fmaf(fj, x.x, gd0);
-                gd1 = fmaf(fj, x.y, gd1);
-            }
-        };
-        for (int c0 = 0; c0 < ncand; c0 += 32) {
-            int r = r0;
-            float mr = m0, lr = l0;
-            if (c0 > 0) {
-                r = cand(c0);
-                mr = -INFINITY;
-                lr = 0.f;
-                if (r >= 0) {
-                    const float2 ml =
-                        __ldcg(reinterpret_cast<const float2 *>(a.rec + (size_t)r * kRecFloats + kHeadDim));
-                    mr = ml.x;
-                    lr = ml.y;
-                }
-            }
+            for (int off = 16; off; off >>= 1)
+                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+            const float Mn = fmaxf(M, mx);
+            const float sc = M == -INFINITY ? 0.f : exp2f(M - Mn);
+            lsum *= sc;
+            o0 *= sc;
+            o1 *= sc;
+            gd0 *= sc;
+            gd1 *= sc;
+            M = Mn;
             const float f = r >= 0 ? exp2f(mr - M) : 0.f;
             lsum = fmaf(f, lr, lsum);
-            int j0 = 0;
-            if (c0 == 0) {
-#pragma unroll
-                for (int j = 0; j < kPre; ++j)
-                    add(__shfl_sync(0xffffffffu, f, j), v[j], j);
-                j0 = kPre;
+            if (rows) {  // every candidate row up to the last live one; absent rows hold garbage
+                const int jn = 32 - __clz(live);
+#pragma unroll 8
+                for (int j = 0; j < jn; ++j) {
+                    const float fj = __shfl_sync(0xffffffffu, f, j);
+                    const float2 x = *reinterpret_cast<const float2 *>(rows + j * kRecFloats + 2 * lane);
+                    if ((live >> j) & 1u) {
+                        if ((j & 1) == 0) {  // ring: acc[64]
+                            o0 = fmaf(fj, x.x, o0);
+                            o1 = fmaf(fj, x.y, o1);
+                        } else if (2 * lane < DD) {  // pages: acc[DD]
+                            gd0 = fmaf(fj, x.x, gd0);
+                            gd1 = fmaf(fj, x.y, gd1);
+                        }
+                    }
+                }
+            } else {
+                for (unsigned lv = live; lv; lv &= lv - 1) {
+                    const int j = __ffs(lv) - 1;
+                    const float fj = __shfl_sync(0xffffffffu, f, j);
+                    const float *row = a.rec + (size_t)__shfl_sync(0xffffffffu, r, j) * kRecFloats;
+                    if ((j & 1) == 0) {  // ring: acc[64]
+                        const float2 x = ld2(row + 2 * lane);
+                        o0 = fmaf(fj, x.x, o0);
+                        o1 = fmaf(fj, x.y, o1);
+                    } else if (2 * lane < DD) {  // pages: acc[DD]
+                        const float2 x = ld2(row + 2 * lane);
+                        gd0 = fmaf(fj, x.x, gd0);
+                        gd1 = fmaf(fj, x.y, gd1);
+                    }
+                }
             }
-            const unsigned live = __ballot_sync(0xffffffffu, r >= 0);
-            for (int j = j0; j < 32; ++j) {
-                if (!((live >> j) & 1u))
-                    continue;
-                const float fj = __shfl_sync(0xffffffffu, f, j);
-                add(fj, acc_of(__shfl_sync(0xffffffffu, r, j), j), j);
-            }
+            __syncwarp();  // the rows are read before the next round refills them
         }
 #pragma unroll
         for (int off = 16; off; off >>= 1)
@@ -674,7 +675,8 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     unsigned char *hdrs = slots + (size_t)kDecWarps * kStages * kSlotBytes;  // [warps][stages][header]
     uint64_t *bars = reinterpret_cast<uint64_t *>(hdrs + (size_t)kDecWarps * kStages * kHdrBytes);
     int4 *meta = reinterpret_cast<int4 *>(bars + kDecWarps * kStages);
-    int *s_pre = reinterpret_cast<int *>(meta + kDecWarps * kStages);  // [B + 1]
+    uint64_t *mbars = reinterpret_cast<uint64_t *>(meta + kDecWarps * kStages);  // [warps]
+    int *s_pre = reinterpret_cast<int *>(mbars + kDecWarps);                    // [B + 1]
     int *s_len = s_pre + a.B + 1;                                      // [B]
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -684,6 +686,8 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     int4 *my_meta = meta + warp * kStages;
     if (lane < kStages)
         mbar_init(&my_bars[lane], 1);
+    if (lane == kStages)
+        mbar_init(&mbars[warp], 1);
     sm100::mbar_init_fence();
     __syncthreads();
     if constexpr (kMma) {
@@ -952,22 +956,35 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     // when the warp runs out of work, so the streaming never waits on them; a
     // count that completes its group's stages makes this warp merge the group.
     int pg = 0, pp = 0, npend = 0;
+    unsigned mphase = 0;  // phase of this warp's merge barrier
     auto flush = [&]() {
         if (npend == 0)
             return;
-        __threadfence();  // this warp's records, GPU-wide, before its counts
+        // each count is an acquire-release atomic: it publishes the warp's
+        // records (ordered before it by the warp barrier) and, for the count
+        // that completes a group, makes the other parts' records visible
+        __syncwarp();
         bool fin = false;
         if (lane < npend) {
-            const int old = atomicAdd(a.counters + pg, pp);
+            int old;
+            asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;"
+                         : "=r"(old)
+                         : "l"(a.counters + pg), "r"(pp)
+                         : "memory");
             fin = old + pp == seq_stages<TPS_W, TPS_D>(s_len[pg / per_chunk], w).n;
         }
         unsigned fm = __ballot_sync(0xffffffffu, fin);
-        if (fm)
-            __threadfence();  // the other parts' records
+        if (fm) {
+            __syncwarp();  // the acquiring lane's view, to the lanes that copy
+            asm volatile("fence.proxy.async.global;" ::: "memory");  // ... and to the bulk copies
+        }
+        // the slots are idle here only if every issued stage has been consumed
+        float *rows = issued == consumed ? reinterpret_cast<float *>(my_slots) : nullptr;
         while (fm) {
             const int j = __ffs(fm) - 1;
             fm &= fm - 1;
-            combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, __shfl_sync(0xffffffffu, pg, j), sp, lane);
+            combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, __shfl_sync(0xffffffffu, pg, j), sp, lane,
+                                                   rows, &mbars[warp], &mphase);
         }
         npend = 0;
     };
@@ -1057,7 +1074,8 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                         flush();
                 } else {
                     __syncwarp();  // this warp's own records, read back by other lanes
-                    combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, pend.x, sp, lane);
+                    combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, pend.x, sp, lane, nullptr, nullptr,
+                                                           &mphase);
                 }
             }
         }
