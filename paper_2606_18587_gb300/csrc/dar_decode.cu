@@ -433,45 +433,38 @@ __device__ __forceinline__ float reduce_scatter(const float (&o)[DD], int lane)
 // Per-sequence tables of one decode call, built by every CTA of the stream
 // kernel into its shared memory: s_len[b] = validated length (-1 if beyond
 // the cache's capacity) and s_pre[b] = stages per group of the sequences
-// before b (s_pre[B] = all).  The CTA loads the lengths; warp 0 (a contiguous
-// run of sequences per lane) scans the stage counts.
-template <int TPS_W, int TPS_D>
-__device__ __forceinline__ void build_tables(const DecodeArgs &a, int *s_pre, int *s_len)
+// before b (s_pre[B] = all).  validated_length reads a length from L2 (an L1
+// copy could predate the append); scan_tables is warp 0's prefix sum over
+// contiguous runs of sequences per lane.
+__device__ __forceinline__ int validated_length(const DecodeArgs &a, int b)
 {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int L = __ldcg(a.seq_lens + b);
+    return (L < 0 || (long long)L - a.w > (long long)a.maxp * kPage) ? -1 : L;
+}
+template <int TPS_W, int TPS_D>
+__device__ __forceinline__ void scan_tables(const DecodeArgs &a, int *s_pre, const int *s_len)
+{
+    const int lane = threadIdx.x & 31;
     const int B = a.B, w = a.w;
-    for (int b = threadIdx.x; b < B; b += blockDim.x) {
-        int L = a.seq_lens[b];
-        if (L < 0 || (long long)L - w > (long long)a.maxp * kPage) {
-            if (blockIdx.x == 0)
-                report(a.status, DAR_ERR_CAPACITY);
-            L = -1;
-        }
-        s_len[b] = L;
-    }
-    __syncthreads();
-    if (warp == 0) {
-        const int per = (B + 31) / 32;
-        const int b0 = min(B, lane * per), b1 = min(B, b0 + per);
-        int mine = 0;
-        for (int b = b0; b < b1; ++b)
-            mine += seq_stages<TPS_W, TPS_D>(s_len[b], w).n;
-        int incl = mine;
+    const int per = (B + 31) / 32;
+    const int b0 = min(B, lane * per), b1 = min(B, b0 + per);
+    int mine = 0;
+    for (int b = b0; b < b1; ++b)
+        mine += seq_stages<TPS_W, TPS_D>(s_len[b], w).n;
+    int incl = mine;
 #pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, off);
-            if (lane >= off)
-                incl += y;
-        }
-        int run = incl - mine;
-        for (int b = b0; b < b1; ++b) {
-            s_pre[b] = run;
-            run += seq_stages<TPS_W, TPS_D>(s_len[b], w).n;
-        }
-        if (lane == 31)
-            s_pre[B] = incl;
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off)
+            incl += y;
     }
-    __syncthreads();
+    int run = incl - mine;
+    for (int b = b0; b < b1; ++b) {
+        s_pre[b] = run;
+        run += seq_stages<TPS_W, TPS_D>(s_len[b], w).n;
+    }
+    if (lane == 31)
+        s_pre[B] = incl;
 }
 
 // The split of the S stages into ranges.  The first Ss stages are divided
@@ -706,19 +699,15 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         for (size_t i = l0 + threadIdx.x; i < l1; i += blockDim.x)
             asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<const char *>(a.block_table) + i * 128));
     }
-    // everything below reads the cache and q~ (the prep kernel waited for the
-    // kernel before it, so both are final)
-    sm100::grid_dep_wait();
-    build_tables<TPS_W, TPS_D>(a, s_pre, s_len);
-    if (blockIdx.x == 0) {  // sequences with nothing to attend to get a zero output
-        T *out = static_cast<T *>(a.out);
-        for (int b = warp; b < a.B; b += kDecWarps) {
-            if (s_len[b] > 0)
-                continue;
-            for (int i = lane; i < a.Hq * kHeadDim; i += 32)
-                out[(size_t)b * a.Hq * kHeadDim + i] = from_f32<T>(0.f);
-        }
-    }
+    // Tables from the lengths as they are now: the kernel before this one
+    // (normally the cache append) may still be changing them, so they are a
+    // guess, checked after the wait below.
+    for (int b = threadIdx.x; b < a.B; b += blockDim.x)
+        s_len[b] = validated_length(a, b);
+    __syncthreads();
+    if (warp == 0)
+        scan_tables<TPS_W, TPS_D>(a, s_pre, s_len);
+    __syncthreads();
 
     const int w = a.w;
     const T *qg = static_cast<const T *>(a.q);
@@ -734,11 +723,10 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     // and the walk over it: sequence wb, group wgh of the sequence, stage wj
     // of the group (the ring's sq.r stages, then the pages')
     const int per_chunk = a.Hkv * a.HS;
-    const Split sp = make_split(s_pre[a.B] * per_chunk, gridDim.x * kDecWarps);
+    Split sp;
     int32_t *pool_next = a.counters + a.B * per_chunk;  // the pool's claim counter
-    int rid = blockIdx.x * kDecWarps + warp;
-    int lo = sp.lo(rid), hi = sp.lo(rid + 1);
-    int iss_s = lo;  // next stage to issue
+    int rid = 0, lo = 0, hi = 0;
+    int iss_s = 0;  // next stage to issue
     int wb = 0, wgh = 0, wj = 0;
     SeqStages sq = {0, 0, 0, 1};
     auto begin_range = [&]() {  // the walk's position at stage lo
@@ -780,13 +768,13 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     // of a range (two stages ahead), and the warp moves on to the claimed
     // chunk as soon as that range's last stage is issued
     int claim = 0;
-    bool asked = false, pool_done = sp.NC == 0;
+    bool asked = false, pool_done = true;
     auto ask = [&]() {
         if (lane == 0)
             claim = atomicAdd(pool_next, 1);
         asked = true;
     };
-    int ask_at = max(lo, hi - 2);
+    int ask_at = 0;
     auto next_range = [&]() {
         if (pool_done)
             return;
@@ -806,11 +794,57 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         begin_range();
         window_for_range();
     };
-    if (lo < hi) {
-        begin_range();
-        window_for_range();
-    } else {
+    // This warp's own range, the walk's start and its first block-table
+    // window: they depend on the lengths only through the per-sequence stage
+    // counts, so they are set up from the guessed tables before the wait and
+    // kept if the counts hold.
+#pragma unroll 1
+    for (int pass = 0;; ++pass) {
+        sp = make_split(s_pre[a.B] * per_chunk, gridDim.x * kDecWarps);
+        rid = blockIdx.x * kDecWarps + warp;
+        lo = sp.lo(rid);
+        hi = sp.lo(rid + 1);
+        iss_s = lo;
+        ask_at = max(lo, hi - 2);
+        pool_done = sp.NC == 0;
+        if (lo < hi) {
+            begin_range();
+            window_for_range();
+        }
+        if (pass > 0)
+            break;
+        // everything below reads the cache and q~ (the prep kernel waited for
+        // the kernel before it, so both are final)
+        sm100::grid_dep_wait();
+        // the final lengths: do their stage counts match the guess?
+        int changed = 0;
+        for (int b = threadIdx.x; b < a.B; b += blockDim.x) {
+            const int L = validated_length(a, b);
+            if (L < 0 && blockIdx.x == 0)
+                report(a.status, DAR_ERR_CAPACITY);
+            const SeqStages was = seq_stages<TPS_W, TPS_D>(s_len[b], w), now = seq_stages<TPS_W, TPS_D>(L, w);
+            changed |= was.r != now.r || was.n != now.n;
+            s_len[b] = L;
+        }
+        if (!__syncthreads_or(changed)) {
+            if (lo < hi)
+                sq = seq_stages<TPS_W, TPS_D>(s_len[wb], w);  // the walk's token bounds
+            break;
+        }
+        if (warp == 0)  // counts changed: rebuild the prefix sums and set up again
+            scan_tables<TPS_W, TPS_D>(a, s_pre, s_len);
+        __syncthreads();
+    }
+    if (lo >= hi)
         next_range();  // no own stages (tiny workloads): straight to the pool
+    if (blockIdx.x == 0) {  // sequences with nothing to attend to get a zero output
+        T *out = static_cast<T *>(a.out);
+        for (int b = warp; b < a.B; b += kDecWarps) {
+            if (s_len[b] > 0)
+                continue;
+            for (int i = lane; i < a.Hq * kHeadDim; i += 32)
+                out[(size_t)b * a.Hq * kHeadDim + i] = from_f32<T>(0.f);
+        }
     }
 
     int issued = 0, consumed = 0;    // stages issued / consumed by this warp
