@@ -145,12 +145,11 @@ __device__ __forceinline__ float *rec_ptr(float *rec, int range, int slot, int t
 }
 
 // Dynamic shared memory of the stream kernel for a batch of B sequences:
-// alignment slack, slots, headers, barriers, stage metadata, merge barriers,
-// the tables.
+// alignment slack, slots, headers, barriers, stage metadata, the tables.
 constexpr size_t decode_smem_bytes(int B)
 {
     return 1024 + (size_t)kDecWarps * kStages * (kSlotBytes + kHdrBytes + sizeof(uint64_t) + sizeof(int4)) +
-           (size_t)kDecWarps * sizeof(uint64_t) + (size_t)(2 * B + 1) * sizeof(int);
+           (size_t)(2 * B + 1) * sizeof(int);
 }
 
 // --------------------------------------------------------------------- prep
@@ -475,17 +474,26 @@ __device__ __forceinline__ void scan_tables(const DecodeArgs &a, int *s_pre, con
 // more of them.  Range ids index the record slots.
 struct Split {
     int S, Ss, NW, C, NC;
-    int q0, r0;  // Ss = q0 NW + r0, so that floor(Ss k / NW) = q0 k + floor(r0 k / NW) in 32 bits
+    int q0, r0;         // Ss = q0 NW + r0, so that floor(Ss k / NW) = q0 k + floor(r0 k / NW) in 32 bits
+    float inv_nw, rate;  // 1 / NW and NW / Ss, for quotient estimates
+    // floor(x / NW) for 0 <= x < 2^24: a float estimate off by at most one, corrected
+    __device__ __forceinline__ int div_nw(int x) const
+    {
+        int q = (int)((float)x * inv_nw);
+        q += (q + 1) * NW <= x;
+        q -= q * NW > x;
+        return q;
+    }
     __device__ __forceinline__ int lo(int k) const
     {
-        return k <= NW ? q0 * k + (r0 * k) / NW : min(S, Ss + (k - NW) * C);
+        return k <= NW ? q0 * k + div_nw(r0 * k) : min(S, Ss + (k - NW) * C);
     }
     __device__ __forceinline__ int owner(int t) const  // the range holding stage t
     {
         if (t >= Ss)
             return NW + (t - Ss) / C;
         // the last k with lo(k) <= t: a float estimate, then exact steps
-        int k = min(NW - 1, (int)((float)t * (float)NW / (float)Ss));
+        int k = min(NW - 1, (int)((float)t * rate));
         while (k > 0 && lo(k) > t)
             --k;
         while (k + 1 < NW && lo(k + 1) <= t)
@@ -508,20 +516,21 @@ __device__ __forceinline__ Split make_split(int S, int NW)
     sp.Ss = S - P;
     sp.q0 = sp.Ss / NW;
     sp.r0 = sp.Ss - sp.q0 * NW;
+    sp.inv_nw = 1.f / (float)NW;
+    sp.rate = sp.Ss > 0 ? (float)NW / (float)sp.Ss : 0.f;
     return sp;
 }
 
 // Merge of group `gid` from the records of all its parts, by one warp: one
 // softmax over all parts (Eq. 4), o = (sum_p f_p acc_p[ring] + (sum_p f_p
 // acc_p[pages]) Uv) / sum_p f_p l_p, f_p = 2^(m_p - max m).  With `rows` (the
-// warp's idle slots, at the end of its streaming) the records are pulled into
-// shared memory by bulk copies, all in flight at once (completion counted on
-// `mbar`, whose phase `mphase` tracks); without it (a group that lies inside
-// one range: two records at most) they are read in place.  Lane j holds
-// entries 2j, 2j + 1 of the output row.
+// warp's idle slots, at the end of its streaming) lane i stages record i of a
+// round of 32 in shared memory, all loads in flight at once; without it (a
+// group that lies inside one range: two records at most) they are read in
+// place.  Lane j holds entries 2j, 2j + 1 of the output row.
 template <typename T, int DD, int GH, int TPS_W, int TPS_D>
 __device__ __noinline__ void combine_group(const DecodeArgs &a, const int *s_pre, const int *s_len, int gid,
-                                           Split sp, int lane, float *rows, uint64_t *mbar, unsigned *mphase)
+                                           Split sp, int lane, float *rows)
 {
     const int per_chunk = a.Hkv * a.HS;
     const int b = gid / per_chunk, gh = gid - b * per_chunk;
@@ -556,17 +565,19 @@ __device__ __noinline__ void combine_group(const DecodeArgs &a, const int *s_pre
                     r = ((wk * 2 + (G0 < rlo ? 0 : 1)) * 2 + (lane & 1)) * GH + k;
             }
             const unsigned live = __ballot_sync(0xffffffffu, r >= 0);
-            // this lane's record: pulled into shared memory by bulk copies (all
-            // in flight at once), or read where it is
+            // this lane's record: staged in shared memory (every lane's loads in
+            // flight at once), or read where it is
             const float *mine = a.rec + (size_t)(r >= 0 ? r : 0) * kRecFloats;
             if (rows) {
-                if (lane == 0)
-                    mbar_expect_tx(mbar, (unsigned)__popc(live) * kRecFloats * 4);
+                if (r >= 0) {  // 16-byte asynchronous copies through L2, no registers
+                    const uint32_t dst = smem_u32(rows + lane * kRecFloats);
+#pragma unroll
+                    for (int i = 0; i < kRecFloats / 4; ++i)
+                        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst + 16 * i), "l"(mine + 4 * i)
+                                     : "memory");
+                }
+                asm volatile("cp.async.wait_all;" ::: "memory");
                 __syncwarp();
-                if (r >= 0)
-                    bulk_g2s(rows + lane * kRecFloats, mine, kRecFloats * 4, mbar);
-                mbar_wait(mbar, *mphase, a.status);
-                *mphase ^= 1u;
                 mine = rows + lane * kRecFloats;
             }
             float mr = -INFINITY, lr = 0.f;
@@ -668,8 +679,7 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     unsigned char *hdrs = slots + (size_t)kDecWarps * kStages * kSlotBytes;  // [warps][stages][header]
     uint64_t *bars = reinterpret_cast<uint64_t *>(hdrs + (size_t)kDecWarps * kStages * kHdrBytes);
     int4 *meta = reinterpret_cast<int4 *>(bars + kDecWarps * kStages);
-    uint64_t *mbars = reinterpret_cast<uint64_t *>(meta + kDecWarps * kStages);  // [warps]
-    int *s_pre = reinterpret_cast<int *>(mbars + kDecWarps);                    // [B + 1]
+    int *s_pre = reinterpret_cast<int *>(meta + kDecWarps * kStages);  // [B + 1]
     int *s_len = s_pre + a.B + 1;                                      // [B]
 
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -679,8 +689,6 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     int4 *my_meta = meta + warp * kStages;
     if (lane < kStages)
         mbar_init(&my_bars[lane], 1);
-    if (lane == kStages)
-        mbar_init(&mbars[warp], 1);
     sm100::mbar_init_fence();
     __syncthreads();
     if constexpr (kMma) {
@@ -990,7 +998,6 @@ __global__ void __launch_bounds__(kDecThreads, 1)
     // when the warp runs out of work, so the streaming never waits on them; a
     // count that completes its group's stages makes this warp merge the group.
     int pg = 0, pp = 0, npend = 0;
-    unsigned mphase = 0;  // phase of this warp's merge barrier
     auto flush = [&]() {
         if (npend == 0)
             return;
@@ -1008,17 +1015,15 @@ __global__ void __launch_bounds__(kDecThreads, 1)
             fin = old + pp == seq_stages<TPS_W, TPS_D>(s_len[pg / per_chunk], w).n;
         }
         unsigned fm = __ballot_sync(0xffffffffu, fin);
-        if (fm) {
-            __syncwarp();  // the acquiring lane's view, to the lanes that copy
-            asm volatile("fence.proxy.async.global;" ::: "memory");  // ... and to the bulk copies
-        }
+        if (fm)
+            __syncwarp();  // the acquiring lane's view, to the lanes that load
         // the slots are idle here only if every issued stage has been consumed
         float *rows = issued == consumed ? reinterpret_cast<float *>(my_slots) : nullptr;
         while (fm) {
             const int j = __ffs(fm) - 1;
             fm &= fm - 1;
             combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, __shfl_sync(0xffffffffu, pg, j), sp, lane,
-                                                   rows, &mbars[warp], &mphase);
+                                                   rows);
         }
         npend = 0;
     };
@@ -1108,8 +1113,7 @@ __global__ void __launch_bounds__(kDecThreads, 1)
                         flush();
                 } else {
                     __syncwarp();  // this warp's own records, read back by other lanes
-                    combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, pend.x, sp, lane, nullptr, nullptr,
-                                                           &mphase);
+                    combine_group<T, DD, GH, TPS_W, TPS_D>(a, s_pre, s_len, pend.x, sp, lane, nullptr);
                 }
             }
         }
