@@ -133,8 +133,10 @@ size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq);
  *   q [B][Hq][d] T; Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][d] T; q, out,
  *   Uk, Uv and the workspace 16-byte aligned.
  * A sequence with L_b == 0 gets a zero output.  Split-K over the sequence:
- * three kernels run in order on `stream` (item set-up and q~, streaming,
- * combine).  B <= DAR_DECODE_MAX_BATCH.  A length beyond the cache's capacity
+ * two kernels run in order on `stream` (q~ and zeroed counters; streaming,
+ * whose warps merge the partial results of each (sequence, KV head) group).
+ * B <= DAR_DECODE_MAX_BATCH and B * Hq * (stages of a full-capacity sequence)
+ * < 2^31, else DAR_ERR_UNSUPPORTED.  A length beyond the cache's capacity
  * or a needed block-table entry outside [0, num_pages) sets
  * *status = DAR_ERR_CAPACITY; out is then undefined for that sequence.
  */
