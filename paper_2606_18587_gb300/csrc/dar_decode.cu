@@ -1028,8 +1028,11 @@ __global__ void __launch_bounds__(kDecThreads, 1)
         npend = 0;
     };
     for (;;) {
-        // refill first, so that the copies run while a finished segment is written
-        while (issued - consumed < kStages && iss_s < hi)
+        // refill first, so that the copies run while a finished segment is written.
+        // The first fill stops one stage short: at the start every warp of the SM
+        // issues at once, and the warp should not wait on the copy unit for its
+        // last stage while its first one may already have landed.
+        while (issued - consumed < (consumed > 0 ? kStages : kStages - 1) && iss_s < hi)
             issue_one();
         if (pend.y & kMetaSegEnd) {
             // ---- segment done: write the partial result (m, l, acc) of every head
