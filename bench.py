@@ -38,7 +38,7 @@ LAUNCHES_PER_STEP = 3
 # decode-160M workload, from an ncu capture of `python bench.py --only decode`
 # (dram__bytes_read.sum + dram__bytes_write.sum); None whenever that kernel
 # has changed since the capture.
-DECODE_TRAFFIC_BYTES = None
+DECODE_TRAFFIC_BYTES = 112_347_648 + 2_752_512
 # multi-function-unit ex2 throughput per SM and the maximum SM clock (the
 # prefill's exponential roofline)
 MUFU_EX2_PER_CLK = 16
