@@ -97,15 +97,14 @@ struct DecodeLayout {
 // Workspace of dar_attn_decode: the absorbed queries, one counter per
 // (sequence, KV head, head slice) group plus the pool's claim counter, and the
 // split-K records of every range the stream kernel can run (one per warp,
-// then the pool chunks).  Every call rewrites what it reads.
+// then the pool chunks if there is a pool).  Every call rewrites what it reads.
 DecodeLayout decode_layout(const dar_cache *c, int Hq, const dar::DecodeGeometry &gm)
 {
     DecodeLayout L;
     L.qt = 0;
     L.counters = L.qt + align256((size_t)c->B * Hq * c->d_down * sizeof(float));
     L.rec = L.counters + align256(((size_t)c->B * c->Hkv * gm.HS + 1) * sizeof(int32_t));
-    const size_t ranges = (size_t)dar::kMaxDecodeCtas * dar::kDecodeWarpsPerCta + dar::kDecodePoolChunks;
-    const size_t recs = ranges * 4 * gm.GH;
+    const size_t recs = (size_t)dar::kDecodeRecordRanges * 4 * gm.GH;
     L.total = L.rec + align256(recs * dar::kRecFloats * sizeof(float));
     return L;
 }

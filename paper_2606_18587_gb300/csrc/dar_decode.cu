@@ -501,7 +501,7 @@ struct Split {
         return k;
     }
 };
-constexpr int kPoolPercent = 0;                               // share of the stages in the pool
+constexpr int kPoolPercent = kDecodePoolPercent;        // share of the stages in the pool
 constexpr int kMaxPoolChunks = kMaxDecodeCtas * kDecWarps * 2;  // pool chunks the records hold
 static_assert(kMaxPoolChunks == kDecodePoolChunks, "record slots of the pool");
 

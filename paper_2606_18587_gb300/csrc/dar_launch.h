@@ -68,12 +68,15 @@ struct DecodeGeometry {
 };
 // The decode stream kernel runs one CTA of kDecodeWarpsPerCta warps per SM, at
 // most kMaxDecodeCtas CTAs.  Its stages fall into ranges -- one per warp, then
-// up to kDecodePoolChunks pool chunks -- and each range owns 2 slots x 2 types
-// x GH records of kRecFloats floats (acc[64], m, l, padding to 16 bytes) in
-// the workspace.
+// up to kDecodePoolChunks pool chunks if kDecodePoolPercent > 0 -- and each
+// range owns 2 slots x 2 types x GH records of kRecFloats floats (acc[64], m,
+// l, padding to 16 bytes) in the workspace.
 constexpr int kDecodeWarpsPerCta = 8;
 constexpr int kMaxDecodeCtas = 160;
-constexpr int kDecodePoolChunks = 2 * kMaxDecodeCtas * kDecodeWarpsPerCta;  // ranges beyond the warps' own
+constexpr int kDecodePoolPercent = 0;  // share of the stages in the claimable pool (0: no pool)
+constexpr int kDecodePoolChunks = 2 * kMaxDecodeCtas * kDecodeWarpsPerCta;  // pool chunks at most
+// ranges the workspace holds records for: one per warp, plus the pool's chunks when there is a pool
+constexpr int kDecodeRecordRanges = kMaxDecodeCtas * kDecodeWarpsPerCta + (kDecodePoolPercent > 0 ? kDecodePoolChunks : 0);
 constexpr int kRecFloats = 68;
 DecodeGeometry decode_geometry(dar_dtype dt, int Hq, int Hkv, int dd, int w, int maxp);
 

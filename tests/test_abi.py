@@ -50,6 +50,29 @@ def test_workspace_sizes_are_host_only(lib):
     assert L.dar_prefill_workspace_bytes(lib.DAR_F32, 0, 3, 100, 16) == 0
 
 
+def _a256(x):
+    return (x + 255) // 256 * 256
+
+
+@pytest.mark.parametrize("B,Hkv,Hq,dd", [(2, 2, 4, 16), (3, 8, 32, 16), (64, 8, 32, 64), (1, 1, 1, 8)])
+def test_decode_workspace_layout(lib, B, Hkv, Hq, dd):
+    """The decode workspace: q~ [B][Hq][dd] fp32, one counter per (sequence, KV
+    head, head slice) group plus the pool's claim counter, and 2 slots x 2 types
+    x GH records of 68 floats for each of the 160 x 8 warp ranges (no pool
+    records while the pool is off) -- independent of the context capacity."""
+    L = lib.load_library()
+    G = Hq // Hkv
+    GH = 4 if G % 4 == 0 else 2 if G % 2 == 0 else 1
+    HS = G // GH
+    want = _a256(B * Hq * dd * 4) + _a256((B * Hkv * HS + 1) * 4) + _a256(160 * 8 * 4 * GH * 68 * 4)
+    for maxp in (1, 64, 4096):
+        c = _cache(lib, B=B, Hkv=Hkv, d_down=dd, max_pages_per_seq=maxp, num_pages=B * maxp)
+        assert L.dar_decode_workspace_bytes(ctypes.byref(c), Hq) == want
+    # a small cache with four query heads per KV head fits the no-alloc entry point's scratch
+    if B * Hq * dd * 4 < (1 << 20):
+        assert want <= 8 << 20
+
+
 @pytest.mark.parametrize("kw,code", [
     (dict(d=32), 2), (dict(d_down=12), 2), (dict(w=0), 1), (dict(Hkv=0), 1), (dict(dtype=7), 1),
     (dict(win_k=0), 1), (dict(win_k=258), 1), (dict(B=5000), 2), (dict(B=1025), 2),
