@@ -15,11 +15,12 @@
 //           page aligned) in stages of TPS_D tokens -- and the groups are laid
 //           end to end, ordered by sequence then group.  Every CTA builds the
 //           per-sequence stage counts and their prefix sums in shared memory.
-//           The first 3/4 of the S stages are split evenly over the NW warps
-//           of the grid (warp k owns [Ss k / NW, Ss (k + 1) / NW)); the rest
-//           is a pool of small chunks that warps claim with an atomic counter
-//           once their own range is done, so that SMs the memory system serves
-//           faster take more of it.  A range cuts groups into parts; within a
+//           The S stages are split evenly over the NW warps of the grid (warp
+//           k owns [Ss k / NW, Ss (k + 1) / NW), Ss = S); with a non-zero
+//           kDecodePoolPercent the last share of the stages instead forms a
+//           pool of small chunks that warps claim with an atomic counter once
+//           their own range is done (off: its per-chunk costs outweighed the
+//           balance it bought).  A range cuts groups into parts; within a
 //           part, the ring stages and the page stages each leave one partial
 //           result per head (running max m, sum l, unnormalised acc) in the
 //           range's record slots.  When a part ends, a group that lies inside
