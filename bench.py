@@ -274,8 +274,8 @@ def run_ours(args, world, rank, local):
 
     def step(i):
         wl = wls[i % R]
-        dar.dar_cache_append(wl.cache, knew[i % R], vnew[i % R], wl.Dk, wl.Dv)
-        dar.dar_attn_decode(wl.cache, wl.q, wl.Uk, wl.Uv, wl.workspace, out=outs[i % R])
+        dar.dar_decode_step(wl.cache, knew[i % R], vnew[i % R], wl.Dk, wl.Dv, wl.q, wl.Uk, wl.Uv, wl.workspace,
+                            out=outs[i % R])
 
     for i in range(Wm):
         step(i)
@@ -295,8 +295,8 @@ def run_ours(args, world, rank, local):
         for j in range(K):
             c = j % R
             wl = wls[c]
-            dar.dar_cache_append(wl.cache, knew[c], vnew[c], wl.Dk, wl.Dv)
-            dar.dar_attn_decode(wl.cache, wl.q, wl.Uk, wl.Uv, wl.workspace, out=outs[c])
+            dar.dar_decode_step(wl.cache, knew[c], vnew[c], wl.Dk, wl.Dv, wl.q, wl.Uk, wl.Uv, wl.workspace,
+                                out=outs[c])
     # warm the graph and size the soak
     graph.replay()
     torch.cuda.synchronize()
@@ -369,8 +369,7 @@ def run_ours(args, world, rank, local):
         wl = wls[c]
         d_in[c].copy_(h_in[c], non_blocking=True)
         k_c, v_c, q_c = views[c]
-        dar.dar_cache_append(wl.cache, k_c, v_c, wl.Dk, wl.Dv)
-        dar.dar_attn_decode(wl.cache, q_c, wl.Uk, wl.Uv, wl.workspace, out=outs[c])
+        dar.dar_decode_step(wl.cache, k_c, v_c, wl.Dk, wl.Dv, q_c, wl.Uk, wl.Uv, wl.workspace, out=outs[c])
         hout[c].copy_(outs[c], non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()

@@ -26,6 +26,11 @@
  *    caller's status word (first error wins) and the affected work is skipped;
  *    the kernels never trap.  dar_last_error() describes the last non-OK
  *    return on the calling thread.
+ *  - Every wait a kernel makes on another part of itself (a copy landing, a
+ *    tensor-core result) is bounded: after 2 s without progress the waiting
+ *    block writes DAR_ERR_DEVICE to the status word, lets its own copies in
+ *    flight land, releases its tensor memory and exits, so the caller finds a
+ *    stuck kernel on the host instead of a hung device.
  *  - `scale` <= 0 selects the default 1/sqrt(d) of Eq. 4.
  */
 #ifndef DAR_H
@@ -43,7 +48,10 @@ typedef enum {
     DAR_ERR_INVALID_ARG = 1, /* null pointer, negative size, inconsistent shape   */
     DAR_ERR_UNSUPPORTED = 2, /* valid but not built (d != 64, d_down not listed)  */
     DAR_ERR_CAPACITY = 3,    /* workspace too small / no page for a token         */
-    DAR_ERR_CUDA = 4         /* the CUDA runtime reported an error at launch      */
+    DAR_ERR_CUDA = 4,        /* the CUDA runtime reported an error at launch      */
+    DAR_ERR_DEVICE = 5       /* written to a status word: a kernel gave up on a
+                                bounded internal wait (see below) and skipped the
+                                rest of its work; the context stays usable        */
 } dar_status;
 
 typedef enum { DAR_F32 = 0, DAR_BF16 = 1 } dar_dtype;
@@ -134,7 +142,8 @@ size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq);
  *   Uk, Uv and the workspace 16-byte aligned.
  * A sequence with L_b == 0 gets a zero output.  Split-K over the sequence:
  * two kernels run in order on `stream` (q~ and zeroed counters; streaming,
- * whose warps merge the partial results of each (sequence, KV head) group).
+ * whose warps merge the partial results of each (sequence, KV head) group);
+ * the first starts only after all earlier work on the stream has finished.
  * B <= DAR_DECODE_MAX_BATCH and B * Hq * (stages of a full-capacity sequence)
  * < 2^31, else DAR_ERR_UNSUPPORTED.  A length beyond the cache's capacity
  * or a needed block-table entry outside [0, num_pages) sets
@@ -143,6 +152,22 @@ size_t dar_decode_workspace_bytes(const dar_cache *cache, int32_t Hq);
 dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, const float *Uk,
                            const float *Uv, float scale, void *out, void *workspace,
                            size_t workspace_bytes, void *stream);
+
+/*
+ * One serving step (Sec. 2.3 inference with the cache scheme of Sec. 5):
+ * dar_cache_append(cache, k_new, v_new, n, n_per_seq, Dk, Dv) followed by
+ * dar_attn_decode(cache, Hq, q, Uk, Uv, scale, out, workspace), with the same
+ * arguments, requirements and results as those two calls made in turn.  All
+ * arguments of both are checked before anything is launched.  The difference
+ * is in the ordering on the device: dar_attn_decode alone starts only after
+ * all earlier work on the stream has finished, while here the decode's
+ * query-side set-up (q~ = q Uk^T) runs while the append is still working,
+ * which is safe because the append writes neither q nor Uk.
+ */
+dar_status dar_decode_step(const dar_cache *cache, const void *k_new, const void *v_new, int32_t n,
+                           const int32_t *n_per_seq, const float *Dk, const float *Dv, int32_t Hq,
+                           const void *q, const float *Uk, const float *Uv, float scale, void *out,
+                           void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * dar_attn_decode for callers that cannot allocate device memory (the paper
@@ -189,6 +214,18 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
                             const void *v, const float *Dk, const float *Uk, const float *Dv,
                             const float *Uv, float scale, void *out, void *workspace,
                             size_t workspace_bytes, int32_t *status, void *stream);
+
+/*
+ * Diagnostic of the failure path every kernel shares (no counterpart in the
+ * paper).  Launches one thread block that allocates tensor memory, starts one
+ * bulk copy into shared memory and then waits on a barrier that nothing ever
+ * completes, with a limit of limit_us microseconds instead of the usual 2 s.
+ * When the limit runs out it does what any kernel of this library does when a
+ * wait gives up: writes DAR_ERR_DEVICE to *status (a device int32, first error
+ * wins), waits for its own copy to land, releases its tensor memory and exits.
+ * The device stays usable.  limit_us must lie in [1, 2000000].
+ */
+dar_status dar_check_bounded_wait(int32_t *status, uint32_t limit_us, void *stream);
 
 /* Message for the last non-OK return on this thread ("" if none). */
 const char *dar_last_error(void);

@@ -109,6 +109,100 @@ DecodeLayout decode_layout(const dar_cache *c, int Hq, const dar::DecodeGeometry
     return L;
 }
 
+// Checks the arguments of dar_cache_append and fills *a; *empty = nothing to launch.
+dar_status prepare_append(const dar_cache *cache, const void *k_new, const void *v_new, int32_t n,
+                          const int32_t *n_per_seq, const float *Dk, const float *Dv, dar::AppendArgs *a,
+                          bool *empty)
+{
+    dar_status s = check_cache(cache);
+    if (s != DAR_OK)
+        return s;
+    if (n < 0)
+        return fail(DAR_ERR_INVALID_ARG, "n=%d", n);
+    *empty = cache->B == 0 || n == 0;
+    if (*empty)
+        return ok();
+    if (!k_new || !v_new || !Dk || !Dv)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(Dk) || !aligned16(Dv))
+        return fail(DAR_ERR_INVALID_ARG, "k_new, v_new, Dk and Dv must be 16-byte aligned");
+    a->k_new = k_new;
+    a->v_new = v_new;
+    a->Dk = Dk;
+    a->Dv = Dv;
+    a->win_k = cache->win_k;
+    a->win_v = cache->win_v;
+    a->pool_kd = cache->pool_kd;
+    a->pool_vd = cache->pool_vd;
+    a->block_table = cache->block_table;
+    a->n_per_seq = n_per_seq;
+    a->seq_lens = cache->seq_lens;
+    a->status = cache->status;
+    a->B = cache->B;
+    a->Hkv = cache->Hkv;
+    a->n = n;
+    a->w = cache->w;
+    a->maxp = cache->max_pages_per_seq;
+    a->num_pages = cache->num_pages;
+    return ok();
+}
+
+// Checks the arguments of dar_attn_decode and fills *a; *empty = nothing to launch.
+dar_status prepare_decode(const dar_cache *cache, int32_t Hq, const void *q, const float *Uk, const float *Uv,
+                          float scale, void *out, void *workspace, size_t workspace_bytes, dar::DecodeArgs *a,
+                          bool *empty)
+{
+    dar_status s = check_cache(cache);
+    if (s != DAR_OK)
+        return s;
+    if (Hq < cache->Hkv || Hq % cache->Hkv)
+        return fail(DAR_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", Hq, cache->Hkv);
+    if (cache->B > DAR_DECODE_MAX_BATCH)
+        return fail(DAR_ERR_UNSUPPORTED, "decode batch %d > %d", cache->B, DAR_DECODE_MAX_BATCH);
+    *empty = cache->B == 0;
+    if (*empty)
+        return ok();
+    if (!q || !Uk || !Uv || !out || !workspace)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(q) || !aligned16(out) || !aligned16(Uk) || !aligned16(Uv) || !aligned16(workspace))
+        return fail(DAR_ERR_INVALID_ARG, "q, out, Uk, Uv and workspace must be 16-byte aligned");
+    dar::DecodeGeometry gm = dar::decode_geometry(cache->dtype, Hq, cache->Hkv, cache->d_down,
+                                                  cache->w, cache->max_pages_per_seq);
+    DecodeLayout L = decode_layout(cache, Hq, gm);
+    if ((double)cache->B * Hq * gm.sph >= 2147483647.0)
+        return fail(DAR_ERR_UNSUPPORTED, "B * Hq * stages = %.0f exceeds the int32 stage index",
+                    (double)cache->B * Hq * gm.sph);
+    if (workspace_bytes < L.total)
+        return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
+    char *ws = static_cast<char *>(workspace);
+    a->q = q;
+    a->out = out;
+    a->win_k = cache->win_k;
+    a->win_v = cache->win_v;
+    a->pool_kd = cache->pool_kd;
+    a->pool_vd = cache->pool_vd;
+    a->block_table = cache->block_table;
+    a->seq_lens = cache->seq_lens;
+    a->status = cache->status;
+    a->Uk = Uk;
+    a->Uv = Uv;
+    a->rec = reinterpret_cast<float *>(ws + L.rec);
+    a->qt = reinterpret_cast<float *>(ws + L.qt);
+    a->counters = reinterpret_cast<int32_t *>(ws + L.counters);
+    a->B = cache->B;
+    a->Hq = Hq;
+    a->Hkv = cache->Hkv;
+    a->G = Hq / cache->Hkv;
+    a->GH = gm.GH;
+    a->HS = gm.HS;
+    a->w = cache->w;
+    a->maxp = cache->max_pages_per_seq;
+    a->num_pages = cache->num_pages;
+    a->qscale = default_scale(scale, cache->d) * kLog2e;
+    a->prep_overlaps_prev = 0;
+    return ok();
+}
+
 }  // namespace
 
 void dar::set_last_error(const char *msg) { g_err = msg ? msg : ""; }
@@ -142,36 +236,11 @@ dar_status dar_cache_append(const dar_cache *cache, const void *k_new, const voi
                             int32_t n, const int32_t *n_per_seq, const float *Dk,
                             const float *Dv, void *stream)
 {
-    dar_status s = check_cache(cache);
-    if (s != DAR_OK)
-        return s;
-    if (n < 0)
-        return fail(DAR_ERR_INVALID_ARG, "n=%d", n);
-    if (cache->B == 0 || n == 0)
-        return ok();
-    if (!k_new || !v_new || !Dk || !Dv)
-        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
-    if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(Dk) || !aligned16(Dv))
-        return fail(DAR_ERR_INVALID_ARG, "k_new, v_new, Dk and Dv must be 16-byte aligned");
     dar::AppendArgs a;
-    a.k_new = k_new;
-    a.v_new = v_new;
-    a.Dk = Dk;
-    a.Dv = Dv;
-    a.win_k = cache->win_k;
-    a.win_v = cache->win_v;
-    a.pool_kd = cache->pool_kd;
-    a.pool_vd = cache->pool_vd;
-    a.block_table = cache->block_table;
-    a.n_per_seq = n_per_seq;
-    a.seq_lens = cache->seq_lens;
-    a.status = cache->status;
-    a.B = cache->B;
-    a.Hkv = cache->Hkv;
-    a.n = n;
-    a.w = cache->w;
-    a.maxp = cache->max_pages_per_seq;
-    a.num_pages = cache->num_pages;
+    bool empty = false;
+    dar_status s = prepare_append(cache, k_new, v_new, n, n_per_seq, Dk, Dv, &a, &empty);
+    if (s != DAR_OK || empty)
+        return s;
     return from_cuda(dar::launch_cache_append(cache->dtype, cache->d_down, a,
                                               static_cast<cudaStream_t>(stream)),
                      "dar_cache_append launch");
@@ -190,56 +259,44 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
                            const float *Uv, float scale, void *out, void *workspace,
                            size_t workspace_bytes, void *stream)
 {
-    dar_status s = check_cache(cache);
-    if (s != DAR_OK)
-        return s;
-    if (Hq < cache->Hkv || Hq % cache->Hkv)
-        return fail(DAR_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", Hq, cache->Hkv);
-    if (cache->B > DAR_DECODE_MAX_BATCH)
-        return fail(DAR_ERR_UNSUPPORTED, "decode batch %d > %d", cache->B, DAR_DECODE_MAX_BATCH);
-    if (cache->B == 0)
-        return ok();
-    if (!q || !Uk || !Uv || !out || !workspace)
-        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
-    if (!aligned16(q) || !aligned16(out) || !aligned16(Uk) || !aligned16(Uv) || !aligned16(workspace))
-        return fail(DAR_ERR_INVALID_ARG, "q, out, Uk, Uv and workspace must be 16-byte aligned");
-    dar::DecodeGeometry gm = dar::decode_geometry(cache->dtype, Hq, cache->Hkv, cache->d_down,
-                                                  cache->w, cache->max_pages_per_seq);
-    DecodeLayout L = decode_layout(cache, Hq, gm);
-    if ((double)cache->B * Hq * gm.sph >= 2147483647.0)
-        return fail(DAR_ERR_UNSUPPORTED, "B * Hq * stages = %.0f exceeds the int32 stage index",
-                    (double)cache->B * Hq * gm.sph);
-    if (workspace_bytes < L.total)
-        return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
-    char *ws = static_cast<char *>(workspace);
     dar::DecodeArgs a;
-    a.q = q;
-    a.out = out;
-    a.win_k = cache->win_k;
-    a.win_v = cache->win_v;
-    a.pool_kd = cache->pool_kd;
-    a.pool_vd = cache->pool_vd;
-    a.block_table = cache->block_table;
-    a.seq_lens = cache->seq_lens;
-    a.status = cache->status;
-    a.Uk = Uk;
-    a.Uv = Uv;
-    a.rec = reinterpret_cast<float *>(ws + L.rec);
-    a.qt = reinterpret_cast<float *>(ws + L.qt);
-    a.counters = reinterpret_cast<int32_t *>(ws + L.counters);
-    a.B = cache->B;
-    a.Hq = Hq;
-    a.Hkv = cache->Hkv;
-    a.G = Hq / cache->Hkv;
-    a.GH = gm.GH;
-    a.HS = gm.HS;
-    a.w = cache->w;
-    a.maxp = cache->max_pages_per_seq;
-    a.num_pages = cache->num_pages;
-    a.qscale = default_scale(scale, cache->d) * kLog2e;
+    bool empty = false;
+    dar_status s = prepare_decode(cache, Hq, q, Uk, Uv, scale, out, workspace, workspace_bytes, &a, &empty);
+    if (s != DAR_OK || empty)
+        return s;
+    a.prep_overlaps_prev = 0;  // the kernel before this call is the caller's: wait for it
     return from_cuda(dar::launch_decode(cache->dtype, cache->d_down, a,
                                         static_cast<cudaStream_t>(stream)),
                      "dar_attn_decode launch");
+}
+
+dar_status dar_decode_step(const dar_cache *cache, const void *k_new, const void *v_new, int32_t n,
+                           const int32_t *n_per_seq, const float *Dk, const float *Dv, int32_t Hq,
+                           const void *q, const float *Uk, const float *Uv, float scale, void *out,
+                           void *workspace, size_t workspace_bytes, void *stream)
+{
+    // every argument of both operations is checked before anything is launched
+    dar::AppendArgs ap;
+    dar::DecodeArgs dc;
+    bool app_empty = false, dec_empty = false;
+    dar_status s = prepare_append(cache, k_new, v_new, n, n_per_seq, Dk, Dv, &ap, &app_empty);
+    if (s != DAR_OK)
+        return s;
+    s = prepare_decode(cache, Hq, q, Uk, Uv, scale, out, workspace, workspace_bytes, &dc, &dec_empty);
+    if (s != DAR_OK)
+        return s;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (!app_empty) {
+        s = from_cuda(dar::launch_cache_append(cache->dtype, cache->d_down, ap, st), "dar_decode_step append launch");
+        if (s != DAR_OK)
+            return s;
+    }
+    if (dec_empty)
+        return ok();
+    // the kernel just before the decode is the append above, which writes
+    // neither q nor Uk: the decode's query-side set-up may overlap it
+    dc.prep_overlaps_prev = app_empty ? 0 : 1;
+    return from_cuda(dar::launch_decode(cache->dtype, cache->d_down, dc, st), "dar_decode_step decode launch");
 }
 
 size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t N,

@@ -252,16 +252,18 @@ template <typename T>
 static cudaError_t cache_append_t(int dd, const AppendArgs &a, cudaStream_t s)
 {
     const size_t smem = (size_t)app_rows<T>(a.Hkv) * 2 * a.Hkv * kHeadDim * sizeof(T);
-    static bool attr = false;  // one-time opt-in to more than 48 KB of shared memory
-    if (!attr) {
+    static PerDeviceOnce once;  // opt-in to more than 48 KB of shared memory, once per device
+    const cudaError_t e = per_device_once(once, [](int) {
         for (auto k : {cache_append_kernel<T, 8>, cache_append_kernel<T, 16>, cache_append_kernel<T, 32>,
                        cache_append_kernel<T, 64>}) {
-            const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kAppStageBytes);
-            if (e != cudaSuccess)
-                return e;
+            const cudaError_t e2 = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kAppStageBytes);
+            if (e2 != cudaSuccess)
+                return e2;
         }
-        attr = true;
-    }
+        return cudaSuccess;
+    });
+    if (e != cudaSuccess)
+        return e;
     switch (dd) {
     case 8: cache_append_kernel<T, 8><<<a.B, kAppThreads, smem, s>>>(a); break;
     case 16: cache_append_kernel<T, 16><<<a.B, kAppThreads, smem, s>>>(a); break;

@@ -1,13 +1,15 @@
 // dar_decode.cu -- one decode step of DAR attention over the mixed-dimension
 // cache (Eq. 3-4 for the query at position L_b - 1; cache scheme of Sec. 5).
 //
-// Two kernels on the caller's stream, both launched with programmatic stream
-// serialisation:
+// Two kernels on the caller's stream:
 //
 //  prep     q~ = q Uk^T for every query row (W_up absorbed into the query,
 //           exact by linearity of Eq. 2) and zeroed group counters.  Neither
-//           needs the cache, so this overlaps the kernel before it (normally
-//           the cache append); it waits for that kernel before exiting.
+//           needs the cache, so when the kernel before it is this library's
+//           cache append (dar_decode_step) prep is launched with programmatic
+//           stream serialisation and overlaps it; it waits for that kernel
+//           before exiting.  Otherwise it starts after all earlier work.
+//           The stream kernel is always launched programmatically after prep.
 //  stream   split-K over the sequence, balanced per warp (stream-K).  The
 //           work of a group (sequence b, KV head g, head slice hs) is a run
 //           of stages -- the ring's tokens (full d = 64 keys/values) in
@@ -104,7 +106,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, int32_
 {
     if (sm100::mbar_wait(bar, parity, nullptr))
         return true;
-    report(status, DAR_ERR_CUDA);
+    report(status, DAR_ERR_DEVICE);
     return false;
 }
 
@@ -157,10 +159,10 @@ constexpr size_t decode_smem_bytes(int B)
 
 // q~ = q Uk^T for every (b, h) row, one row per warp (fp32, four partial sums
 // over t mod 4), and zeroed group counters.  Neither depends on the cache, so
-// with programmatic launch this kernel runs while the kernel before it
-// (normally the cache append) finishes; it waits for that kernel before
-// exiting, so the stream kernel, which waits for this one, sees the finished
-// cache.
+// when launched programmatically after the cache append (which writes neither
+// q nor Uk) this kernel runs while the append finishes; it waits for the
+// kernel before it before exiting, so the stream kernel, which waits for this
+// one, sees the finished cache.
 template <typename T, int DD>
 __global__ void __launch_bounds__(kPrepThreads) decode_prep_kernel(DecodeArgs a)
 {
@@ -1375,35 +1377,45 @@ static cudaError_t decode_t(const DecodeArgs &a, cudaStream_t s)
     }
     // one-time set-up per instantiation (kept out of the launch path so launches
     // stay cheap and can be captured in a CUDA graph)
-    static int ctas = 0;
-    if (ctas == 0) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)decode_smem_bytes(DAR_DECODE_MAX_BATCH));
-        if (e != cudaSuccess)
-            return e;
-        int dev = 0, n = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        ctas = n < kMaxDecodeCtas ? n : kMaxDecodeCtas;  // the workspace holds records for this many
-    }
+    static PerDeviceOnce once;
+    int ctas = 0;
+    cudaError_t e = per_device_once(
+        once,
+        [&](int dev) {
+            cudaError_t e2 = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                  (int)decode_smem_bytes(DAR_DECODE_MAX_BATCH));
+            int n = 0;
+            if (e2 == cudaSuccess)
+                e2 = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+            once.value[dev] = n < kMaxDecodeCtas ? n : kMaxDecodeCtas;  // the workspace holds records for this many
+            return e2;
+        },
+        &ctas);
+    if (e != cudaSuccess)
+        return e;
     const int rows = a.B * a.Hq;
     const int prep_blocks = min(2 * ctas, max(1, (rows + kPrepThreads / 32 - 1) / (kPrepThreads / 32)));
-    // both kernels use programmatic launch: prep computes q~ while the kernel
-    // before it finishes (and waits for it before exiting); the stream kernel
-    // sets up while prep drains
+    // The stream kernel always uses programmatic launch: it sets up while prep
+    // drains (prep is this library's own kernel and writes nothing the set-up
+    // reads).  prep itself reads q and Uk before its dependency wait, so it may
+    // overlap the kernel before it only when the caller vouches that this
+    // kernel writes neither (a.prep_overlaps_prev: this library's own cache
+    // append, launched by dar_decode_step); otherwise it starts after all
+    // earlier work on the stream has finished.
     cudaLaunchAttribute pdl[1];
     pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     pdl[0].val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.stream = s;
     cfg.attrs = pdl;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = a.prep_overlaps_prev ? 1 : 0;
     cfg.gridDim = dim3(prep_blocks);
     cfg.blockDim = dim3(kPrepThreads);
-    cudaError_t e = cudaLaunchKernelEx(&cfg, decode_prep_kernel<T, DD>, a);
+    e = cudaLaunchKernelEx(&cfg, decode_prep_kernel<T, DD>, a);
     if (e != cudaSuccess)
         return e;
     // one CTA per SM (the records of the workspace are sized for kMaxDecodeCtas)
+    cfg.numAttrs = 1;
     cfg.gridDim = dim3(ctas);
     cfg.blockDim = dim3(kDecThreads);
     cfg.dynamicSmemBytes = decode_smem_bytes(a.B);

@@ -16,8 +16,9 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_decode_scratch[DAR_DECODE_NOALLOC_MAX_BYTES];
 
-constexpr int kMaxDevices = 64;
-void *g_scratch_ptr[kMaxDevices] = {};  // device address of g_decode_scratch, per device
+// device address of g_decode_scratch, looked up once per device (thread-safe)
+dar::PerDeviceOnce g_scratch_once;
+void *g_scratch_ptr[dar::kMaxDevices] = {};
 
 }  // namespace
 
@@ -26,20 +27,23 @@ extern "C" dar_status dar_attn_decode_noalloc(const dar_cache *cache, int32_t Hq
                                               void *stream)
 {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= dar::kMaxDevices) {
         dar::set_last_error("dar_attn_decode_noalloc: no usable current device");
         return DAR_ERR_CUDA;
     }
     // One-time set-up on this device (with it current): the host-side name of
     // the array is not a device address, so ask the runtime for the address.
-    if (!g_scratch_ptr[dev]) {
+    const cudaError_t e = dar::per_device_once(g_scratch_once, [](int d) {
         void *p = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&p, g_decode_scratch);
-        if (e != cudaSuccess || !p) {
-            dar::set_last_error(cudaGetErrorString(e));
-            return DAR_ERR_CUDA;
-        }
-        g_scratch_ptr[dev] = p;
+        cudaError_t e2 = cudaGetSymbolAddress(&p, g_decode_scratch);
+        if (e2 == cudaSuccess && !p)
+            e2 = cudaErrorInvalidSymbol;
+        g_scratch_ptr[d] = p;
+        return e2;
+    });
+    if (e != cudaSuccess) {
+        dar::set_last_error(cudaGetErrorString(e));
+        return DAR_ERR_CUDA;
     }
     const size_t need = dar_decode_workspace_bytes(cache, Hq);
     if (need == 0)  // invalid cache or Hq: the regular entry point reports which, launching nothing

@@ -6,6 +6,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "dar.h"
 
 namespace dar {
@@ -36,6 +38,10 @@ struct DecodeArgs {
     int32_t *counters;  // [B][Hkv][HS] finished stages per group, then the pool's claim counter
     int B, Hq, Hkv, G, GH, HS, w, maxp, num_pages;
     float qscale;  // scale * log2(e)
+    // the kernel before the decode on the stream is this library's cache
+    // append (which writes neither q nor Uk): the decode's query-side set-up
+    // may overlap it
+    int prep_overlaps_prev;
 };
 
 struct PrefillArgs {
@@ -86,5 +92,33 @@ bool make_tma_2d_bf16(CUtensorMap *map, const void *base, unsigned long long row
 
 // Set the message dar_last_error() returns on this thread.
 void set_last_error(const char *msg);
+
+// One-time set-up per device: kernel attributes (such as the shared-memory
+// opt-in) apply only to the device that is current when they are set, so each
+// device runs the set-up once, with itself current.  Thread-safe; a failed
+// set-up keeps its error.
+constexpr int kMaxDevices = 64;
+struct PerDeviceOnce {
+    std::once_flag flag[kMaxDevices];
+    cudaError_t err[kMaxDevices] = {};
+    int value[kMaxDevices] = {};  // whatever the set-up records (e.g. a CTA count)
+};
+
+// Runs fn(dev) once for the current device dev; returns its error and stores
+// *value = the value fn recorded (fn returns cudaError_t and may write o.value[dev]).
+template <typename F>
+cudaError_t per_device_once(PerDeviceOnce &o, F &&fn, int *value = nullptr)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return e;
+    if (dev < 0 || dev >= kMaxDevices)
+        return cudaErrorInvalidDevice;
+    std::call_once(o.flag[dev], [&] { o.err[dev] = fn(dev); });
+    if (value)
+        *value = o.value[dev];
+    return o.err[dev];
+}
 
 }  // namespace dar

@@ -184,13 +184,12 @@ static cudaError_t simt_t(const PrefillArgs &a, cudaStream_t s)
 {
     auto kern = prefill_simt_kernel<T, DD>;
     const size_t smem = simt_smem_floats<DD>() * sizeof(float);
-    static bool configured = false;  // one-time attribute set-up per instantiation
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess)
-            return e;
-        configured = true;
-    }
+    static PerDeviceOnce once;  // attribute set-up per instantiation and device
+    const cudaError_t e = per_device_once(once, [&](int) {
+        return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    });
+    if (e != cudaSuccess)
+        return e;
     dim3 grid((a.N + kSimtRows - 1) / kSimtRows, a.B * a.Hq);
     kern<<<grid, 256, smem, s>>>(a);
     return cudaGetLastError();

@@ -553,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     __syncthreads();
     tc_fence_after();
     if (threadIdx.x == 0 && *abort_flag)
-        report(a.status, DAR_ERR_CUDA);
+        report(a.status, DAR_ERR_DEVICE);
     if (warp == 1)
         tmem_dealloc(tmem, kTmemCols);
 }
@@ -612,13 +612,12 @@ static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
         return cudaErrorInvalidValue;
     auto kern = prefill_tc_kernel<DP>;
     const size_t smem = Layout<DP>::TOTAL + 1024;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess)
-            return e;
-        configured = true;
-    }
+    static PerDeviceOnce once;
+    cudaError_t e = per_device_once(once, [&](int) {
+        return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    });
+    if (e != cudaSuccess)
+        return e;
     dim3 grid(a.B * a.Hq, (a.N + BM - 1) / BM);
     kern<<<grid, kThreads, smem, s>>>(mq, mqt, mk, mv, mkd, mvd, a);
     return cudaGetLastError();

@@ -80,10 +80,11 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, unsigned pari
     return ok != 0;
 }
 
-// Wait for the phase with the given parity.  Gives up after kWaitLimitNs of
-// wall time, or as soon as *abort is set by another thread; returns false
-// then (and sets *abort).
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, volatile int *abort)
+// Wait for the phase with the given parity.  Gives up after limit_ns of wall
+// time (kWaitLimitNs unless a caller asks for less), or as soon as *abort is
+// set by another thread; returns false then (and sets *abort).
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, volatile int *abort,
+                                          unsigned long long limit_ns = kWaitLimitNs)
 {
     if (mbar_try_wait(bar, parity))
         return true;
@@ -94,7 +95,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, unsigned parity, volati
         if ((i & 7u) == 0u) {
             if (abort && *abort)
                 return false;
-            if (globaltimer_ns() - t0 > kWaitLimitNs)
+            if (globaltimer_ns() - t0 > limit_ns)
                 break;
         }
     }

@@ -18,7 +18,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libdar_gb300.so")
 HEADER = os.path.join(os.path.dirname(_HERE), "include", "dar.h")
 
-DAR_OK, DAR_ERR_INVALID_ARG, DAR_ERR_UNSUPPORTED, DAR_ERR_CAPACITY, DAR_ERR_CUDA = range(5)
+DAR_OK, DAR_ERR_INVALID_ARG, DAR_ERR_UNSUPPORTED, DAR_ERR_CAPACITY, DAR_ERR_CUDA, DAR_ERR_DEVICE = range(6)
 DAR_F32, DAR_BF16 = 0, 1
 PAGE_SIZE = 64
 _TORCH_DTYPE = {DAR_F32: torch.float32, DAR_BF16: torch.bfloat16}
@@ -63,6 +63,8 @@ def load_library(path: str = LIB_PATH):
         "dar_decode_workspace_bytes": ([CP, I32], SZ),
         "dar_attn_decode": ([CP, I32, P, P, P, F, P, P, SZ, P], ctypes.c_int),
         "dar_attn_decode_noalloc": ([CP, I32, P, P, P, F, P, P], ctypes.c_int),
+        "dar_decode_step": ([CP, P, P, I32, P, P, P, I32, P, P, P, F, P, P, SZ, P], ctypes.c_int),
+        "dar_check_bounded_wait": ([P, ctypes.c_uint32, P], ctypes.c_int),
         "dar_prefill_workspace_bytes": ([ctypes.c_int, I32, I32, I32, I32], SZ),
         "dar_attn_prefill": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, P, P,
                               SZ, P, P], ctypes.c_int),
@@ -212,6 +214,37 @@ def dar_attn_decode(cache: DarCache, q, Uk, Uv, workspace, scale=0.0, out=None, 
                                           _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                           _stream(stream)))
     return out
+
+
+def dar_decode_step(cache: DarCache, k_new, v_new, Dk, Dv, q, Uk, Uv, workspace, scale=0.0, out=None,
+                    n_per_seq=None, stream=None):
+    """dar_cache_append of ``k_new, v_new [B,Hkv,n,d]`` then dar_attn_decode of
+    ``q [B,Hq,d]``, in one call (the decode's query set-up overlaps the append)."""
+    _dev(k_new, "k_new", cache.dtype)
+    _dev(v_new, "v_new", cache.dtype)
+    _dev(Dk, "Dk", torch.float32)
+    _dev(Dv, "Dv", torch.float32)
+    _dev(q, "q", cache.dtype)
+    _dev(Uk, "Uk", torch.float32)
+    _dev(Uv, "Uv", torch.float32)
+    _dev(workspace, "workspace")
+    if n_per_seq is not None:
+        _dev(n_per_seq, "n_per_seq", torch.int32)
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", cache.dtype)
+    _check(load_library().dar_decode_step(
+        cache.struct, _ptr(k_new), _ptr(v_new), k_new.shape[2], _ptr(n_per_seq), _ptr(Dk), _ptr(Dv), q.shape[1],
+        _ptr(q), _ptr(Uk), _ptr(Uv), float(scale), _ptr(out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+    return out
+
+
+def dar_check_bounded_wait(status, limit_us: int, stream=None):
+    """Run the library's wait-gives-up path on a barrier nothing completes;
+    ``status`` (device int32) receives DAR_ERR_DEVICE after ``limit_us``."""
+    _dev(status, "status", torch.int32)
+    _check(load_library().dar_check_bounded_wait(_ptr(status), int(limit_us), _stream(stream)))
 
 
 def dar_attn_decode_noalloc(cache: DarCache, q, Uk, Uv, scale=0.0, out=None, stream=None):

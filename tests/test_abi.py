@@ -116,3 +116,29 @@ def test_append_rejects_bad_arguments(lib):
     assert L.dar_cache_append(ctypes.byref(c), 0, 256, 4, None, 256, 256, None) == 1
     assert L.dar_cache_append(ctypes.byref(_cache(lib, w=0)), 256, 256, 4, None, 256, 256, None) == 1
     assert L.dar_cache_append(ctypes.byref(c), 256, 256, 0, None, 256, 256, None) == 0
+
+
+def test_decode_step_checks_both_halves_before_launching(lib):
+    """dar_decode_step refuses a bad append or a bad decode argument on the
+    host (the same codes as the two calls alone), launching neither."""
+    L = lib.load_library()
+    c = _cache(lib)
+    P = 4096
+
+    def call(kn=P, n=1, Hq=4, q=P, ws=P, wsb=1 << 30, cache=c):
+        return L.dar_decode_step(ctypes.byref(cache), kn, P, n, None, P, P, Hq, q, P, P, 0.0, P, ws, wsb, None)
+    assert call(kn=0) == 1          # append: NULL k_new
+    assert call(n=-1) == 1          # append: negative count
+    assert call(Hq=3) == 1          # decode: Hq not a multiple of Hkv
+    assert call(q=P + 8) == 1       # decode: misaligned query
+    assert call(wsb=16) == 3        # decode: workspace too small
+    assert "workspace" in L.dar_last_error().decode()
+    assert call(cache=_cache(lib, d=32)) == 2
+
+
+def test_bounded_wait_check_rejects_bad_arguments(lib):
+    L = lib.load_library()
+    assert L.dar_check_bounded_wait(None, 1000, None) == 1
+    assert L.dar_check_bounded_wait(4096, 0, None) == 1
+    assert L.dar_check_bounded_wait(4096, 2000001, None) == 1
+    assert "limit_us" in L.dar_last_error().decode()
