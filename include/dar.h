@@ -202,9 +202,8 @@ size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int3
  *   q [B][Hq][N][d], k, v [B][Hkv][N][d] T; Dk, Dv [Hkv][d][d_down] fp32;
  *   Uk, Uv [Hkv][d_down][d] fp32; out [B][Hq][N][d] T.
  * w >= 0; w = 0 is the paper's uniform reduction (no token is local).
- * The workspace (no initialisation needed) receives k^D, v^D.  For bf16, out
- * also serves as scratch during the call (it first receives q~ = q Uk^T), so
- * out must not overlap q, k, v or the workspace.  `status` (a device int32,
+ * The workspace (no initialisation needed) receives k^D, v^D; out must not
+ * overlap q, k, v or the workspace.  `status` (a device int32,
  * may be NULL) is set to a dar_status if a kernel gives up on a bounded
  * internal wait; the caller clears it.  bf16 runs on the tcgen05 tensor
  * cores, fp32 on the CUDA cores (fp32 FMA, no TF32).

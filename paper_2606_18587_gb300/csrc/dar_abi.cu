@@ -336,9 +336,7 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
     char *kd = static_cast<char *>(workspace);
     char *vd = kd + need / 2;
     const int kstride = dar::prefill_kd_stride(dtype, d_down);
-    cudaError_t e = dar::launch_down_project(dtype, d_down, k, Dk, kd, B, Hkv, N, kstride, st);
-    if (e == cudaSuccess)
-        e = dar::launch_down_project(dtype, d_down, v, Dv, vd, B, Hkv, N, kstride, st);
+    cudaError_t e = dar::launch_down_project_kv(dtype, d_down, k, v, Dk, Dv, kd, vd, B, Hkv, N, kstride, st);
     if (e != cudaSuccess)
         return from_cuda(e, "dar_attn_prefill down-projection launch");
     dar::PrefillArgs a;

@@ -11,50 +11,127 @@
 namespace dar {
 
 // ---------------------------------------------------------------- bulk Eq. 1
-// grid (ceil(n / 128), B * Hkv), 128 threads; one thread per token row.
-template <typename T, int DD>
-__global__ void __launch_bounds__(128) down_project_kernel(const T *__restrict__ x,
-                                                           const float *__restrict__ W,
-                                                           T *__restrict__ out, int Hkv, int n,
-                                                           int ostride)
-{
-    __shared__ float Ws[kHeadDim * DD];
-    const int bg = blockIdx.y;
-    const int g = bg % Hkv;
-    for (int i = threadIdx.x; i < kHeadDim * DD; i += blockDim.x)
-        Ws[i] = W[(size_t)g * kHeadDim * DD + i];
-    __syncthreads();
+//
+// A block stages kStageBytesBulk of contiguous token rows in shared memory
+// with coalesced 16-byte loads (chunk c of row r stored at chunk c ^ (r & 7),
+// so a warp reading one chunk of 32 different rows touches every bank group
+// once); then each thread runs the chains of RPT rows at once, so that every
+// W[t][c] read from shared memory feeds RPT rows.  Two chains advance per
+// instruction (fma.rn.f32x2: outputs c and c + 1 share x_t); each element is
+// still the exact fp32 chain acc = fma(x_t, W[t][c], acc), t = 0..63.
+// blockIdx.z selects the tensor: 0 = (x0, W0, out0), 1 = (x1, W1, out1).
+constexpr int kStageBytesBulk = 32 << 10;
 
-    const int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= n)
-        return;
+template <typename T>
+__host__ __device__ constexpr int rows_bulk()
+{
+    return kStageBytesBulk / (kHeadDim * (int)sizeof(T));
+}
+template <int DD>
+__host__ __device__ constexpr int rows_per_thread()
+{
+    return DD <= 16 ? 4 : DD == 32 ? 2 : 1;
+}
+template <typename T, int DD>
+__host__ __device__ constexpr int threads_bulk()
+{
+    return rows_bulk<T>() / rows_per_thread<DD>();
+}
+
+struct BulkArgs {
+    const void *x[2];
+    const float *W[2];
+    void *out[2];
+    int Hkv, n, ostride;
+};
+
+template <typename T, int DD>
+__global__ void __launch_bounds__(threads_bulk<T, DD>()) down_project_kernel(BulkArgs a)
+{
+    constexpr int R = rows_bulk<T>();
+    constexpr int RPT = rows_per_thread<DD>();
+    constexpr int NT = threads_bulk<T, DD>();
     constexpr int E = Granule<T>::kElems;
-    const T *row = x + ((size_t)bg * n + j) * kHeadDim;
-    float xv[kHeadDim];
-#pragma unroll
-    for (int q = 0; q < kHeadDim / E; ++q) {
-        uint4 r = *reinterpret_cast<const uint4 *>(row + q * E);
-        float f[E];
-        unpack(r, f, T());
-#pragma unroll
-        for (int e = 0; e < E; ++e)
-            xv[q * E + e] = f[e];
+    constexpr int CPR = kHeadDim / E;  // 16-byte chunks per row (8 for bf16, 16 for fp32)
+    __shared__ __align__(16) unsigned char rows[kStageBytesBulk];
+    __shared__ __align__(16) float Ws[kHeadDim * DD];
+    const bool z = blockIdx.z != 0;  // (selects, not indexes: the arguments stay in parameter space)
+    const T *x = static_cast<const T *>(z ? a.x[1] : a.x[0]);
+    const int bg = blockIdx.y, g = bg % a.Hkv;
+    const int j0 = blockIdx.x * R;
+    const int nr = min(R, a.n - j0);
+    const float *W = (z ? a.W[1] : a.W[0]) + (size_t)g * kHeadDim * DD;
+    for (int i = threadIdx.x; i < kHeadDim * DD / 4; i += NT)
+        reinterpret_cast<float4 *>(Ws)[i] = __ldg(reinterpret_cast<const float4 *>(W) + i);
+    const uint4 *src = reinterpret_cast<const uint4 *>(x + ((size_t)bg * a.n + j0) * kHeadDim);
+    for (int i = threadIdx.x; i < nr * CPR; i += NT) {
+        const int r = i / CPR, c = i % CPR;
+        reinterpret_cast<uint4 *>(rows)[r * CPR + (c ^ (r & 7))] = ld_stream_v4(src + i);
     }
-    float acc[DD];
+    __syncthreads();
+    // this thread's rows: threadIdx.x + k * NT, k < RPT (rows past nr compute on
+    // stale staging bytes and are not stored)
+    float acc[RPT][DD];
 #pragma unroll
-    for (int c = 0; c < DD; ++c)
-        acc[c] = 0.0f;
-#pragma unroll
-    for (int t = 0; t < kHeadDim; ++t)
+    for (int k = 0; k < RPT; ++k)
 #pragma unroll
         for (int c = 0; c < DD; ++c)
-            acc[c] = __fmaf_rn(xv[t], Ws[t * DD + c], acc[c]);
-    T *o = out + ((size_t)bg * n + j) * ostride;
+            acc[k][c] = 0.0f;
+#pragma unroll 1
+    for (int q = 0; q < CPR; ++q) {
+        float xf[RPT][E];
 #pragma unroll
-    for (int c = 0; c < DD; ++c)
-        o[c] = from_f32<T>(acc[c]);
-    for (int c = DD; c < ostride; ++c)
-        o[c] = from_f32<T>(0.f);
+        for (int k = 0; k < RPT; ++k) {
+            const int r = threadIdx.x + k * NT;
+            unpack(reinterpret_cast<const uint4 *>(rows)[r * CPR + (q ^ (r & 7))], xf[k], T());
+        }
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            const int t = q * E + e;
+#pragma unroll
+            for (int c = 0; c < DD; c += 4) {
+                const float4 w4 = *reinterpret_cast<const float4 *>(Ws + t * DD + c);
+#pragma unroll
+                for (int k = 0; k < RPT; ++k) {
+                    sm100::ffma2(acc[k][c], acc[k][c + 1], xf[k][e], xf[k][e], w4.x, w4.y, acc[k][c], acc[k][c + 1]);
+                    sm100::ffma2(acc[k][c + 2], acc[k][c + 3], xf[k][e], xf[k][e], w4.z, w4.w, acc[k][c + 2],
+                                 acc[k][c + 3]);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < RPT; ++k) {
+        const int r = threadIdx.x + k * NT;
+        if (r >= nr)
+            continue;
+        T *o = static_cast<T *>(z ? a.out[1] : a.out[0]) + ((size_t)bg * a.n + j0 + r) * a.ostride;
+        if (a.ostride == DD && (DD * sizeof(T)) % 16 == 0) {
+            constexpr int OE = 16 / sizeof(T);
+#pragma unroll
+            for (int c = 0; c < DD; c += OE) {
+                uint32_t u[4];
+                if constexpr (sizeof(T) == 2) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        __nv_bfloat162 v = __floats2bfloat162_rn(acc[k][c + 2 * i], acc[k][c + 2 * i + 1]);
+                        u[i] = *reinterpret_cast<uint32_t *>(&v);
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        u[i] = __float_as_uint(acc[k][c + i]);
+                }
+                *reinterpret_cast<uint4 *>(o + c) = make_uint4(u[0], u[1], u[2], u[3]);
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < DD; ++c)
+                o[c] = from_f32<T>(acc[k][c]);
+            for (int c = DD; c < a.ostride; ++c)
+                o[c] = from_f32<T>(0.f);
+        }
+    }
 }
 
 // ------------------------------------------------------------ cache append
@@ -223,29 +300,40 @@ __global__ void __launch_bounds__(kAppThreads) cache_append_kernel(AppendArgs a)
 // ----------------------------------------------------------------- launchers
 
 template <typename T>
-static cudaError_t down_project_t(int dd, const void *x, const float *W, void *out, int B,
-                                  int Hkv, int n, int os, cudaStream_t s)
+static cudaError_t down_project_t(int dd, const BulkArgs &a, int B, int nz, cudaStream_t s)
 {
-    dim3 grid((n + 127) / 128, B * Hkv);
-    const T *xi = static_cast<const T *>(x);
-    T *o = static_cast<T *>(out);
+    constexpr int R = rows_bulk<T>();
+    dim3 grid((a.n + R - 1) / R, B * a.Hkv, nz);
     switch (dd) {
-    case 8: down_project_kernel<T, 8><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
-    case 16: down_project_kernel<T, 16><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
-    case 32: down_project_kernel<T, 32><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
-    case 64: down_project_kernel<T, 64><<<grid, 128, 0, s>>>(xi, W, o, Hkv, n, os); break;
+    case 8: down_project_kernel<T, 8><<<grid, threads_bulk<T, 8>(), 0, s>>>(a); break;
+    case 16: down_project_kernel<T, 16><<<grid, threads_bulk<T, 16>(), 0, s>>>(a); break;
+    case 32: down_project_kernel<T, 32><<<grid, threads_bulk<T, 32>(), 0, s>>>(a); break;
+    case 64: down_project_kernel<T, 64><<<grid, threads_bulk<T, 64>(), 0, s>>>(a); break;
     default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();
 }
 
+static cudaError_t down_project_any(dar_dtype dt, int dd, const BulkArgs &a, int B, int nz, cudaStream_t s)
+{
+    if (a.n == 0 || B == 0)
+        return cudaSuccess;
+    return dt == DAR_F32 ? down_project_t<float>(dd, a, B, nz, s) : down_project_t<bf16>(dd, a, B, nz, s);
+}
+
 cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float *W, void *out,
                                 int B, int Hkv, int n, int ostride, cudaStream_t s)
 {
-    if (n == 0 || B == 0)
-        return cudaSuccess;
-    return dt == DAR_F32 ? down_project_t<float>(dd, x, W, out, B, Hkv, n, ostride, s)
-                         : down_project_t<bf16>(dd, x, W, out, B, Hkv, n, ostride, s);
+    BulkArgs a = {{x, x}, {W, W}, {out, out}, Hkv, n, ostride};
+    return down_project_any(dt, dd, a, B, 1, s);
+}
+
+cudaError_t launch_down_project_kv(dar_dtype dt, int dd, const void *k, const void *v, const float *Dk,
+                                   const float *Dv, void *kd, void *vd, int B, int Hkv, int n, int ostride,
+                                   cudaStream_t s)
+{
+    BulkArgs a = {{k, v}, {Dk, Dv}, {kd, vd}, Hkv, n, ostride};
+    return down_project_any(dt, dd, a, B, 2, s);
 }
 
 template <typename T>

@@ -62,6 +62,10 @@ inline int prefill_kd_stride(dar_dtype dt, int dd) { return (dt == DAR_BF16 && d
 // Eq. 1 into rows of `ostride` elements (entries dd..ostride-1 are zeroed).
 cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float *W, void *out,
                                 int B, int Hkv, int n, int ostride, cudaStream_t s);
+// The same for keys and values in one launch: kd = k Dk, vd = v Dv.
+cudaError_t launch_down_project_kv(dar_dtype dt, int dd, const void *k, const void *v, const float *Dk,
+                                   const float *Dv, void *kd, void *vd, int B, int Hkv, int n, int ostride,
+                                   cudaStream_t s);
 cudaError_t launch_cache_append(dar_dtype dt, int dd, const AppendArgs &a, cudaStream_t s);
 cudaError_t launch_decode(dar_dtype dt, int dd, const DecodeArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_simt(dar_dtype dt, int dd, const PrefillArgs &a, cudaStream_t s);

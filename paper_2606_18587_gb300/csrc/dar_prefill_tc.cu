@@ -7,22 +7,32 @@
 //   local part   S_loc  = Q  K^T       (M128 N64 K64)   O_loc  += P_loc  V    (N64)
 //   global part  S_glob = Q~ (K^D)^T   (M128 N64 Kdd)   O_glob += P_glob V^D  (Ndd)
 // with q~ = q Uk^T (W_up absorbed into the query, exact by linearity of
-// Eq. 2).  A tile that holds both kinds (the window edge crosses it) is run
-// as two virtual tiles, each with the other kind masked out.  One online
-// softmax over every virtual tile (Eq. 4), with the running max raised lazily
-// (only when it grows by more than 2^8), and the epilogue lifts the global
-// part once:  o = (O_loc + O_glob Uv) / l.
+// Eq. 2), computed at the start of the CTA by one more tensor-core product
+// (Q times Uk^T, M128 N(dd) K64) and kept in shared memory as a bf16 operand.
+// A tile that holds both kinds (the window edge crosses it) is run as two
+// virtual tiles, each with the other kind masked out.  One online softmax over
+// every virtual tile (Eq. 4), with the running max raised lazily (only when it
+// grows by more than 2^8), and the epilogue lifts the global part once:
+//   o = (O_loc + O_glob Uv) / l.
+// The softmax denominator l is summed by the tensor core as well: each P also
+// multiplies a block of ones into 16 extra accumulator columns, so l adds up
+// exactly the bf16 weights the numerators use and is rescaled with them.
+//
+// Softmax arithmetic per score (the kernel is bound by the exponentials: one
+// per causal pair, 32 per clock per SM on the multi-function unit): a 3-input
+// max for the tile maximum, then per pair of scores one fp32x2 FMA
+// (x = s * scale * log2(e) - m), one conversion of the pair to bf16x2 and one
+// bf16x2 exp2, whose result is the packed bf16 P the PV product reads.
 //
 // Warp roles (192 threads): warp 0 issues TMA loads, warp 1 allocates TMEM and
-// issues the MMAs (one thread), warps 2-5 own one query row per thread
-// (TMEM lane = row) for the softmax and the epilogue.  q~ is computed by a
-// pre-pass into the first d_down entries of each output row and loaded with Q.  The softmax writes
-// P (bf16) into TMEM with tcgen05.st and the PV products take it from there
-// as their A operand, so P never touches shared memory.  Two S buffers (when
-// d_down <= 32) let S run two virtual tiles ahead of the softmax.  256 TMEM
-// columns and ~80 KB of shared memory per CTA let two CTAs share an SM, so
-// one CTA's softmax overlaps the other's MMA and load waits.  Every wait is
-// bounded; on a timeout the CTA flags *status and exits.
+// issues the MMAs (one thread), warps 2-5 own one query row per thread (TMEM
+// lane = row) for the softmax and the epilogue.  The softmax releases S as
+// soon as it has loaded it (so S(t + 1) is computed while it works on tile t)
+// and writes P into one of two TMEM buffers, where the PV products take it as
+// their A operand.  The MMA thread builds every shared-memory descriptor once
+// and only adds offsets per tile, so it issues a tile's products quickly.  Two CTAs share an SM (256 TMEM columns and ~110 KB of
+// shared memory each), so one CTA's softmax overlaps the other's waits.  Every
+// wait is bounded; on a timeout the CTA flags *status and exits.
 #include <cuda.h>
 
 #include "dar_common.cuh"
@@ -38,31 +48,38 @@ constexpr int BM = 128, BN = 64;
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 256;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p stays below 2^8 between rescales
+constexpr uint32_t kOnesBf16x2 = 0x3F803F80u;
 
 constexpr uint32_t align_up(uint32_t x, uint32_t a) { return (x + a - 1) / a * a; }
 
 // Tensor-memory columns of one CTA (256 of the SM's 512, two CTAs per SM):
-// S buffers (fp32, BN columns each; two when they fit, so S runs two virtual
-// tiles ahead of the softmax), O_loc (64), O_glob (DP) and P (bf16 pairs,
-// BN / 2 columns; the A operand of the PV products).
+// S (fp32, BN columns; the softmax releases it as soon as it has loaded it,
+// so one buffer keeps S(t + 1) computing while tile t's softmax runs), O_loc
+// (64), O_glob (DP), the row sum (16 identical columns) and P (bf16 pairs,
+// BN / 2 columns each; the A operand of the PV products), in two buffers when
+// they fit, so the softmax can write P(t + 1) while PV(t) still reads P(t).
+// q~ passes through the O_loc columns before the accumulators are cleared.
 template <int DP>
 struct Tmem {
-    static constexpr int NSB = DP <= 32 ? 2 : 1;
-    static constexpr uint32_t S = 0;  // buffer b at S + b * BN
-    static constexpr uint32_t OL = NSB * BN;
+    static constexpr uint32_t S = 0;
+    static constexpr uint32_t OL = BN;
     static constexpr uint32_t OG = OL + 64;
-    static constexpr uint32_t P = kTmemCols - BN / 2;
-    static_assert(OG + DP <= P, "tensor-memory columns overlap");
+    static constexpr uint32_t SUM = OG + DP;
+    static constexpr uint32_t P = SUM + 16;  // buffer b at P + b * BN / 2
+    static constexpr int NPB = P + BN <= kTmemCols ? 2 : 1;
+    static_assert(P + NPB * BN / 2 <= kTmemCols, "tensor-memory columns overflow");
 };
 
 // Shared-memory layout (offsets from a 1024-byte aligned base).  A stage holds
 // the operands of one virtual tile: K and V (local) or K^D and V^D (global).
 template <int DP>
 struct Layout {
-    static constexpr int NS = 3;                          // K/V stages
+    static constexpr int NS = DP == 16 ? 5 : DP == 32 ? 4 : 3;  // K/V stages (two CTAs per SM)
     static constexpr uint32_t Q = 0;                      // [128][64] bf16, 128B swizzle
-    static constexpr uint32_t QT = BM * 64 * 2;           // [128][DP] bf16 (q~, loaded by TMA)
-    static constexpr uint32_t STG = align_up(QT + BM * DP * 2, 1024);
+    static constexpr uint32_t QT = BM * 64 * 2;           // [128][DP] bf16 q~ (written by the softmax warps)
+    static constexpr uint32_t UKB = align_up(QT + BM * DP * 2, 1024);  // [DP][64] bf16 Uk, 128B swizzle
+    static constexpr uint32_t ONES = align_up(UKB + DP * 64 * 2, 1024);  // 1 KB of bf16 ones
+    static constexpr uint32_t STG = ONES + 1024;
     static constexpr uint32_t K_OFF = 0;                  // [64][64]
     static constexpr uint32_t V_OFF = BN * 64 * 2;        // [64][64]
     static constexpr uint32_t KD_OFF = 0;                 // [64][DP]
@@ -94,21 +111,6 @@ __device__ __forceinline__ TileKind tile_kind(int i0, int i_last, int j0, int w)
     return k;
 }
 
-template <int N>
-__device__ __forceinline__ float tree_max(const float (&v)[N])
-{
-    float t[N / 2];
-#pragma unroll
-    for (int e = 0; e < N / 2; ++e)
-        t[e] = fmaxf(v[2 * e], v[2 * e + 1]);
-#pragma unroll
-    for (int n = N / 4; n >= 1; n /= 2)
-#pragma unroll
-        for (int e = 0; e < n; ++e)
-            t[e] = fmaxf(t[e], t[e + n]);
-    return t[0];
-}
-
 __device__ __forceinline__ float max3(float a, float b, float c)
 {
     float d;
@@ -116,37 +118,23 @@ __device__ __forceinline__ float max3(float a, float b, float c)
     return d;
 }
 
-// Maximum of N values with the 3-input max.f32: four independent running
-// maxima, two new values per step each.
+// Maximum of N values (N = 64) with the 3-input max.f32, as a shallow tree:
+// 21 independent maxima of 3, then 7, then 3, then 1 (depth 4).
 template <int N>
 __device__ __forceinline__ float tree_max3(const float (&v)[N])
 {
-    float m[4] = {v[0], v[1], v[2], v[3]};
+    static_assert(N == 64, "tree shaped for 64 values");
+    float a[22];
 #pragma unroll
-    for (int e = 4; e + 8 <= N; e += 8)
+    for (int k = 0; k < 21; ++k)
+        a[k] = max3(v[3 * k], v[3 * k + 1], v[3 * k + 2]);
+    a[21] = v[63];
+    float b[8];
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-            m[k] = max3(m[k], v[e + 2 * k], v[e + 2 * k + 1]);
-    constexpr int R = 4 + (N - 4) / 8 * 8;
-#pragma unroll
-    for (int e = R; e < N; ++e)
-        m[e & 3] = fmaxf(m[e & 3], v[e]);
-    return max3(m[0], m[1], fmaxf(m[2], m[3]));
-}
-
-template <int N>
-__device__ __forceinline__ float tree_sum(const float (&v)[N])
-{
-    float t[N / 2];
-#pragma unroll
-    for (int e = 0; e < N / 2; ++e)
-        t[e] = v[2 * e] + v[2 * e + 1];
-#pragma unroll
-    for (int n = N / 4; n >= 1; n /= 2)
-#pragma unroll
-        for (int e = 0; e < n; ++e)
-            t[e] = t[e] + t[e + n];
-    return t[0];
+    for (int k = 0; k < 7; ++k)
+        b[k] = max3(a[3 * k], a[3 * k + 1], a[3 * k + 2]);
+    b[7] = a[21];
+    return max3(max3(b[0], b[1], b[2]), max3(b[3], b[4], b[5]), fmaxf(b[6], b[7]));
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
@@ -163,14 +151,6 @@ __device__ __forceinline__ void st_swz(unsigned char *base, int r, int c, uint4 
     constexpr int mask = RB / 16 - 1;
     const int phys = c ^ ((r * RB >> 7) & mask);
     *reinterpret_cast<uint4 *>(base + (size_t)r * RB + phys * 16) = v;
-}
-
-template <int RB>
-__device__ __forceinline__ uint4 ld_swz(const unsigned char *base, int r, int c)
-{
-    constexpr int mask = RB / 16 - 1;
-    const int phys = c ^ ((r * RB >> 7) & mask);
-    return *reinterpret_cast<const uint4 *>(base + (size_t)r * RB + phys * 16);
 }
 
 // Virtual tiles: a key tile whose pairs are all local or all global is one
@@ -211,26 +191,28 @@ __device__ __forceinline__ int vt_count(int i0, int i_last, int w)
 
 template <int DP>
 __global__ void __launch_bounds__(kThreads, 2)
-    prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQT,
-                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                      const __grid_constant__ CUtensorMap tmKD, const __grid_constant__ CUtensorMap tmVD,
-                      PrefillArgs a)
+    prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                      const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKD,
+                      const __grid_constant__ CUtensorMap tmVD, PrefillArgs a)
 {
     using Ly = Layout<DP>;
     using Tm = Tmem<DP>;
     constexpr int NS = Ly::NS;
-    constexpr int NSB = Tm::NSB;
+    constexpr int NPB = Tm::NPB;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + Ly::BAR);
     uint64_t *full = bars;                 // [NS] TMA -> MMA
     uint64_t *empty = bars + NS;           // [NS] MMA -> TMA
-    uint64_t *s_full = bars + 2 * NS;      // [NSB] S of a virtual tile computed
-    uint64_t *q_full = s_full + NSB;       // Q and q~ landed
-    uint64_t *qt_ready = q_full + 1;       // O zeroed (128 arrivals)
-    uint64_t *p_full = q_full + 2;         // P written to TMEM (128 arrivals)
-    uint64_t *pv_done = q_full + 3;        // PV of a virtual tile finished
+    uint64_t *s_full = bars + 2 * NS;      // S of a virtual tile computed
+    uint64_t *s_free = s_full + 1;         // S loaded by the softmax (4 warp arrivals)
+    uint64_t *p_full = s_free + 1;         // [NPB] P written to TMEM buffer b (4 warp arrivals)
+    uint64_t *pv_done = p_full + NPB;      // [NPB] PV (and row sums) reading P buffer b finished
+    uint64_t *q_full = pv_done + NPB;      // Q landed
+    uint64_t *ukb_ready = q_full + 1;      // Uk (bf16) and the ones block written (128 arrivals)
+    uint64_t *qt_mma = q_full + 2;         // q~ = Q Uk^T computed into TMEM
+    uint64_t *qt_ready = q_full + 3;       // q~ in shared memory, accumulators zeroed (128 arrivals)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_full + 4);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -247,12 +229,16 @@ __global__ void __launch_bounds__(kThreads, 2)
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
-        for (int b2 = 0; b2 < NSB; ++b2)
-            mbar_init(&s_full[b2], 1);
+        mbar_init(s_full, 1);
+        mbar_init(s_free, 4);
+        for (int b2 = 0; b2 < NPB; ++b2) {
+            mbar_init(&p_full[b2], 4);
+            mbar_init(&pv_done[b2], 1);
+        }
         mbar_init(q_full, 1);
+        mbar_init(ukb_ready, 128);
+        mbar_init(qt_mma, 1);
         mbar_init(qt_ready, 128);
-        mbar_init(p_full, 128);
-        mbar_init(pv_done, 1);
         *abort_flag = 0;
         mbar_init_fence();
     }
@@ -269,14 +255,12 @@ __global__ void __launch_bounds__(kThreads, 2)
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             prefetch_tensormap(&tmQ);
-            prefetch_tensormap(&tmQT);
             prefetch_tensormap(&tmK);
             prefetch_tensormap(&tmV);
             prefetch_tensormap(&tmKD);
             prefetch_tensormap(&tmVD);
-            mbar_expect_tx(q_full, BM * 64 * 2 + BM * DP * 2);
+            mbar_expect_tx(q_full, BM * 64 * 2);
             tma_load_2d(sm + Ly::Q, &tmQ, 0, (b * a.Hq + h) * N + i0, q_full);
-            tma_load_2d(sm + Ly::QT, &tmQT, 0, (b * a.Hq + h) * N + i0, q_full);
             VTile vt = vt_first(i0, i_last, w);
             for (int t = 0; t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
                 const int s = t % NS;
@@ -301,66 +285,94 @@ __global__ void __launch_bounds__(kThreads, 2)
             constexpr uint32_t idS = idesc_bf16(BM, BN, false);
             constexpr uint32_t idPV = idesc_bf16(BM, 64, true);
             constexpr uint32_t idPVg = idesc_bf16(BM, DP, true);
-            const uint32_t sQ = smem_u32(sm + Ly::Q), sQT = smem_u32(sm + Ly::QT);
-            bool ok = mbar_wait(qt_ready, 0, abort_flag);
-            tc_fence_after();
+            constexpr uint32_t idQT = idesc_bf16(BM, DP, false);
+            constexpr uint32_t idSum = idesc_bf16(BM, 16, false);
+            // Shared-memory descriptors, built once: a k-step of 16 elements adds
+            // 32 bytes along a K-major row (2 in the address field) and 16 rows
+            // (16 * row bytes) along an MN-major operand.
+            const uint64_t dQ = smem_desc(smem_u32(sm + Ly::Q), 16, 1024, kSw128);
+            const uint64_t dQT = smem_desc(smem_u32(sm + Ly::QT), 16, 8 * DP * 2, dp_swizzle<DP>());
+            const uint64_t dUKB = smem_desc(smem_u32(sm + Ly::UKB), 16, 1024, kSw128);
+            const uint64_t dStg = smem_desc(smem_u32(sm + Ly::STG), 16, 1024, kSw128);  // stage 0, K tile
+            const uint64_t dStgD = smem_desc(smem_u32(sm + Ly::STG), 16, 8 * DP * 2, dp_swizzle<DP>());
+            constexpr uint64_t kStageStep = Ly::STAGE >> 4;
+            constexpr uint64_t kVOff = Ly::V_OFF >> 4, kVDOff = Ly::VD_OFF >> 4;
+            constexpr uint64_t kVStep = (16 * 128) >> 4, kVDStep = (16 * DP * 2) >> 4;
+            // all-ones B operand (16 columns x 16 keys per k-step; every byte pair is 1.0)
+            const uint64_t ones_desc = smem_desc(smem_u32(sm + Ly::ONES), 128, 256, kSwNone);
+            const uint32_t tS = tmem + Tm::S, tOL = tmem + Tm::OL, tOG = tmem + Tm::OG;
+            const uint32_t tSum = tmem + Tm::SUM, tP = tmem + Tm::P;
+            // q~ = Q Uk^T into the O_loc columns
+            bool ok = mbar_wait(q_full, 0, abort_flag) && mbar_wait(ukb_ready, 0, abort_flag);
+            if (ok) {
+                tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    mma_f16_ss(tOL, dQ + 2 * kk, dUKB + 2 * kk, idQT, kk > 0);
+                mma_commit(qt_mma);
+                ok = mbar_wait(qt_ready, 0, abort_flag);
+                tc_fence_after();
+            }
             auto issue_S = [&](int t, VTile vt) -> bool {
-                const int s = t % NS, sb = t % NSB;
+                const int s = t % NS;
                 if (!mbar_wait(&full[s], (t / NS) & 1, abort_flag))
                     return false;
+                if (t >= 1 && !mbar_wait(s_free, (t - 1) & 1, abort_flag))
+                    return false;
                 tc_fence_after();
-                const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
-                const uint32_t dS = tmem + Tm::S + sb * BN;
-                if (vt.loc)
+                if (vt.loc) {
+                    const uint64_t dK = dStg + s * kStageStep;
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        mma_f16_ss(dS, smem_desc(sQ + kk * 32, 16, 1024, kSw128),
-                                   smem_desc(st + Ly::K_OFF + kk * 32, 16, 1024, kSw128), idS, kk > 0);
-                else
+                        mma_f16_ss(tS, dQ + 2 * kk, dK + 2 * kk, idS, kk > 0);
+                } else {
+                    const uint64_t dKD = dStgD + s * kStageStep;
 #pragma unroll
                     for (int kk = 0; kk < DP / 16; ++kk)
-                        mma_f16_ss(dS, smem_desc(sQT + kk * 32, 16, 8 * DP * 2, dp_swizzle<DP>()),
-                                   smem_desc(st + Ly::KD_OFF + kk * 32, 16, 8 * DP * 2, dp_swizzle<DP>()), idS,
-                                   kk > 0);
-                mma_commit(&s_full[sb]);
+                        mma_f16_ss(tS, dQT + 2 * kk, dKD + 2 * kk, idS, kk > 0);
+                }
+                mma_commit(s_full);
                 return true;
             };
             auto issue_PV = [&](int t, VTile vt) -> bool {
-                const int s = t % NS;
-                if (!mbar_wait(p_full, t & 1, abort_flag))
+                const int s = t % NS, pb = t % NPB;
+                if (!mbar_wait(&p_full[pb], (t / NPB) & 1, abort_flag))
                     return false;
                 tc_fence_after();
-                const uint32_t st = smem_u32(sm + Ly::STG + s * Ly::STAGE);
-                const uint32_t P = tmem + Tm::P;
+                const uint32_t aP = tP + pb * (BN / 2);
+                if (vt.loc) {
+                    const uint64_t dV = dStg + s * kStageStep + kVOff;
 #pragma unroll
-                for (int kk = 0; kk < BN / 16; ++kk) {  // P (TMEM, 8 columns per 16 keys) times V / V^D
-                    const uint32_t aP = P + kk * 8;
-                    if (vt.loc)
-                        mma_f16_ts(tmem + Tm::OL, aP, smem_desc(st + Ly::V_OFF + kk * 16 * 128, 16, 1024, kSw128),
-                                   idPV, true);
-                    else
-                        mma_f16_ts(tmem + Tm::OG, aP,
-                                   smem_desc(st + Ly::VD_OFF + kk * 16 * DP * 2, 16, 8 * DP * 2, dp_swizzle<DP>()),
-                                   idPVg, true);
+                    for (int kk = 0; kk < BN / 16; ++kk) {  // P (TMEM, 8 columns per 16 keys) times V
+                        mma_f16_ts(tOL, aP + kk * 8, dV + kk * kVStep, idPV, true);
+                        mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);  // row sums of P
+                    }
+                } else {
+                    const uint64_t dVD = dStgD + s * kStageStep + kVDOff;
+#pragma unroll
+                    for (int kk = 0; kk < BN / 16; ++kk) {  // P times V^D
+                        mma_f16_ts(tOG, aP + kk * 8, dVD + kk * kVDStep, idPVg, true);
+                        mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);
+                    }
                 }
-                mma_commit(pv_done);
+                mma_commit(&pv_done[pb]);
                 mma_commit(&empty[s]);
                 return true;
             };
-            // S runs NSB virtual tiles ahead: S(t + NSB) reuses the buffer of S(t),
-            // which P(t) being written proves the softmax has read
+            // S(t + 1) needs S(t) loaded by the softmax; PV(t) needs P(t)
             VTile vs = vt_first(i0, i_last, w), vp = vs;
-            for (int t = 0; ok && t < NSB && t < VT; ++t) {
-                ok = issue_S(t, vs);
+            if (ok && VT > 0) {
+                ok = issue_S(0, vs);
                 vs = vt_next(vs, i0, i_last, w);
             }
             for (int t = 0; ok && t < VT; ++t) {
-                ok = issue_PV(t, vp);
-                vp = vt_next(vp, i0, i_last, w);
-                if (ok && t + NSB < VT) {
-                    ok = issue_S(t + NSB, vs);
+                if (t + 1 < VT) {
+                    ok = issue_S(t + 1, vs);
                     vs = vt_next(vs, i0, i_last, w);
                 }
+                if (ok)
+                    ok = issue_PV(t, vp);
+                vp = vt_next(vp, i0, i_last, w);
             }
         }
     } else {
@@ -370,19 +382,53 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int i = i0 + row;
         const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
         const int stid = threadIdx.x - 64;  // 0..127
-        float *sUv = reinterpret_cast<float *>(sm + Ly::UV);
-        for (int idx = stid; idx < DP * 64; idx += 128) {
-            const int c = idx / 64, t = idx % 64;
-            sUv[idx] = c < a.dd ? a.Uv[((size_t)g * a.dd + c) * 64 + t] : 0.f;
+        // ---- set-up: Uk as a bf16 operand, the ones block, Uv for the epilogue
+        {
+            const float *Ukg = a.Uk + (size_t)g * a.dd * 64;
+            for (int idx = stid; idx < DP * 8; idx += 128) {  // row c, chunk ch of 8 values
+                const int c = idx / 8, ch = idx % 8;
+                uint4 v = make_uint4(0u, 0u, 0u, 0u);
+                if (c < a.dd) {
+                    const float4 u0 = *reinterpret_cast<const float4 *>(Ukg + c * 64 + ch * 8);
+                    const float4 u1 = *reinterpret_cast<const float4 *>(Ukg + c * 64 + ch * 8 + 4);
+                    v = make_uint4(pack_bf16(u0.x, u0.y), pack_bf16(u0.z, u0.w), pack_bf16(u1.x, u1.y),
+                                   pack_bf16(u1.z, u1.w));
+                }
+                st_swz<128>(sm + Ly::UKB, c, ch, v);
+            }
+            if (stid < 64)
+                reinterpret_cast<uint4 *>(sm + Ly::ONES)[stid] =
+                    make_uint4(kOnesBf16x2, kOnesBf16x2, kOnesBf16x2, kOnesBf16x2);
+            fence_proxy_async_smem();
+            mbar_arrive(ukb_ready);
+            float *sUv = reinterpret_cast<float *>(sm + Ly::UV);
+            for (int idx = stid; idx < DP * 64; idx += 128) {
+                const int c = idx / 64, t = idx % 64;
+                sUv[idx] = c < a.dd ? a.Uv[((size_t)g * a.dd + c) * 64 + t] : 0.f;
+            }
         }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
         // tcgen05.ld/st are warp-collective: every branch around them is warp-uniform
         auto wait_uniform = [&](uint64_t *bar, unsigned parity) {
             const bool r = mbar_wait(bar, parity, abort_flag);
             return __all_sync(0xffffffffu, r) != 0;
         };
-        bool ok = wait_uniform(q_full, 0);
-        {  // zero the accumulators
+        bool ok = wait_uniform(qt_mma, 0);
+        if (ok) {
+            // q~ (fp32, TMEM) -> bf16 operand rows in shared memory; then clear the accumulators
+            tc_fence_after();
+            uint32_t r[16];
+            unsigned char *qrow = sm + Ly::QT;
+#pragma unroll
+            for (int c = 0; c < DP; c += 16) {
+                tmem_ld16(tl + Tm::OL + c, r);
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    st_swz<DP * 2>(qrow, row, c / 8 + k,
+                                   make_uint4(pack_bf16(__uint_as_float(r[8 * k + 0]), __uint_as_float(r[8 * k + 1])),
+                                              pack_bf16(__uint_as_float(r[8 * k + 2]), __uint_as_float(r[8 * k + 3])),
+                                              pack_bf16(__uint_as_float(r[8 * k + 4]), __uint_as_float(r[8 * k + 5])),
+                                              pack_bf16(__uint_as_float(r[8 * k + 6]), __uint_as_float(r[8 * k + 7]))));
+            }
             uint32_t z[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e)
@@ -391,59 +437,78 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int c = 0; c < 64; c += 16)
                 tmem_st16(tl + Tm::OL + c, z);
 #pragma unroll
-            for (int c = 0; c < DP; c += 16)
+            for (int c = 0; c < DP + 16; c += 16)  // O_glob and the row-sum columns
                 tmem_st16(tl + Tm::OG + c, z);
             tmem_wait_st();
+            fence_proxy_async_smem();
         }
+        asm volatile("bar.sync 1, 128;" ::: "memory");  // Uv staged by all softmax threads
         tc_fence_before();
         mbar_arrive(qt_ready);
 
         const float c2 = a.qscale;  // softmax scale * log2(e)
-        float m_used = -INFINITY, l = 0.f;
-        int pv_waited = -1;  // highest virtual tile whose PV completion has been observed
+        float m_used = -INFINITY;
+        // highest PV(t') observed complete, per P buffer (t' even / odd)
+        int pv_seen0 = -NPB, pv_seen1 = 1 - NPB;
+        // wait until PV(u) (and so every tensor-core op issued before it) has completed
+        auto wait_pv = [&](int u) -> bool {
+            const bool odd = NPB == 2 && (u & 1);
+            if (u < 0 || (odd ? pv_seen1 : pv_seen0) >= u)
+                return true;
+            if (!wait_uniform(&pv_done[odd ? 1 : 0], (u / NPB) & 1))
+                return false;
+            if (odd)
+                pv_seen1 = u;
+            else
+                pv_seen0 = u;
+            tc_fence_after();
+            return true;
+        };
         VTile vt = vt_first(i0, i_last, w);
         for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
             const int j0 = vt.kt * BN;
-            const int sb = t % NSB;
-            if (!wait_uniform(&s_full[sb], (t / NSB) & 1)) {
+            if (!wait_uniform(s_full, t & 1)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
             float s[BN];
             {
-                uint32_t r[BN];  // both halves in flight, one wait
-                tmem_ld32_nowait(tl + Tm::S + sb * BN, *reinterpret_cast<uint32_t(*)[32]>(&r[0]));
-                tmem_ld32_nowait(tl + Tm::S + sb * BN + 32, *reinterpret_cast<uint32_t(*)[32]>(&r[32]));
-                tmem_wait_ld_regs(r);
+                uint32_t r[BN];
+                tmem_ld64(tl + Tm::S, r);
 #pragma unroll
                 for (int e = 0; e < BN; ++e)
                     s[e] = __uint_as_float(r[e]);
             }
+            // the S columns may be overwritten now (S(t + 1))
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(s_free);
             // masks: causal (tiles reaching past row i0), the other part of a
-            // band tile, rows past the end
-            if (j0 + BN - 1 > i0 || vt.band || i >= N) {
-#pragma unroll
-                for (int e = 0; e < BN; ++e) {
-                    const int j = j0 + e;
-                    const bool keep = j <= i && i < N && (!vt.band || ((i - j < w) == vt.loc));
-                    s[e] = keep ? s[e] : -INFINITY;
+            // band tile, rows past the end; the kept columns form one range
+            if (j0 + BN - 1 > i0 || vt.band || i0 + BM > N) {
+                int e_hi = i < N ? i - j0 : -1, e_lo = 0;
+                if (vt.band) {
+                    if (vt.loc)
+                        e_lo = i - w - j0 + 1;
+                    else
+                        e_hi = min(e_hi, i - w - j0);
                 }
+#pragma unroll
+                for (int e = 0; e < BN; ++e)
+                    s[e] = (e >= e_lo && e <= e_hi) ? s[e] : -INFINITY;
             }
             const float mt = tree_max3(s) * c2;
             // raise the running max only when it grows by more than the threshold
             const bool raise = mt > m_used + kRescaleThreshold;
             const bool scale_o = raise && m_used != -INFINITY;
-            const float alpha = scale_o ? ex2_approx(m_used - mt) : 1.f;
             if (__any_sync(0xffffffffu, scale_o)) {
+                const float alpha = scale_o ? ex2_approx(m_used - mt) : 1.f;
                 // every earlier PV must have landed before O is rescaled
-                if (pv_waited < t - 1) {
-                    if (!wait_uniform(pv_done, (t - 1) & 1)) {
-                        ok = false;
-                        break;
-                    }
-                    pv_waited = t - 1;
-                    tc_fence_after();
+                if (!wait_pv(t - 1)) {
+                    ok = false;
+                    break;
                 }
 #pragma unroll
                 for (int c = 0; c < 64; c += 16) {
@@ -455,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tmem_st16(tl + Tm::OL + c, r);
                 }
 #pragma unroll
-                for (int c = 0; c < DP; c += 16) {
+                for (int c = 0; c < DP + 16; c += 16) {  // O_glob and the row sums
                     uint32_t r[16];
                     tmem_ld16(tl + Tm::OG + c, r);
 #pragma unroll
@@ -464,49 +529,47 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tmem_st16(tl + Tm::OG + c, r);
                 }
             }
-            l *= alpha;
             if (raise)
                 m_used = mt;
-            // P = 2^(s * c2 - m) (masked entries give 0); the PV of the previous
-            // virtual tile must be done reading the P columns
+            // P = 2^(s * c2 - m) in bf16 pairs (masked entries give 0)
             const float mneg = m_used == -INFINITY ? 0.f : -m_used;
             uint32_t pk[BN / 2];
-            float ls = 0.f;
 #pragma unroll
             for (int e = 0; e < BN; e += 2) {
-                const float p0 = ex2_approx(fmaf(s[e], c2, mneg));
-                const float p1 = ex2_approx(fmaf(s[e + 1], c2, mneg));
-                ls += p0 + p1;
-                pk[e / 2] = pack_bf16(p0, p1);
+                float x0, x1;
+                ffma2(x0, x1, s[e], s[e + 1], c2, c2, mneg, mneg);
+                pk[e / 2] = ex2_bf16x2(cvt_bf16x2(x0, x1));
             }
-            l += ls;
-            if (t > 0 && pv_waited < t - 1) {
-                if (!wait_uniform(pv_done, (t - 1) & 1)) {
-                    ok = false;
-                    break;
-                }
-                pv_waited = t - 1;
-                tc_fence_after();
+            // the PV that last read this P buffer (tile t - NPB) must be done with it
+            if (!wait_pv(t - NPB)) {
+                ok = false;
+                break;
             }
-            tmem_st16(tl + Tm::P, *reinterpret_cast<const uint32_t(*)[16]>(&pk[0]));
-            tmem_st16(tl + Tm::P + 16, *reinterpret_cast<const uint32_t(*)[16]>(&pk[16]));
+            const int pb = t % NPB;
+            tmem_st32(tl + Tm::P + pb * (BN / 2), pk);
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(p_full);
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&p_full[pb]);
         }
 
         // ---- epilogue: o = (O_loc + O_glob Uv) / l
-        // every PV before the last has been waited for (before writing P)
-        if (ok && wait_uniform(pv_done, (VT - 1) & 1)) {
-            tc_fence_after();
+        if (ok && wait_pv(VT - 1)) {
+            const float *sUv = reinterpret_cast<const float *>(sm + Ly::UV);
             float og[DP];
-#pragma unroll
-            for (int c = 0; c < DP; c += 16) {
+            float l;
+            {
                 uint32_t r[16];
-                tmem_ld16(tl + Tm::OG + c, r);
 #pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    og[c + e] = __uint_as_float(r[e]);
+                for (int c = 0; c < DP; c += 16) {
+                    tmem_ld16(tl + Tm::OG + c, r);
+#pragma unroll
+                    for (int e = 0; e < 16; ++e)
+                        og[c + e] = __uint_as_float(r[e]);
+                }
+                tmem_ld16(tl + Tm::SUM, r);
+                l = __uint_as_float(r[0]);
             }
             const float inv = l > 0.f ? 1.f / l : 0.f;
             bf16 *orow = static_cast<bf16 *>(a.out) + (((size_t)b * a.Hq + h) * N + i) * 64;
@@ -567,14 +630,15 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
 static EncodeTiledFn encode_fn()
 {
     static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    static std::once_flag once;
+    std::call_once(once, [] {
         void *p = nullptr;
         cudaDriverEntryPointQueryResult q;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
                 cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
             fn = reinterpret_cast<EncodeTiledFn>(p);
-    }
+    });
     return fn;
 }
 
@@ -598,14 +662,12 @@ static bool make_map(CUtensorMap *m, const void *base, unsigned long long rows, 
 template <int DP>
 static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
 {
-    CUtensorMap mq, mqt, mk, mv, mkd, mvd;
+    CUtensorMap mq, mk, mv, mkd, mvd;
     const CUtensorMapSwizzle swd = DP == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
                                    : DP == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
                                               : CU_TENSOR_MAP_SWIZZLE_128B;
     const unsigned long long rq = (unsigned long long)a.B * a.Hq * a.N, rk = (unsigned long long)a.B * a.Hkv * a.N;
-    // q~ sits in the first DP entries of each output row (written by the pre-pass)
     if (!make_map(&mq, a.q, rq, 64, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&mqt, a.out, rq, DP, BM, swd, 64) ||
         !make_map(&mk, a.k, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&mv, a.v, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) || !make_map(&mkd, a.kd, rk, DP, BN, swd) ||
         !make_map(&mvd, a.vd, rk, DP, BN, swd))
@@ -614,77 +676,17 @@ static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
     const size_t smem = Layout<DP>::TOTAL + 1024;
     static PerDeviceOnce once;
     cudaError_t e = per_device_once(once, [&](int) {
-        return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        // two CTAs per SM need the largest shared-memory carve-out of the unified L1
+        cudaError_t e2 = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e2 == cudaSuccess)
+            e2 = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                      (int)cudaSharedmemCarveoutMaxShared);
+        return e2;
     });
     if (e != cudaSuccess)
         return e;
     dim3 grid(a.B * a.Hq, (a.N + BM - 1) / BM);
-    kern<<<grid, kThreads, smem, s>>>(mq, mqt, mk, mv, mkd, mvd, a);
-    return cudaGetLastError();
-}
-
-// ---------------------------------------------------------------- q~ pre-pass
-
-// q~ = q Uk^T for every query row (fp32 chains, rounded once to bf16), written
-// into the first DP entries of the row's output slot (entries dd..DP-1 zero):
-// the CTA that owns a row reads its q~ before it writes the row's output.
-// grid (ceil(N / 128), B * Hq), 128 threads, one row per thread.
-template <int DP>
-__global__ void __launch_bounds__(128) qtilde_kernel(const bf16 *__restrict__ q, const float *__restrict__ Uk,
-                                                     bf16 *__restrict__ out, int Hq, int G, int dd, int N)
-{
-    __shared__ __align__(16) float sUk[DP * 64];
-    const int bh = blockIdx.y, g = (bh % Hq) / G;
-    for (int i = threadIdx.x; i < DP * 64; i += blockDim.x)
-        sUk[i] = i / 64 < dd ? Uk[((size_t)g * dd + i / 64) * 64 + i % 64] : 0.f;
-    __syncthreads();
-    const int j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= N)
-        return;
-    const size_t row = (size_t)bh * N + j;
-    float x[64];
-    const uint4 *q4 = reinterpret_cast<const uint4 *>(q + row * 64);
-#pragma unroll
-    for (int c = 0; c < 8; ++c) {
-        const uint4 v = q4[c];
-        x[8 * c + 0] = bf16lo(v.x);
-        x[8 * c + 1] = bf16hi(v.x);
-        x[8 * c + 2] = bf16lo(v.y);
-        x[8 * c + 3] = bf16hi(v.y);
-        x[8 * c + 4] = bf16lo(v.z);
-        x[8 * c + 5] = bf16hi(v.z);
-        x[8 * c + 6] = bf16lo(v.w);
-        x[8 * c + 7] = bf16hi(v.w);
-    }
-    uint4 *o4 = reinterpret_cast<uint4 *>(out + row * 64);
-#pragma unroll 1
-    for (int c8 = 0; c8 < DP / 8; ++c8) {
-        float o[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const float4 *u4 = reinterpret_cast<const float4 *>(sUk + (c8 * 8 + e) * 64);
-            float a0 = 0.f, a1 = 0.f;
-#pragma unroll
-            for (int t4 = 0; t4 < 16; ++t4) {
-                const float4 u = u4[t4];
-                a0 = fmaf(x[4 * t4 + 0], u.x, a0);
-                a1 = fmaf(x[4 * t4 + 1], u.y, a1);
-                a0 = fmaf(x[4 * t4 + 2], u.z, a0);
-                a1 = fmaf(x[4 * t4 + 3], u.w, a1);
-            }
-            o[e] = a0 + a1;
-        }
-        o4[c8] = make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]),
-                            pack_bf16(o[6], o[7]));
-    }
-}
-
-template <int DP>
-static cudaError_t launch_qtilde(const PrefillArgs &a, cudaStream_t s)
-{
-    dim3 grid((a.N + 127) / 128, a.B * a.Hq);
-    qtilde_kernel<DP><<<grid, 128, 0, s>>>(static_cast<const bf16 *>(a.q), a.Uk, static_cast<bf16 *>(a.out), a.Hq,
-                                           a.Hq / a.Hkv, a.dd, a.N);
+    kern<<<grid, kThreads, smem, s>>>(mq, mk, mv, mkd, mvd, a);
     return cudaGetLastError();
 }
 
@@ -703,11 +705,10 @@ cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s)
 {
     if (a.B == 0 || a.N == 0)
         return cudaSuccess;
-    cudaError_t e;
     switch (a.kd_stride) {
-    case 16: e = tcp::launch_qtilde<16>(a, s); return e != cudaSuccess ? e : tcp::launch_dp<16>(a, s);
-    case 32: e = tcp::launch_qtilde<32>(a, s); return e != cudaSuccess ? e : tcp::launch_dp<32>(a, s);
-    case 64: e = tcp::launch_qtilde<64>(a, s); return e != cudaSuccess ? e : tcp::launch_dp<64>(a, s);
+    case 16: return tcp::launch_dp<16>(a, s);
+    case 32: return tcp::launch_dp<32>(a, s);
+    case 64: return tcp::launch_dp<64>(a, s);
     default: return cudaErrorInvalidValue;
     }
 }
