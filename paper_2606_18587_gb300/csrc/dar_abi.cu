@@ -304,8 +304,9 @@ size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int3
 {
     if (!dtype_valid(dtype) || B < 0 || Hkv < 0 || N < 0 || d_down < 1)
         return 0;
-    const int stride = dar::prefill_kd_stride(dtype, d_down);
-    return 2 * align256((size_t)B * Hkv * N * stride * esize(dtype));
+    const size_t rows = (size_t)B * Hkv * N;
+    return align256(rows * dar::prefill_kd_stride(dtype, d_down) * esize(dtype)) +
+           align256(rows * dar::prefill_vd_stride(dtype, d_down) * esize(dtype));
 }
 
 dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
@@ -333,10 +334,12 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
     if (workspace_bytes < need)
         return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, need);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    char *kd = static_cast<char *>(workspace);
-    char *vd = kd + need / 2;
     const int kstride = dar::prefill_kd_stride(dtype, d_down);
-    cudaError_t e = dar::launch_down_project_kv(dtype, d_down, k, v, Dk, Dv, kd, vd, B, Hkv, N, kstride, st);
+    const int vstride = dar::prefill_vd_stride(dtype, d_down);
+    char *kd = static_cast<char *>(workspace);
+    char *vd = kd + align256((size_t)B * Hkv * N * kstride * esize(dtype));
+    cudaError_t e = dar::launch_down_project_kv(dtype, d_down, k, v, Dk, Dv, kd, vd, B, Hkv, N, kstride, vstride,
+                                                dar::prefill_vd_ones_col(dtype, d_down), st);
     if (e != cudaSuccess)
         return from_cuda(e, "dar_attn_prefill down-projection launch");
     dar::PrefillArgs a;
@@ -356,6 +359,7 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
     a.w = w;
     a.dd = d_down;
     a.kd_stride = kstride;
+    a.vd_stride = vstride;
     a.qscale = default_scale(scale, d) * kLog2e;
     if (dtype == DAR_BF16)
         return from_cuda(dar::launch_prefill_tc(d_down, a, st), "dar_attn_prefill (tcgen05) launch");

@@ -42,7 +42,9 @@ struct BulkArgs {
     const void *x[2];
     const float *W[2];
     void *out[2];
-    int Hkv, n, ostride;
+    int Hkv, n;
+    int ostride[2];   // output row stride of each tensor (columns dd.. are padding)
+    int ones_col[2];  // first of 16 padding columns set to 1 (-1: all padding is 0)
 };
 
 template <typename T, int DD>
@@ -100,13 +102,15 @@ __global__ void __launch_bounds__(threads_bulk<T, DD>()) down_project_kernel(Bul
             }
         }
     }
+    const int ostride = z ? a.ostride[1] : a.ostride[0];
+    const int ones_col = z ? a.ones_col[1] : a.ones_col[0];
 #pragma unroll
     for (int k = 0; k < RPT; ++k) {
         const int r = threadIdx.x + k * NT;
         if (r >= nr)
             continue;
-        T *o = static_cast<T *>(z ? a.out[1] : a.out[0]) + ((size_t)bg * a.n + j0 + r) * a.ostride;
-        if (a.ostride == DD && (DD * sizeof(T)) % 16 == 0) {
+        T *o = static_cast<T *>(z ? a.out[1] : a.out[0]) + ((size_t)bg * a.n + j0 + r) * ostride;
+        if (ostride == DD && (DD * sizeof(T)) % 16 == 0) {
             constexpr int OE = 16 / sizeof(T);
 #pragma unroll
             for (int c = 0; c < DD; c += OE) {
@@ -124,12 +128,40 @@ __global__ void __launch_bounds__(threads_bulk<T, DD>()) down_project_kernel(Bul
                 }
                 *reinterpret_cast<uint4 *>(o + c) = make_uint4(u[0], u[1], u[2], u[3]);
             }
+        } else if ((ostride * sizeof(T)) % 16 == 0 && ostride <= kHeadDim) {
+            // padded rows (values, then zeros or a block of 16 ones), 16 bytes at a time
+            constexpr int OE = 16 / sizeof(T);
+#pragma unroll
+            for (int c0 = 0; c0 < kHeadDim; c0 += OE) {
+                if (c0 >= ostride)
+                    break;
+                float v[OE];
+#pragma unroll
+                for (int e = 0; e < OE; ++e) {
+                    const int c = c0 + e;
+                    v[e] = c < DD ? acc[k][c < DD ? c : 0]
+                                  : (ones_col >= 0 && c >= ones_col && c < ones_col + 16 ? 1.f : 0.f);
+                }
+                uint32_t u[4];
+                if constexpr (sizeof(T) == 2) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        __nv_bfloat162 b2 = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+                        u[i] = *reinterpret_cast<uint32_t *>(&b2);
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        u[i] = __float_as_uint(v[i]);
+                }
+                *reinterpret_cast<uint4 *>(o + c0) = make_uint4(u[0], u[1], u[2], u[3]);
+            }
         } else {
 #pragma unroll
             for (int c = 0; c < DD; ++c)
                 o[c] = from_f32<T>(acc[k][c]);
-            for (int c = DD; c < a.ostride; ++c)
-                o[c] = from_f32<T>(0.f);
+            for (int c = DD; c < ostride; ++c)
+                o[c] = from_f32<T>(c >= ones_col && c < ones_col + 16 && ones_col >= 0 ? 1.f : 0.f);
         }
     }
 }
@@ -324,15 +356,15 @@ static cudaError_t down_project_any(dar_dtype dt, int dd, const BulkArgs &a, int
 cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float *W, void *out,
                                 int B, int Hkv, int n, int ostride, cudaStream_t s)
 {
-    BulkArgs a = {{x, x}, {W, W}, {out, out}, Hkv, n, ostride};
+    BulkArgs a = {{x, x}, {W, W}, {out, out}, Hkv, n, {ostride, ostride}, {-1, -1}};
     return down_project_any(dt, dd, a, B, 1, s);
 }
 
 cudaError_t launch_down_project_kv(dar_dtype dt, int dd, const void *k, const void *v, const float *Dk,
-                                   const float *Dv, void *kd, void *vd, int B, int Hkv, int n, int ostride,
-                                   cudaStream_t s)
+                                   const float *Dv, void *kd, void *vd, int B, int Hkv, int n, int kstride,
+                                   int vstride, int v_ones_col, cudaStream_t s)
 {
-    BulkArgs a = {{k, v}, {Dk, Dv}, {kd, vd}, Hkv, n, ostride};
+    BulkArgs a = {{k, v}, {Dk, Dv}, {kd, vd}, Hkv, n, {kstride, vstride}, {-1, v_ones_col}};
     return down_project_any(dt, dd, a, B, 2, s);
 }
 

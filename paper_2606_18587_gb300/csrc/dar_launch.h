@@ -46,26 +46,45 @@ struct DecodeArgs {
 
 struct PrefillArgs {
     const void *q, *k, *v;  // [B][Hq|Hkv][N][64]
-    const void *kd, *vd;    // [B][Hkv][N][kd_stride]   (Eq. 1 output, zero padded)
+    const void *kd, *vd;    // [B][Hkv][N][kd_stride], [B][Hkv][N][vd_stride] (Eq. 1 output, padded)
     const float *Uk, *Uv;   // [Hkv][dd][64]
     void *out;              // [B][Hq][N][64]
     int32_t *status;        // device error word or nullptr
-    int B, Hq, Hkv, N, w, dd, kd_stride;
+    int B, Hq, Hkv, N, w, dd, kd_stride, vd_stride;
     float qscale;  // scale * log2(e)
 };
 
 // Row stride (elements) of the prefill bottleneck workspace: the tensor-core
 // path needs rows of at least 16 bf16 (one MMA K step).
 inline int prefill_kd_stride(dar_dtype dt, int dd) { return (dt == DAR_BF16 && dd < 16) ? 16 : dd; }
+// Row stride of the prefill's v^D workspace.  The tensor-core path appends 16
+// columns of ones after the kd_stride values (zero padding after them), so one
+// PV product also sums P into the softmax denominator: 32 for d_down <= 16, 64
+// for d_down = 32; d_down = 64 keeps plain rows (its sums take a product of
+// their own).
+inline int prefill_vd_stride(dar_dtype dt, int dd)
+{
+    if (dt != DAR_BF16)
+        return dd;
+    const int ks = prefill_kd_stride(dt, dd);
+    return ks == 16 ? 32 : ks == 32 ? 64 : ks;
+}
+// First column of the ones block in a v^D row (-1: none).
+inline int prefill_vd_ones_col(dar_dtype dt, int dd)
+{
+    const int ks = prefill_kd_stride(dt, dd);
+    return prefill_vd_stride(dt, dd) > ks ? ks : -1;
+}
 
 // Each launcher returns cudaSuccess or the launch error.
 // Eq. 1 into rows of `ostride` elements (entries dd..ostride-1 are zeroed).
 cudaError_t launch_down_project(dar_dtype dt, int dd, const void *x, const float *W, void *out,
                                 int B, int Hkv, int n, int ostride, cudaStream_t s);
-// The same for keys and values in one launch: kd = k Dk, vd = v Dv.
+// The same for keys and values in one launch: kd = k Dk (rows of kstride),
+// vd = v Dv (rows of vstride, with 16 ones from column v_ones_col if >= 0).
 cudaError_t launch_down_project_kv(dar_dtype dt, int dd, const void *k, const void *v, const float *Dk,
-                                   const float *Dv, void *kd, void *vd, int B, int Hkv, int n, int ostride,
-                                   cudaStream_t s);
+                                   const float *Dv, void *kd, void *vd, int B, int Hkv, int n, int kstride,
+                                   int vstride, int v_ones_col, cudaStream_t s);
 cudaError_t launch_cache_append(dar_dtype dt, int dd, const AppendArgs &a, cudaStream_t s);
 cudaError_t launch_decode(dar_dtype dt, int dd, const DecodeArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_simt(dar_dtype dt, int dd, const PrefillArgs &a, cudaStream_t s);

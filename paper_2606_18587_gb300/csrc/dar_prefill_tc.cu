@@ -16,7 +16,9 @@
 //   o = (O_loc + O_glob Uv) / l.
 // The softmax denominator l is summed by the tensor core as well: each P also
 // multiplies a block of ones into 16 extra accumulator columns, so l adds up
-// exactly the bf16 weights the numerators use and is rescaled with them.
+// exactly the bf16 weights the numerators use and is rescaled with them.  For
+// the global part the ones ride in the v^D rows of the workspace (16 columns
+// after the d_down values), so one product of N = d_down + 16 gives both.
 //
 // Softmax arithmetic per score (the kernel is bound by the exponentials: one
 // per causal pair, 32 per clock per SM on the multi-function unit): a 3-input
@@ -24,13 +26,14 @@
 // (x = s * scale * log2(e) - m), one conversion of the pair to bf16x2 and one
 // bf16x2 exp2, whose result is the packed bf16 P the PV product reads.
 //
-// Warp roles (192 threads): warp 0 issues TMA loads, warp 1 allocates TMEM and
-// issues the MMAs (one thread), warps 2-5 own one query row per thread (TMEM
-// lane = row) for the softmax and the epilogue.  The softmax releases S as
-// soon as it has loaded it (so S(t + 1) is computed while it works on tile t)
-// and writes P into one of two TMEM buffers, where the PV products take it as
-// their A operand.  The MMA thread builds every shared-memory descriptor once
-// and only adds offsets per tile, so it issues a tile's products quickly.  Two CTAs share an SM (256 TMEM columns and ~110 KB of
+// Warp roles (224 threads): warp 0 issues TMA loads, warp 6 issues the S
+// products (and q~), warp 1 allocates TMEM and issues the PV products (one
+// thread each), warps 2-5 own one query row per thread (TMEM lane = row) for
+// the softmax and the epilogue.  The softmax releases an S buffer as soon as
+// it has loaded it (so S(t + NSB) is computed while it works on tile t) and
+// writes P into TMEM, where the PV products take it as their A operand.  The
+// issuing threads build their shared-memory descriptors once and only add
+// offsets per tile.  Two CTAs share an SM (256 TMEM columns and ~110 KB of
 // shared memory each), so one CTA's softmax overlaps the other's waits.  Every
 // wait is bounded; on a timeout the CTA flags *status and exits.
 #include <cuda.h>
@@ -45,24 +48,53 @@ namespace tcp {
 using namespace sm100;
 
 constexpr int BM = 128, BN = 64;
-constexpr int kThreads = 192;
+constexpr int kSoftmaxWarps = 4, kSoftmaxThreads = 32 * kSoftmaxWarps;  // one thread per query row
+constexpr int kThreads = 32 * (3 + kSoftmaxWarps);
+constexpr int kWarpPV = 1, kWarpS = 2 + kSoftmaxWarps;  // MMA issuers (warp 0: TMA, warps 2-5: softmax)
 constexpr uint32_t kTmemCols = 256;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p stays below 2^8 between rescales
 constexpr uint32_t kOnesBf16x2 = 0x3F803F80u;
 
 constexpr uint32_t align_up(uint32_t x, uint32_t a) { return (x + a - 1) / a * a; }
 
+template <int DP>
+__host__ __device__ constexpr Swizzle dp_swizzle()
+{
+    return DP == 16 ? kSw32 : DP == 32 ? kSw64 : kSw128;
+}
+
+// Elements per v^D row in the workspace: the DP values, then (DP < 64) 16
+// ones and zero padding to a swizzle width, so the global PV product with
+// N = DP + 16 also sums P into the row-sum columns that follow O_glob.
+template <int DP>
+__host__ __device__ constexpr int vd_row()
+{
+    return DP == 16 ? 32 : 64;
+}
+template <int DP>
+__host__ __device__ constexpr bool vd_has_ones()
+{
+    return vd_row<DP>() > DP;
+}
+template <int DP>
+__host__ __device__ constexpr Swizzle vd_swizzle()
+{
+    return vd_row<DP>() == 32 ? kSw64 : kSw128;
+}
+
 // Tensor-memory columns of one CTA (256 of the SM's 512, two CTAs per SM):
 // S (fp32, BN columns; the softmax releases it as soon as it has loaded it,
-// so one buffer keeps S(t + 1) computing while tile t's softmax runs), O_loc
-// (64), O_glob (DP), the row sum (16 identical columns) and P (bf16 pairs,
-// BN / 2 columns each; the A operand of the PV products), in two buffers when
-// they fit, so the softmax can write P(t + 1) while PV(t) still reads P(t).
-// q~ passes through the O_loc columns before the accumulators are cleared.
+// and the S issuer, a thread of its own, computes S(t + 1) into it while tile
+// t's softmax runs), O_loc (64), O_glob (DP), the row sum (16 identical
+// columns) and P (bf16 pairs, BN / 2 columns; the A operand of the PV
+// products), in two buffers when they fit, so the softmax writes P(t + 1)
+// while PV(t) still reads P(t).  q~ passes through the O_loc columns before
+// the accumulators are cleared.
 template <int DP>
 struct Tmem {
-    static constexpr uint32_t S = 0;
-    static constexpr uint32_t OL = BN;
+    static constexpr int NSB = 1;
+    static constexpr uint32_t S = 0;  // buffer b at S + b * BN
+    static constexpr uint32_t OL = NSB * BN;
     static constexpr uint32_t OG = OL + 64;
     static constexpr uint32_t SUM = OG + DP;
     static constexpr uint32_t P = SUM + 16;  // buffer b at P + b * BN / 2
@@ -83,20 +115,14 @@ struct Layout {
     static constexpr uint32_t K_OFF = 0;                  // [64][64]
     static constexpr uint32_t V_OFF = BN * 64 * 2;        // [64][64]
     static constexpr uint32_t KD_OFF = 0;                 // [64][DP]
-    static constexpr uint32_t VD_OFF = align_up(BN * DP * 2, 1024);
+    static constexpr uint32_t VD_OFF = align_up(BN * DP * 2, 1024);  // [64][vd_row] (values, ones)
     static constexpr uint32_t STAGE = align_up(2 * BN * 64 * 2, 1024);
     static constexpr uint32_t UV = STG + NS * STAGE;      // fp32 [DP][64]
     static constexpr uint32_t BAR = UV + DP * 64 * 4;
     static constexpr uint32_t TOTAL = BAR + 256;
     static_assert(STAGE % 1024 == 0 && STG % 1024 == 0, "operand tiles must stay 1024-byte aligned");
-    static_assert(VD_OFF + BN * DP * 2 <= STAGE, "a stage holds either part");
+    static_assert(VD_OFF + BN * vd_row<DP>() * 2 <= STAGE, "a stage holds either part");
 };
-
-template <int DP>
-__host__ __device__ constexpr Swizzle dp_swizzle()
-{
-    return DP == 16 ? kSw32 : DP == 32 ? kSw64 : kSw128;
-}
 
 struct TileKind {
     bool loc, glob;
@@ -199,20 +225,21 @@ __global__ void __launch_bounds__(kThreads, 2)
     using Tm = Tmem<DP>;
     constexpr int NS = Ly::NS;
     constexpr int NPB = Tm::NPB;
+    constexpr int NSB = Tm::NSB;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + Ly::BAR);
     uint64_t *full = bars;                 // [NS] TMA -> MMA
     uint64_t *empty = bars + NS;           // [NS] MMA -> TMA
-    uint64_t *s_full = bars + 2 * NS;      // S of a virtual tile computed
-    uint64_t *s_free = s_full + 1;         // S loaded by the softmax (4 warp arrivals)
-    uint64_t *p_full = s_free + 1;         // [NPB] P written to TMEM buffer b (4 warp arrivals)
+    uint64_t *s_full = bars + 2 * NS;      // [NSB] S of a virtual tile computed into buffer b
+    uint64_t *s_free = s_full + NSB;       // [NSB] S buffer b loaded by the softmax (one arrival per softmax warp)
+    uint64_t *p_full = s_free + NSB;       // [NPB] P written to TMEM buffer b (one arrival per softmax warp)
     uint64_t *pv_done = p_full + NPB;      // [NPB] PV (and row sums) reading P buffer b finished
     uint64_t *q_full = pv_done + NPB;      // Q landed
-    uint64_t *ukb_ready = q_full + 1;      // Uk (bf16) and the ones block written (128 arrivals)
+    uint64_t *ukb_ready = q_full + 1;      // Uk (bf16) and the ones block written (every softmax thread)
     uint64_t *qt_mma = q_full + 2;         // q~ = Q Uk^T computed into TMEM
-    uint64_t *qt_ready = q_full + 3;       // q~ in shared memory, accumulators zeroed (128 arrivals)
+    uint64_t *qt_ready = q_full + 3;       // q~ in shared memory, accumulators zeroed (every softmax thread)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_full + 4);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -227,18 +254,20 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], 1);
+            mbar_init(&empty[s], 2);  // the S and the PV issuer both release a stage
         }
-        mbar_init(s_full, 1);
-        mbar_init(s_free, 4);
+        for (int b2 = 0; b2 < NSB; ++b2) {
+            mbar_init(&s_full[b2], 1);
+            mbar_init(&s_free[b2], kSoftmaxWarps);
+        }
         for (int b2 = 0; b2 < NPB; ++b2) {
-            mbar_init(&p_full[b2], 4);
+            mbar_init(&p_full[b2], kSoftmaxWarps);
             mbar_init(&pv_done[b2], 1);
         }
         mbar_init(q_full, 1);
-        mbar_init(ukb_ready, 128);
+        mbar_init(ukb_ready, kSoftmaxThreads);
         mbar_init(qt_mma, 1);
-        mbar_init(qt_ready, 128);
+        mbar_init(qt_ready, kSoftmaxThreads);
         *abort_flag = 0;
         mbar_init_fence();
     }
@@ -273,37 +302,35 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tma_load_2d(st + Ly::K_OFF, &tmK, 0, krow, &full[s]);
                     tma_load_2d(st + Ly::V_OFF, &tmV, 0, krow, &full[s]);
                 } else {
-                    mbar_expect_tx(&full[s], 2 * BN * DP * 2);
+                    mbar_expect_tx(&full[s], BN * DP * 2 + BN * vd_row<DP>() * 2);
                     tma_load_2d(st + Ly::KD_OFF, &tmKD, 0, krow, &full[s]);
                     tma_load_2d(st + Ly::VD_OFF, &tmVD, 0, krow, &full[s]);
                 }
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+    } else if (warp == kWarpS || warp == kWarpPV) {
+        // ------------------------------------------------------------ MMA issuers
+        // Two threads in two warps: S products (and q~) from one, PV products
+        // from the other.  A tensor-core instruction costs a thread ~50-150
+        // cycles to issue, independently of other issuing threads, so splitting
+        // the two streams lets each keep up with the softmax.  They write
+        // disjoint TMEM columns; each commit covers its own thread's products,
+        // and a stage is free once both have committed (empty[s] counts 2).
+        constexpr uint64_t kStageStep = Ly::STAGE >> 4;
+        const uint64_t dStg = smem_desc(smem_u32(sm + Ly::STG), 16, 1024, kSw128);  // stage 0, K / V tile
+        bool ok = true;
+        if (lane == 0 && warp == kWarpS) {
             constexpr uint32_t idS = idesc_bf16(BM, BN, false);
-            constexpr uint32_t idPV = idesc_bf16(BM, 64, true);
-            constexpr uint32_t idPVg = idesc_bf16(BM, DP, true);
             constexpr uint32_t idQT = idesc_bf16(BM, DP, false);
-            constexpr uint32_t idSum = idesc_bf16(BM, 16, false);
             // Shared-memory descriptors, built once: a k-step of 16 elements adds
-            // 32 bytes along a K-major row (2 in the address field) and 16 rows
-            // (16 * row bytes) along an MN-major operand.
+            // 32 bytes along a K-major row (2 in the address field).
             const uint64_t dQ = smem_desc(smem_u32(sm + Ly::Q), 16, 1024, kSw128);
             const uint64_t dQT = smem_desc(smem_u32(sm + Ly::QT), 16, 8 * DP * 2, dp_swizzle<DP>());
             const uint64_t dUKB = smem_desc(smem_u32(sm + Ly::UKB), 16, 1024, kSw128);
-            const uint64_t dStg = smem_desc(smem_u32(sm + Ly::STG), 16, 1024, kSw128);  // stage 0, K tile
             const uint64_t dStgD = smem_desc(smem_u32(sm + Ly::STG), 16, 8 * DP * 2, dp_swizzle<DP>());
-            constexpr uint64_t kStageStep = Ly::STAGE >> 4;
-            constexpr uint64_t kVOff = Ly::V_OFF >> 4, kVDOff = Ly::VD_OFF >> 4;
-            constexpr uint64_t kVStep = (16 * 128) >> 4, kVDStep = (16 * DP * 2) >> 4;
-            // all-ones B operand (16 columns x 16 keys per k-step; every byte pair is 1.0)
-            const uint64_t ones_desc = smem_desc(smem_u32(sm + Ly::ONES), 128, 256, kSwNone);
-            const uint32_t tS = tmem + Tm::S, tOL = tmem + Tm::OL, tOG = tmem + Tm::OG;
-            const uint32_t tSum = tmem + Tm::SUM, tP = tmem + Tm::P;
+            const uint32_t tS = tmem + Tm::S, tOL = tmem + Tm::OL;
             // q~ = Q Uk^T into the O_loc columns
-            bool ok = mbar_wait(q_full, 0, abort_flag) && mbar_wait(ukb_ready, 0, abort_flag);
+            ok = mbar_wait(q_full, 0, abort_flag) && mbar_wait(ukb_ready, 0, abort_flag);
             if (ok) {
                 tc_fence_after();
 #pragma unroll
@@ -313,31 +340,50 @@ __global__ void __launch_bounds__(kThreads, 2)
                 ok = mbar_wait(qt_ready, 0, abort_flag);
                 tc_fence_after();
             }
-            auto issue_S = [&](int t, VTile vt) -> bool {
-                const int s = t % NS;
-                if (!mbar_wait(&full[s], (t / NS) & 1, abort_flag))
-                    return false;
-                if (t >= 1 && !mbar_wait(s_free, (t - 1) & 1, abort_flag))
-                    return false;
+            // S(t) into buffer t % NSB once the buffer's previous S has been loaded
+            VTile vt = vt_first(i0, i_last, w);
+            for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
+                const int s = t % NS, sb = t % NSB;
+                if (!mbar_wait(&full[s], (t / NS) & 1, abort_flag) ||
+                    (t >= NSB && !mbar_wait(&s_free[sb], ((t / NSB) - 1) & 1, abort_flag))) {
+                    ok = false;
+                    break;
+                }
                 tc_fence_after();
+                const uint32_t tSb = tS + sb * BN;
                 if (vt.loc) {
                     const uint64_t dK = dStg + s * kStageStep;
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        mma_f16_ss(tS, dQ + 2 * kk, dK + 2 * kk, idS, kk > 0);
+                        mma_f16_ss(tSb, dQ + 2 * kk, dK + 2 * kk, idS, kk > 0);
                 } else {
                     const uint64_t dKD = dStgD + s * kStageStep;
 #pragma unroll
                     for (int kk = 0; kk < DP / 16; ++kk)
-                        mma_f16_ss(tS, dQT + 2 * kk, dKD + 2 * kk, idS, kk > 0);
+                        mma_f16_ss(tSb, dQT + 2 * kk, dKD + 2 * kk, idS, kk > 0);
                 }
-                mma_commit(s_full);
-                return true;
-            };
-            auto issue_PV = [&](int t, VTile vt) -> bool {
+                mma_commit(&s_full[sb]);
+                mma_commit(&empty[s]);
+            }
+        } else if (lane == 0 && warp == kWarpPV) {
+            constexpr uint32_t idPV = idesc_bf16(BM, 64, true);
+            // global PV: N = DP + 16 when v^D rows carry the ones (O_glob, then the row sums)
+            constexpr uint32_t idPVg = idesc_bf16(BM, vd_has_ones<DP>() ? DP + 16 : DP, true);
+            constexpr uint32_t idSum = idesc_bf16(BM, 16, false);
+            // a k-step of 16 keys adds 16 rows (16 * row bytes) along an MN-major operand
+            const uint64_t dStgVD = smem_desc(smem_u32(sm + Ly::STG), 16, 8 * vd_row<DP>() * 2, vd_swizzle<DP>());
+            constexpr uint64_t kVOff = Ly::V_OFF >> 4, kVDOff = Ly::VD_OFF >> 4;
+            constexpr uint64_t kVStep = (16 * 128) >> 4, kVDStep = (16 * vd_row<DP>() * 2) >> 4;
+            // all-ones B operand (16 columns x 16 keys per k-step; every byte pair is 1.0)
+            const uint64_t ones_desc = smem_desc(smem_u32(sm + Ly::ONES), 128, 256, kSwNone);
+            const uint32_t tOL = tmem + Tm::OL, tOG = tmem + Tm::OG, tSum = tmem + Tm::SUM, tP = tmem + Tm::P;
+            VTile vt = vt_first(i0, i_last, w);
+            for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
                 const int s = t % NS, pb = t % NPB;
-                if (!mbar_wait(&p_full[pb], (t / NPB) & 1, abort_flag))
-                    return false;
+                if (!mbar_wait(&p_full[pb], (t / NPB) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
                 tc_fence_after();
                 const uint32_t aP = tP + pb * (BN / 2);
                 if (vt.loc) {
@@ -348,44 +394,30 @@ __global__ void __launch_bounds__(kThreads, 2)
                         mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);  // row sums of P
                     }
                 } else {
-                    const uint64_t dVD = dStgD + s * kStageStep + kVDOff;
+                    const uint64_t dVD = dStgVD + s * kStageStep + kVDOff;
 #pragma unroll
-                    for (int kk = 0; kk < BN / 16; ++kk) {  // P times V^D
+                    for (int kk = 0; kk < BN / 16; ++kk) {  // P times [V^D | ones]
                         mma_f16_ts(tOG, aP + kk * 8, dVD + kk * kVDStep, idPVg, true);
-                        mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);
+                        if constexpr (!vd_has_ones<DP>())
+                            mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);
                     }
                 }
                 mma_commit(&pv_done[pb]);
                 mma_commit(&empty[s]);
-                return true;
-            };
-            // S(t + 1) needs S(t) loaded by the softmax; PV(t) needs P(t)
-            VTile vs = vt_first(i0, i_last, w), vp = vs;
-            if (ok && VT > 0) {
-                ok = issue_S(0, vs);
-                vs = vt_next(vs, i0, i_last, w);
-            }
-            for (int t = 0; ok && t < VT; ++t) {
-                if (t + 1 < VT) {
-                    ok = issue_S(t + 1, vs);
-                    vs = vt_next(vs, i0, i_last, w);
-                }
-                if (ok)
-                    ok = issue_PV(t, vp);
-                vp = vt_next(vp, i0, i_last, w);
             }
         }
-    } else {
+    } else {  // warps 2 .. 2 + kSoftmaxWarps - 1
         // ------------------------------------------------------------ softmax warps
+        // one query row per thread: warp w reads TMEM lanes 32 (w % 4) .. + 31
         const int quad = warp & 3;
         const int row = 32 * quad + lane;
         const int i = i0 + row;
         const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
-        const int stid = threadIdx.x - 64;  // 0..127
+        const int stid = threadIdx.x - 64;  // 0 .. kSoftmaxThreads - 1
         // ---- set-up: Uk as a bf16 operand, the ones block, Uv for the epilogue
         {
             const float *Ukg = a.Uk + (size_t)g * a.dd * 64;
-            for (int idx = stid; idx < DP * 8; idx += 128) {  // row c, chunk ch of 8 values
+            for (int idx = stid; idx < DP * 8; idx += kSoftmaxThreads) {  // row c, chunk ch of 8 values
                 const int c = idx / 8, ch = idx % 8;
                 uint4 v = make_uint4(0u, 0u, 0u, 0u);
                 if (c < a.dd) {
@@ -402,7 +434,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             fence_proxy_async_smem();
             mbar_arrive(ukb_ready);
             float *sUv = reinterpret_cast<float *>(sm + Ly::UV);
-            for (int idx = stid; idx < DP * 64; idx += 128) {
+            for (int idx = stid; idx < DP * 64; idx += kSoftmaxThreads) {
                 const int c = idx / 64, t = idx % 64;
                 sUv[idx] = c < a.dd ? a.Uv[((size_t)g * a.dd + c) * 64 + t] : 0.f;
             }
@@ -414,35 +446,37 @@ __global__ void __launch_bounds__(kThreads, 2)
         };
         bool ok = wait_uniform(qt_mma, 0);
         if (ok) {
-            // q~ (fp32, TMEM) -> bf16 operand rows in shared memory; then clear the accumulators
             tc_fence_after();
-            uint32_t r[16];
-            unsigned char *qrow = sm + Ly::QT;
-#pragma unroll
-            for (int c = 0; c < DP; c += 16) {
-                tmem_ld16(tl + Tm::OL + c, r);
-#pragma unroll
-                for (int k = 0; k < 2; ++k)
-                    st_swz<DP * 2>(qrow, row, c / 8 + k,
-                                   make_uint4(pack_bf16(__uint_as_float(r[8 * k + 0]), __uint_as_float(r[8 * k + 1])),
-                                              pack_bf16(__uint_as_float(r[8 * k + 2]), __uint_as_float(r[8 * k + 3])),
-                                              pack_bf16(__uint_as_float(r[8 * k + 4]), __uint_as_float(r[8 * k + 5])),
-                                              pack_bf16(__uint_as_float(r[8 * k + 6]), __uint_as_float(r[8 * k + 7]))));
-            }
             uint32_t z[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e)
                 z[e] = 0u;
+            {
+                // q~ (fp32, TMEM) -> bf16 operand rows in shared memory; then clear the accumulators
+                uint32_t r[16];
+                unsigned char *qrow = sm + Ly::QT;
 #pragma unroll
-            for (int c = 0; c < 64; c += 16)
-                tmem_st16(tl + Tm::OL + c, z);
+                for (int c = 0; c < DP; c += 16) {
+                    tmem_ld16(tl + Tm::OL + c, r);
 #pragma unroll
-            for (int c = 0; c < DP + 16; c += 16)  // O_glob and the row-sum columns
-                tmem_st16(tl + Tm::OG + c, z);
+                    for (int k = 0; k < 2; ++k)
+                        st_swz<DP * 2>(qrow, row, c / 8 + k,
+                                       make_uint4(pack_bf16(__uint_as_float(r[8 * k + 0]), __uint_as_float(r[8 * k + 1])),
+                                                  pack_bf16(__uint_as_float(r[8 * k + 2]), __uint_as_float(r[8 * k + 3])),
+                                                  pack_bf16(__uint_as_float(r[8 * k + 4]), __uint_as_float(r[8 * k + 5])),
+                                                  pack_bf16(__uint_as_float(r[8 * k + 6]), __uint_as_float(r[8 * k + 7]))));
+                }
+#pragma unroll
+                for (int c = 0; c < 64; c += 16)
+                    tmem_st16(tl + Tm::OL + c, z);
+#pragma unroll
+                for (int c = 0; c < DP + 16; c += 16)  // O_glob and the row-sum columns
+                    tmem_st16(tl + Tm::OG + c, z);
+            }
             tmem_wait_st();
             fence_proxy_async_smem();
         }
-        asm volatile("bar.sync 1, 128;" ::: "memory");  // Uv staged by all softmax threads
+        asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");  // Uv staged by all softmax threads
         tc_fence_before();
         mbar_arrive(qt_ready);
 
@@ -467,7 +501,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         VTile vt = vt_first(i0, i_last, w);
         for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
             const int j0 = vt.kt * BN;
-            if (!wait_uniform(s_full, t & 1)) {
+            const int sb = t % NSB;
+            if (!wait_uniform(&s_full[sb], (t / NSB) & 1)) {
                 ok = false;
                 break;
             }
@@ -475,16 +510,17 @@ __global__ void __launch_bounds__(kThreads, 2)
             float s[BN];
             {
                 uint32_t r[BN];
-                tmem_ld64(tl + Tm::S, r);
+                tmem_ld64(tl + Tm::S + sb * BN, r);
 #pragma unroll
                 for (int e = 0; e < BN; ++e)
                     s[e] = __uint_as_float(r[e]);
             }
-            // the S columns may be overwritten now (S(t + 1))
+            // this S buffer may be overwritten now (S(t + NSB))
             tc_fence_before();
             __syncwarp();
             if (lane == 0)
-                mbar_arrive(s_free);
+                mbar_arrive(&s_free[sb]);
+
             // masks: causal (tiles reaching past row i0), the other part of a
             // band tile, rows past the end; the kept columns form one range
             if (j0 + BN - 1 > i0 || vt.band || i0 + BM > N) {
@@ -503,9 +539,22 @@ __global__ void __launch_bounds__(kThreads, 2)
             // raise the running max only when it grows by more than the threshold
             const bool raise = mt > m_used + kRescaleThreshold;
             const bool scale_o = raise && m_used != -INFINITY;
+            // O's scale factor when the running max is raised (applied below, once P is computed)
+            const float alpha = scale_o ? ex2_approx(m_used - mt) : 1.f;
+            if (raise)
+                m_used = mt;
+            // P = 2^(s * c2 - m) in bf16 pairs (masked entries give 0)
+            const float mneg = m_used == -INFINITY ? 0.f : -m_used;
+            uint32_t pk[BN / 2];
+#pragma unroll
+            for (int e = 0; e < BN; e += 2) {
+                float x0, x1;
+                ffma2(x0, x1, s[e], s[e + 1], c2, c2, mneg, mneg);
+                pk[e / 2] = ex2_bf16x2(cvt_bf16x2(x0, x1));
+            }
             if (__any_sync(0xffffffffu, scale_o)) {
-                const float alpha = scale_o ? ex2_approx(m_used - mt) : 1.f;
-                // every earlier PV must have landed before O is rescaled
+                // every earlier PV must have landed before O is rescaled (and PV(t),
+                // which needs P(t), cannot start before it is)
                 if (!wait_pv(t - 1)) {
                     ok = false;
                     break;
@@ -528,17 +577,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                         r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
                     tmem_st16(tl + Tm::OG + c, r);
                 }
-            }
-            if (raise)
-                m_used = mt;
-            // P = 2^(s * c2 - m) in bf16 pairs (masked entries give 0)
-            const float mneg = m_used == -INFINITY ? 0.f : -m_used;
-            uint32_t pk[BN / 2];
-#pragma unroll
-            for (int e = 0; e < BN; e += 2) {
-                float x0, x1;
-                ffma2(x0, x1, s[e], s[e + 1], c2, c2, mneg, mneg);
-                pk[e / 2] = ex2_bf16x2(cvt_bf16x2(x0, x1));
             }
             // the PV that last read this P buffer (tile t - NPB) must be done with it
             if (!wait_pv(t - NPB)) {
@@ -670,7 +708,10 @@ static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
     if (!make_map(&mq, a.q, rq, 64, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&mk, a.k, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !make_map(&mv, a.v, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) || !make_map(&mkd, a.kd, rk, DP, BN, swd) ||
-        !make_map(&mvd, a.vd, rk, DP, BN, swd))
+        !make_map(&mvd, a.vd, rk, vd_row<DP>(), BN,
+                  vd_row<DP>() == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    if (a.vd_stride != vd_row<DP>())
         return cudaErrorInvalidValue;
     auto kern = prefill_tc_kernel<DP>;
     const size_t smem = Layout<DP>::TOTAL + 1024;

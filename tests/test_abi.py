@@ -45,7 +45,10 @@ def test_workspace_sizes_are_host_only(lib):
     assert n > 0 and n % 256 == 0
     assert L.dar_decode_workspace_bytes(ctypes.byref(c), 3) == 0      # Hq not a multiple of Hkv
     assert L.dar_decode_workspace_bytes(ctypes.byref(_cache(lib, d=32)), 4) == 0
-    assert L.dar_prefill_workspace_bytes(lib.DAR_BF16, 2, 3, 100, 16) == 2 * 19200  # K and V, 2*3*100*16*2 B each
+    # k^D rows of 16 bf16 (2*3*100*16*2 B); v^D rows of 32 (16 values, then 16 ones for the row sums)
+    assert L.dar_prefill_workspace_bytes(lib.DAR_BF16, 2, 3, 100, 16) == 19200 + 38400
+    assert L.dar_prefill_workspace_bytes(lib.DAR_BF16, 1, 1, 4, 32) == 256 + 512   # rows of 32 and 64
+    assert L.dar_prefill_workspace_bytes(lib.DAR_F32, 1, 1, 4, 32) == 2 * 512     # fp32: plain rows
     assert L.dar_prefill_workspace_bytes(lib.DAR_BF16, 1, 1, 3, 8) == 2 * 256  # 48 B rounded up to 256
     assert L.dar_prefill_workspace_bytes(lib.DAR_F32, 0, 3, 100, 16) == 0
 

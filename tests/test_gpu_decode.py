@@ -49,16 +49,16 @@ def test_decode_160m_repeat_calls_identical():
     np.testing.assert_array_equal(a, b)
 
 
-def test_decode_1b_gqa_paged_sampled():
+def test_decode_1b_gqa_paged():
     """B64 Hq32 Hkv8 dd16 w256, ragged L in [1024, 32768], shuffled 64-token
-    pages; the oracle checks every head of the shortest, the longest and a few
-    other sequences."""
+    pages; the oracle checks one head of every sequence (cycling through the
+    heads) and every head of the shortest, the longest and a few others."""
     cfg = I.DECODE_1B_GQA
     wl = W.DecodeWorkload(cfg, keep_history=True)
     got = gpu_out(wl)
     lens = wl.lens
     seqs = sorted({int(np.argmin(lens)), int(np.argmax(lens)), 0, 17, 42})
-    heads = [(b, h) for b in seqs for h in range(cfg.Hq)]
+    heads = sorted({(b, h) for b in seqs for h in range(cfg.Hq)} | {(b, (5 * b) % cfg.Hq) for b in range(cfg.B)})
     want = oracle_decode(wl, heads=heads)
     err = max(np.abs(got[b, h] - want[b, h]).max() for b, h in heads)
     assert err <= TOL["bf16"], err
@@ -68,11 +68,13 @@ def test_decode_1b_gqa_paged_sampled():
 @pytest.mark.parametrize("k", range(16))
 def test_decode_sweep_point(k):
     """B16 H16 L16384, w in {64, 256, 1024, 16384} x d_down in {8, 16, 32, 64}:
-    two sequences checked head by head (w = 16384 is plain attention)."""
+    one head of every sequence, and every head of the first and last
+    (w = 16384 is plain attention)."""
     cfg = I.sweep_point(k)
     wl = W.DecodeWorkload(cfg, keep_history=True)
     got = gpu_out(wl)
-    heads = [(b, h) for b in (0, cfg.B - 1) for h in range(cfg.Hq)]
+    heads = sorted({(b, h) for b in (0, cfg.B - 1) for h in range(cfg.Hq)} | {(b, (3 * b + k) % cfg.Hq)
+                                                                           for b in range(cfg.B)})
     want = oracle_decode(wl, heads=heads)
     err = max(np.abs(got[b, h] - want[b, h]).max() for b, h in heads)
     assert err <= TOL["bf16"], err

@@ -65,16 +65,22 @@ def test_prefill_small_cases(case):
     assert np.isfinite(got).all()
 
 
-def test_prefill_410m_sampled_rows():
+def test_prefill_410m_full_head_and_tile_edges():
     """B8 H16 N8192 d64 dd16 w512 bf16 at full size, in the configuration the
-    benchmark times; the oracle evaluates a sample of rows one by one (first,
-    window edges, tile edges, last)."""
+    benchmark times.  The oracle evaluates every row of one (b, h), and in all
+    128 (b, h) the rows at tile and window edges (first, 63/64, 127/128, w - 1,
+    w, w + 63, the last tiles, the last row) plus random rows."""
     cfg = I.PREFILL_410M
     wl, got = gpu_prefill(cfg)
+    assert np.isfinite(got).all()
     rng = np.random.default_rng(0)
-    pos = [0, 1, cfg.w - 1, cfg.w, cfg.w + 1, 127, 128, 4095, 4096, cfg.N - 1] + list(rng.integers(0, cfg.N, 6))
-    rows = np.array([(b, h, i) for b, h in [(0, 0), (3, 7), (7, 15)] for i in pos])
+    N, w = cfg.N, cfg.w
+    edges = [0, 1, 63, 64, 127, 128, w - 1, w, w + 1, w + 63, w + 64, N - 129, N - 128, N - 65, N - 64, N - 1]
+    rows = [(5, 11, i) for i in range(N)]
+    for b in range(cfg.B):
+        for h in range(cfg.Hq):
+            rows += [(b, h, i) for i in edges + list(rng.integers(0, N, 2))]
+    rows = np.array(rows)
     want = oracle_prefill(wl, rows=rows)
     err = np.abs(got[rows[:, 0], rows[:, 1], rows[:, 2]] - want).max()
     assert err <= TOL["bf16"], err
-    assert np.isfinite(got).all()
