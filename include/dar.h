@@ -226,6 +226,32 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
  */
 dar_status dar_check_bounded_wait(int32_t *status, uint32_t limit_us, void *stream);
 
+/*
+ * Chunked prefill over an existing cache (Sec. 2.3 inference with the cache
+ * scheme of Sec. 5: a long prompt enters the cache in chunks).  Every sequence
+ * b holds L_b = seq_lens[b] tokens and takes n more: k_new, v_new
+ * [B][Hkv][n][d] at positions L_b .. L_b + n - 1, with queries q [B][Hq][n][d].
+ * out[b][h][r] (same layout as q) is row L_b + r of the causal forward over
+ * the whole sequence (Eq. 3-4: local keys i - j < w at full d, the others
+ * through the bottleneck), i.e. what dar_attn_prefill would give for those
+ * rows over the concatenated sequence.  The call then appends the chunk
+ * exactly as dar_cache_append(cache, k_new, v_new, n, NULL, Dk, Dv) does
+ * (the cache bytes equal n one-token appends).
+ *   bf16 caches with d_down in {16, 32, 64}; Dk, Dv [Hkv][d][d_down] and
+ *   Uk, Uv [Hkv][d_down][d] fp32; all pointers 16-byte aligned; workspace of
+ *   dar_prefill_chunk_workspace_bytes(cache, n) bytes (no initialisation).
+ * Three kernels run in order on `stream`: a gather of the keys the chunk's
+ * queries can see (window rows, and bottleneck rows of the tokens the chunk
+ * pushes out of the window), the attention, and the append.  A needed
+ * block-table entry outside [0, num_pages) or a length beyond the cache's
+ * capacity sets *status = DAR_ERR_CAPACITY.
+ */
+size_t dar_prefill_chunk_workspace_bytes(const dar_cache *cache, int32_t n);
+dar_status dar_prefill_chunk(const dar_cache *cache, int32_t Hq, int32_t n, const void *q,
+                             const void *k_new, const void *v_new, const float *Dk, const float *Uk,
+                             const float *Dv, const float *Uv, float scale, void *out, void *workspace,
+                             size_t workspace_bytes, void *stream);
+
 /* Message for the last non-OK return on this thread ("" if none). */
 const char *dar_last_error(void);
 

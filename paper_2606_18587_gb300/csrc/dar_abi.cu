@@ -203,6 +203,28 @@ dar_status prepare_decode(const dar_cache *cache, int32_t Hq, const void *q, con
     return ok();
 }
 
+struct ChunkLayout {
+    size_t pos0, kw, vw, kdt, vdt, total;
+};
+
+// Workspace of dar_prefill_chunk: the lengths before the chunk, the window
+// buffers (full-d keys / values the chunk's queries can see as local) and the
+// tail buffers (bottleneck keys / values near the window edge).
+ChunkLayout chunk_layout(const dar_cache *c, int n)
+{
+    ChunkLayout L;
+    const size_t bg = (size_t)c->B * c->Hkv;
+    const size_t win = bg * dar::chunk_window_rows(c->w, n) * c->d * sizeof(uint16_t);
+    const size_t tail = bg * dar::chunk_tail_rows(n) * c->d_down * sizeof(uint16_t);
+    L.pos0 = 0;
+    L.kw = align256((size_t)c->B * sizeof(int32_t));
+    L.vw = L.kw + align256(win);
+    L.kdt = L.vw + align256(win);
+    L.vdt = L.kdt + align256(tail);
+    L.total = L.vdt + align256(tail);
+    return L;
+}
+
 }  // namespace
 
 void dar::set_last_error(const char *msg) { g_err = msg ? msg : ""; }
@@ -297,6 +319,80 @@ dar_status dar_decode_step(const dar_cache *cache, const void *k_new, const void
     // neither q nor Uk: the decode's query-side set-up may overlap it
     dc.prep_overlaps_prev = app_empty ? 0 : 1;
     return from_cuda(dar::launch_decode(cache->dtype, cache->d_down, dc, st), "dar_decode_step decode launch");
+}
+
+size_t dar_prefill_chunk_workspace_bytes(const dar_cache *cache, int32_t n)
+{
+    if (check_cache(cache) != DAR_OK || n < 0)
+        return 0;
+    return chunk_layout(cache, n).total;
+}
+
+dar_status dar_prefill_chunk(const dar_cache *cache, int32_t Hq, int32_t n, const void *q,
+                             const void *k_new, const void *v_new, const float *Dk, const float *Uk,
+                             const float *Dv, const float *Uv, float scale, void *out, void *workspace,
+                             size_t workspace_bytes, void *stream)
+{
+    dar::AppendArgs ap;
+    bool empty = false;
+    dar_status s = prepare_append(cache, k_new, v_new, n, nullptr, Dk, Dv, &ap, &empty);
+    if (s != DAR_OK)
+        return s;
+    if (cache->dtype != DAR_BF16 || cache->d_down < 16)
+        return fail(DAR_ERR_UNSUPPORTED, "dar_prefill_chunk: bf16 caches with d_down in {16, 32, 64}");
+    if (Hq < cache->Hkv || Hq % cache->Hkv)
+        return fail(DAR_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", Hq, cache->Hkv);
+    if (empty)
+        return ok();
+    if (!q || !Uk || !Uv || !out || !workspace)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(q) || !aligned16(out) || !aligned16(Uk) || !aligned16(Uv) || !aligned16(workspace))
+        return fail(DAR_ERR_INVALID_ARG, "q, out, Uk, Uv and workspace must be 16-byte aligned");
+    if ((long long)cache->B * Hq > 65535 || (long long)cache->B * cache->Hkv > 65535)
+        return fail(DAR_ERR_UNSUPPORTED, "B*Hq=%lld > 65535", (long long)cache->B * Hq);
+    if ((double)cache->B * Hq * n >= 2147483647.0 ||
+        (double)cache->B * cache->Hkv * dar::chunk_window_rows(cache->w, n) >= 2147483647.0 ||
+        (double)cache->num_pages * cache->Hkv * DAR_PAGE_SIZE >= 2147483647.0)
+        return fail(DAR_ERR_UNSUPPORTED, "dar_prefill_chunk: row indices beyond int32");
+    const ChunkLayout L = chunk_layout(cache, n);
+    if (workspace_bytes < L.total)
+        return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, L.total);
+    char *ws = static_cast<char *>(workspace);
+    dar::ChunkArgs c;
+    c.app = ap;
+    c.win_k = cache->win_k;
+    c.win_v = cache->win_v;
+    c.pos0 = reinterpret_cast<int32_t *>(ws + L.pos0);
+    c.kw = ws + L.kw;
+    c.vw = ws + L.vw;
+    c.kdt = ws + L.kdt;
+    c.vdt = ws + L.vdt;
+    dar::PrefillArgs &a = c.pf;
+    a.q = q;
+    a.k = a.v = a.kd = a.vd = nullptr;
+    a.Uk = Uk;
+    a.Uv = Uv;
+    a.out = out;
+    a.status = cache->status;
+    a.B = cache->B;
+    a.Hq = Hq;
+    a.Hkv = cache->Hkv;
+    a.N = 0;
+    a.w = cache->w;
+    a.dd = cache->d_down;
+    a.kd_stride = a.vd_stride = cache->d_down;
+    a.qscale = default_scale(scale, cache->d) * kLog2e;
+    a.pos0 = c.pos0;
+    a.block_table = cache->block_table;
+    a.pool_kd = cache->pool_kd;
+    a.pool_vd = cache->pool_vd;
+    a.n = n;
+    a.NW = dar::chunk_window_rows(cache->w, n);
+    a.NT = dar::chunk_tail_rows(n);
+    a.maxp = cache->max_pages_per_seq;
+    a.num_pages = cache->num_pages;
+    return from_cuda(dar::launch_prefill_chunk(cache->d_down, c, static_cast<cudaStream_t>(stream)),
+                     "dar_prefill_chunk launch");
 }
 
 size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int32_t N,

@@ -52,6 +52,16 @@ struct PrefillArgs {
     int32_t *status;        // device error word or nullptr
     int B, Hq, Hkv, N, w, dd, kd_stride, vd_stride;
     float qscale;  // scale * log2(e)
+    // chunked prefill over a cache (dar_prefill_chunk): query b sits at
+    // position pos0[b] + r, r < n; local keys come from a window buffer of NW
+    // rows per (b, KV head), starting at the 64-aligned position below
+    // pos0[b] - w + 1; global keys from whole pages through the block table,
+    // and from a tail buffer of NT rows per (b, KV head) from the 64-aligned
+    // position below pos0[b] - w on (k, v, kd, vd then point at the buffers)
+    const int32_t *pos0 = nullptr;
+    const int32_t *block_table = nullptr;
+    const void *pool_kd = nullptr, *pool_vd = nullptr;
+    int n = 0, NW = 0, NT = 0, maxp = 0, num_pages = 0;
 };
 
 // Row stride (elements) of the prefill bottleneck workspace: the tensor-core
@@ -89,6 +99,20 @@ cudaError_t launch_cache_append(dar_dtype dt, int dd, const AppendArgs &a, cudaS
 cudaError_t launch_decode(dar_dtype dt, int dd, const DecodeArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_simt(dar_dtype dt, int dd, const PrefillArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s);
+
+// Chunked prefill over a cache: gather kernel, attention (chunk mode), then
+// the cache append of the chunk.  Buffers of the workspace (see dar_abi.cu).
+struct ChunkArgs {
+    PrefillArgs pf;        // attention arguments (q, out, Uk, Uv, scale, chunk fields)
+    AppendArgs app;        // the append of the chunk (k_new, v_new, Dk, Dv, cache)
+    const void *win_k, *win_v;  // the cache ring (read by the gather kernel)
+    void *kw, *vw, *kdt, *vdt;  // window and tail buffers
+    int32_t *pos0;              // [B] lengths before the chunk
+};
+cudaError_t launch_prefill_chunk(int dd, const ChunkArgs &c, cudaStream_t s);
+// Rows per (sequence, KV head) of the chunk's window and tail buffers.
+inline int chunk_window_rows(int w, int n) { return (w + n + 126 + 63) / 64 * 64; }
+inline int chunk_tail_rows(int n) { return (n + 127 + 63) / 64 * 64; }
 
 // Split-K geometry of the decode kernel (shared by workspace sizing and launch).
 struct DecodeGeometry {

@@ -215,11 +215,17 @@ __device__ __forceinline__ int vt_count(int i0, int i_last, int w)
     return n;
 }
 
-template <int DP>
+// CH = false: the causal forward over positions 0..N-1 of q, k, v.  CH = true:
+// chunked prefill over a cache (positions pos0[b] .. pos0[b] + n - 1; local
+// keys from the window buffer, global keys from whole pages (tmPK, tmPV)
+// or the tail buffer; v^D rows without ones, so every row sum takes a
+// product of its own).
+template <int DP, bool CH>
 __global__ void __launch_bounds__(kThreads, 2)
     prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKD,
-                      const __grid_constant__ CUtensorMap tmVD, PrefillArgs a)
+                      const __grid_constant__ CUtensorMap tmVD, const __grid_constant__ CUtensorMap tmPK,
+                      const __grid_constant__ CUtensorMap tmPV, PrefillArgs a)
 {
     using Ly = Layout<DP>;
     using Tm = Tmem<DP>;
@@ -243,13 +249,22 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_full + 4);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
+    // global pv rows carry the ones of the row sums (plain rows in chunk mode)
+    constexpr bool kOnes = !CH && vd_has_ones<DP>();
+    constexpr int VR = kOnes ? vd_row<DP>() : DP;  // elements per v^D row in a stage
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int N = a.N, w = a.w;
-    const int nqt = (N + BM - 1) / BM;
-    const int qt = nqt - 1 - (int)blockIdx.y;  // longest rows first
+    const int w = a.w;
     const int bh = blockIdx.x, b = bh / a.Hq, h = bh % a.Hq, g = h / (a.Hq / a.Hkv);
-    const int i0 = qt * BM, i_last = min(i0 + BM, N) - 1;
+    const int L0 = CH ? __ldg(a.pos0 + b) : 0;  // position of query row 0
+    const int nrows = CH ? a.n : a.N;            // query rows per (b, h)
+    const int N = L0 + nrows;                    // end of the query positions
+    const int nqt = (nrows + BM - 1) / BM;
+    const int qt = nqt - 1 - (int)blockIdx.y;  // longest rows first
+    const int i0 = L0 + qt * BM, i_last = min(i0 + BM, N) - 1;
     const int VT = vt_count(i0, i_last, w);
+    // chunk mode: first positions of the window and tail buffers
+    const int kb0 = CH ? max(0, L0 - w + 1) / BN * BN : 0;
+    const int kt0 = CH ? max(0, L0 - w) / BN * BN : 0;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; ++s) {
@@ -288,23 +303,40 @@ __global__ void __launch_bounds__(kThreads, 2)
             prefetch_tensormap(&tmV);
             prefetch_tensormap(&tmKD);
             prefetch_tensormap(&tmVD);
+            if constexpr (CH) {
+                prefetch_tensormap(&tmPK);
+                prefetch_tensormap(&tmPV);
+            }
             mbar_expect_tx(q_full, BM * 64 * 2);
-            tma_load_2d(sm + Ly::Q, &tmQ, 0, (b * a.Hq + h) * N + i0, q_full);
+            tma_load_2d(sm + Ly::Q, &tmQ, 0, (b * a.Hq + h) * nrows + qt * BM, q_full);
             VTile vt = vt_first(i0, i_last, w);
             for (int t = 0; t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
                 const int s = t % NS;
                 if (t >= NS && !mbar_wait(&empty[s], ((t / NS) - 1) & 1, abort_flag))
                     break;
                 unsigned char *st = sm + Ly::STG + s * Ly::STAGE;
-                const int krow = (b * a.Hkv + g) * N + vt.kt * BN;
+                const int j0 = vt.kt * BN;
                 if (vt.loc) {
+                    const int krow = CH ? (b * a.Hkv + g) * a.NW + (j0 - kb0) : (b * a.Hkv + g) * a.N + j0;
                     mbar_expect_tx(&full[s], 2 * BN * 64 * 2);
                     tma_load_2d(st + Ly::K_OFF, &tmK, 0, krow, &full[s]);
                     tma_load_2d(st + Ly::V_OFF, &tmV, 0, krow, &full[s]);
                 } else {
-                    mbar_expect_tx(&full[s], BN * DP * 2 + BN * vd_row<DP>() * 2);
-                    tma_load_2d(st + Ly::KD_OFF, &tmKD, 0, krow, &full[s]);
-                    tma_load_2d(st + Ly::VD_OFF, &tmVD, 0, krow, &full[s]);
+                    mbar_expect_tx(&full[s], BN * DP * 2 + BN * VR * 2);
+                    if (CH && j0 + BN <= kt0) {  // a whole page migrated before this call
+                        int pid = a.block_table[(size_t)b * a.maxp + vt.kt];
+                        if (pid < 0 || pid >= a.num_pages) {
+                            report(a.status, DAR_ERR_CAPACITY);
+                            pid = 0;
+                        }
+                        const int prow = (pid * a.Hkv + g) * BN;
+                        tma_load_2d(st + Ly::KD_OFF, &tmPK, 0, prow, &full[s]);
+                        tma_load_2d(st + Ly::VD_OFF, &tmPV, 0, prow, &full[s]);
+                    } else {
+                        const int krow = CH ? (b * a.Hkv + g) * a.NT + (j0 - kt0) : (b * a.Hkv + g) * a.N + j0;
+                        tma_load_2d(st + Ly::KD_OFF, &tmKD, 0, krow, &full[s]);
+                        tma_load_2d(st + Ly::VD_OFF, &tmVD, 0, krow, &full[s]);
+                    }
                 }
             }
         }
@@ -368,12 +400,13 @@ __global__ void __launch_bounds__(kThreads, 2)
         } else if (lane == 0 && warp == kWarpPV) {
             constexpr uint32_t idPV = idesc_bf16(BM, 64, true);
             // global PV: N = DP + 16 when v^D rows carry the ones (O_glob, then the row sums)
-            constexpr uint32_t idPVg = idesc_bf16(BM, vd_has_ones<DP>() ? DP + 16 : DP, true);
+            constexpr uint32_t idPVg = idesc_bf16(BM, kOnes ? DP + 16 : DP, true);
             constexpr uint32_t idSum = idesc_bf16(BM, 16, false);
             // a k-step of 16 keys adds 16 rows (16 * row bytes) along an MN-major operand
-            const uint64_t dStgVD = smem_desc(smem_u32(sm + Ly::STG), 16, 8 * vd_row<DP>() * 2, vd_swizzle<DP>());
+            const uint64_t dStgVD = smem_desc(smem_u32(sm + Ly::STG), 16, 8 * VR * 2,
+                                              kOnes ? vd_swizzle<DP>() : dp_swizzle<DP>());
             constexpr uint64_t kVOff = Ly::V_OFF >> 4, kVDOff = Ly::VD_OFF >> 4;
-            constexpr uint64_t kVStep = (16 * 128) >> 4, kVDStep = (16 * vd_row<DP>() * 2) >> 4;
+            constexpr uint64_t kVStep = (16 * 128) >> 4, kVDStep = (16 * VR * 2) >> 4;
             // all-ones B operand (16 columns x 16 keys per k-step; every byte pair is 1.0)
             const uint64_t ones_desc = smem_desc(smem_u32(sm + Ly::ONES), 128, 256, kSwNone);
             const uint32_t tOL = tmem + Tm::OL, tOG = tmem + Tm::OG, tSum = tmem + Tm::SUM, tP = tmem + Tm::P;
@@ -398,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
                     for (int kk = 0; kk < BN / 16; ++kk) {  // P times [V^D | ones]
                         mma_f16_ts(tOG, aP + kk * 8, dVD + kk * kVDStep, idPVg, true);
-                        if constexpr (!vd_has_ones<DP>())
+                        if constexpr (!kOnes)
                             mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);
                     }
                 }
@@ -610,7 +643,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 l = __uint_as_float(r[0]);
             }
             const float inv = l > 0.f ? 1.f / l : 0.f;
-            bf16 *orow = static_cast<bf16 *>(a.out) + (((size_t)b * a.Hq + h) * N + i) * 64;
+            bf16 *orow = static_cast<bf16 *>(a.out) + (((size_t)b * a.Hq + h) * nrows + (i - L0)) * 64;
 #pragma unroll
             for (int c = 0; c < 64; c += 16) {
                 uint32_t r[16];
@@ -697,23 +730,16 @@ static bool make_map(CUtensorMap *m, const void *base, unsigned long long rows, 
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int DP>
-static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
+constexpr CUtensorMapSwizzle dp_map_swizzle(int DP)
 {
-    CUtensorMap mq, mk, mv, mkd, mvd;
-    const CUtensorMapSwizzle swd = DP == 16 ? CU_TENSOR_MAP_SWIZZLE_32B
-                                   : DP == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                              : CU_TENSOR_MAP_SWIZZLE_128B;
-    const unsigned long long rq = (unsigned long long)a.B * a.Hq * a.N, rk = (unsigned long long)a.B * a.Hkv * a.N;
-    if (!make_map(&mq, a.q, rq, 64, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&mk, a.k, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !make_map(&mv, a.v, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) || !make_map(&mkd, a.kd, rk, DP, BN, swd) ||
-        !make_map(&mvd, a.vd, rk, vd_row<DP>(), BN,
-                  vd_row<DP>() == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B))
-        return cudaErrorInvalidValue;
-    if (a.vd_stride != vd_row<DP>())
-        return cudaErrorInvalidValue;
-    auto kern = prefill_tc_kernel<DP>;
+    return DP == 16 ? CU_TENSOR_MAP_SWIZZLE_32B : DP == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
+}
+
+// One-time attribute set-up per device and instantiation, then the launch.
+template <int DP, bool CH>
+static cudaError_t launch_kernel(const CUtensorMap (&m)[7], const PrefillArgs &a, int nrows, cudaStream_t s)
+{
+    auto kern = prefill_tc_kernel<DP, CH>;
     const size_t smem = Layout<DP>::TOTAL + 1024;
     static PerDeviceOnce once;
     cudaError_t e = per_device_once(once, [&](int) {
@@ -726,9 +752,142 @@ static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
     });
     if (e != cudaSuccess)
         return e;
-    dim3 grid(a.B * a.Hq, (a.N + BM - 1) / BM);
-    kern<<<grid, kThreads, smem, s>>>(mq, mk, mv, mkd, mvd, a);
+    dim3 grid(a.B * a.Hq, (nrows + BM - 1) / BM);
+    kern<<<grid, kThreads, smem, s>>>(m[0], m[1], m[2], m[3], m[4], m[5], m[6], a);
     return cudaGetLastError();
+}
+
+template <int DP>
+static cudaError_t launch_dp(const PrefillArgs &a, cudaStream_t s)
+{
+    CUtensorMap m[7];
+    const unsigned long long rq = (unsigned long long)a.B * a.Hq * a.N, rk = (unsigned long long)a.B * a.Hkv * a.N;
+    if (!make_map(&m[0], a.q, rq, 64, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m[1], a.k, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m[2], a.v, rk, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m[3], a.kd, rk, DP, BN, dp_map_swizzle(DP)) ||
+        !make_map(&m[4], a.vd, rk, vd_row<DP>(), BN,
+                  vd_row<DP>() == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    if (a.vd_stride != vd_row<DP>())
+        return cudaErrorInvalidValue;
+    m[5] = m[3];  // no pages in this mode
+    m[6] = m[4];
+    return launch_kernel<DP, false>(m, a, a.N, s);
+}
+
+// ---------------------------------------------------------------- chunked prefill: gather
+
+// For sequence b (L0 = its length before the chunk) and KV head g:
+//  window buffer rows r < NW hold the full-d key / value of position kb0 + r
+//    when it can be local to a chunk query (kb0 + r in [L0 - w + 1, L0 + n)):
+//    from the ring for positions < L0, from k_new / v_new after; zero otherwise.
+//  tail buffer rows r < NT hold k^D / v^D of position kt0 + r when it is
+//    global to some chunk query (< L0 + n - w): copied from its page when it
+//    migrated before this call (< L0 - w), else Eq. 1 of its full-d row with
+//    the same fp32 chain as the cache append; zero otherwise.
+// grid (B, Hkv), 256 threads.  Block (b, 0) records L0 in pos0[b].
+template <int DD>
+__global__ void __launch_bounds__(256) chunk_gather_kernel(ChunkArgs c)
+{
+    const AppendArgs &ap = c.app;
+    const int b = blockIdx.x, g = blockIdx.y, tid = threadIdx.x;
+    const int w = ap.w, n = ap.n, Hkv = ap.Hkv;
+    const int NW = c.pf.NW, NT = c.pf.NT;
+    int L0 = __ldcg(ap.seq_lens + b);
+    if (L0 < 0 || (long long)L0 + n - w > (long long)ap.maxp * kPage) {
+        if (tid == 0 && g == 0)
+            report(ap.status, DAR_ERR_CAPACITY);
+        L0 = max(0, min(L0, ap.maxp * kPage + w - n));
+    }
+    if (g == 0 && tid == 0)
+        c.pos0[b] = L0;
+    const int kb0 = max(0, L0 - w + 1) / BN * BN, kt0 = max(0, L0 - w) / BN * BN;
+    const int loc_lo = max(0, L0 - w + 1);
+    const size_t bg = (size_t)b * Hkv + g;
+    const bf16 *ring_k = static_cast<const bf16 *>(c.win_k) + bg * w * 64;
+    const bf16 *ring_v = static_cast<const bf16 *>(c.win_v) + bg * w * 64;
+    const bf16 *new_k = static_cast<const bf16 *>(ap.k_new) + bg * n * 64;
+    const bf16 *new_v = static_cast<const bf16 *>(ap.v_new) + bg * n * 64;
+    // full-d row of position p (ring or chunk); nullptr when neither holds it
+    auto row_of = [&](int p, bool v) -> const bf16 * {
+        if (p >= max(0, L0 - w) && p < L0)
+            return (v ? ring_v : ring_k) + (size_t)(p % w) * 64;
+        if (p >= L0 && p < L0 + n)
+            return (v ? new_v : new_k) + (size_t)(p - L0) * 64;
+        return nullptr;
+    };
+    // ---- window rows, 16 bytes at a time
+    uint4 *kw = reinterpret_cast<uint4 *>(static_cast<bf16 *>(c.kw) + bg * NW * 64);
+    uint4 *vw = reinterpret_cast<uint4 *>(static_cast<bf16 *>(c.vw) + bg * NW * 64);
+    for (int i = tid; i < NW * 8; i += blockDim.x) {
+        const int p = kb0 + i / 8, ch = i % 8;
+        uint4 k4 = make_uint4(0u, 0u, 0u, 0u), v4 = k4;
+        if (p >= loc_lo && p < L0 + n) {
+            k4 = reinterpret_cast<const uint4 *>(row_of(p, false))[ch];
+            v4 = reinterpret_cast<const uint4 *>(row_of(p, true))[ch];
+        }
+        kw[i] = k4;
+        vw[i] = v4;
+    }
+    // ---- tail rows, one element per thread and tensor
+    bf16 *kdt = static_cast<bf16 *>(c.kdt) + bg * NT * DD;
+    bf16 *vdt = static_cast<bf16 *>(c.vdt) + bg * NT * DD;
+    const bf16 *pk = static_cast<const bf16 *>(ap.pool_kd);
+    const bf16 *pv = static_cast<const bf16 *>(ap.pool_vd);
+    for (int i = tid; i < NT * DD; i += blockDim.x) {
+        const int r = i / DD, col = i % DD, p = kt0 + r;
+        bf16 kx = __float2bfloat16_rn(0.f), vx = kx;
+        if (p < L0 - w) {  // migrated before this call: its page
+            int pid = ap.block_table[(size_t)b * ap.maxp + p / kPage];
+            if (pid >= 0 && pid < ap.num_pages) {
+                const size_t off = (((size_t)pid * Hkv + g) * kPage + p % kPage) * DD + col;
+                kx = pk[off];
+                vx = pv[off];
+            } else {
+                report(ap.status, DAR_ERR_CAPACITY);
+            }
+        } else if (p < L0 + n - w) {  // leaves the window in this chunk: Eq. 1
+            const bf16 *xk = row_of(p, false), *xv = row_of(p, true);
+            const float *Wk = ap.Dk + (size_t)g * 64 * DD + col, *Wv = ap.Dv + (size_t)g * 64 * DD + col;
+            float ak = 0.0f, av = 0.0f;  // the fp32 chain over t = 0..63 of the cache append
+            for (int t = 0; t < 64; ++t) {
+                ak = __fmaf_rn(__bfloat162float(xk[t]), __ldg(Wk + (size_t)t * DD), ak);
+                av = __fmaf_rn(__bfloat162float(xv[t]), __ldg(Wv + (size_t)t * DD), av);
+            }
+            kx = __float2bfloat16_rn(ak);
+            vx = __float2bfloat16_rn(av);
+        }
+        kdt[i] = kx;
+        vdt[i] = vx;
+    }
+}
+
+template <int DP>
+static cudaError_t launch_chunk_dp(const ChunkArgs &c, cudaStream_t s)
+{
+    const PrefillArgs &a = c.pf;
+    chunk_gather_kernel<DP><<<dim3(a.B, a.Hkv), 256, 0, s>>>(c);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return e;
+    CUtensorMap m[7];
+    const unsigned long long rq = (unsigned long long)a.B * a.Hq * a.n;
+    const unsigned long long rw = (unsigned long long)a.B * a.Hkv * a.NW, rt = (unsigned long long)a.B * a.Hkv * a.NT;
+    const unsigned long long rp = (unsigned long long)(a.num_pages > 0 ? a.num_pages : 1) * a.Hkv * kPage;
+    if (!make_map(&m[0], a.q, rq, 64, BM, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m[1], c.kw, rw, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m[2], c.vw, rw, 64, BN, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !make_map(&m[3], c.kdt, rt, DP, BN, dp_map_swizzle(DP)) ||
+        !make_map(&m[4], c.vdt, rt, DP, BN, dp_map_swizzle(DP)) ||
+        !make_map(&m[5], a.pool_kd, rp, DP, BN, dp_map_swizzle(DP)) ||
+        !make_map(&m[6], a.pool_vd, rp, DP, BN, dp_map_swizzle(DP)))
+        return cudaErrorInvalidValue;
+    e = launch_kernel<DP, true>(m, a, a.n, s);
+    if (e != cudaSuccess)
+        return e;
+    // the chunk joins the cache last: its ring slots and migrated pages
+    return launch_cache_append(DAR_BF16, DP, c.app, s);
 }
 
 }  // namespace tcp
@@ -740,6 +899,18 @@ bool make_tma_2d_bf16(CUtensorMap *map, const void *base, unsigned long long row
                                   : cols == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
                                                : CU_TENSOR_MAP_SWIZZLE_128B;
     return tcp::make_map(map, base, rows, cols, box_rows, sw);
+}
+
+cudaError_t launch_prefill_chunk(int dd, const ChunkArgs &c, cudaStream_t s)
+{
+    if (c.pf.B == 0 || c.pf.n == 0)
+        return cudaSuccess;
+    switch (dd) {
+    case 16: return tcp::launch_chunk_dp<16>(c, s);
+    case 32: return tcp::launch_chunk_dp<32>(c, s);
+    case 64: return tcp::launch_chunk_dp<64>(c, s);
+    default: return cudaErrorInvalidValue;
+    }
 }
 
 cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s)

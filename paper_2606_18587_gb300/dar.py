@@ -66,6 +66,8 @@ def load_library(path: str = LIB_PATH):
         "dar_decode_step": ([CP, P, P, I32, P, P, P, I32, P, P, P, F, P, P, SZ, P], ctypes.c_int),
         "dar_check_bounded_wait": ([P, ctypes.c_uint32, P], ctypes.c_int),
         "dar_prefill_workspace_bytes": ([ctypes.c_int, I32, I32, I32, I32], SZ),
+        "dar_prefill_chunk_workspace_bytes": ([CP, I32], SZ),
+        "dar_prefill_chunk": ([CP, I32, I32, P, P, P, P, P, P, P, F, P, P, SZ, P], ctypes.c_int),
         "dar_attn_prefill": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, P, P,
                               SZ, P, P], ctypes.c_int),
         "dar_last_error": ([], ctypes.c_char_p),
@@ -292,4 +294,32 @@ def dar_attn_prefill(q, k, v, Dk, Uk, Dv, Uv, w, scale=0.0, out=None, workspace=
     _check(load_library().dar_attn_prefill(
         _code(q), B, Hq, Hkv, N, d, dd, int(w), _ptr(q), _ptr(k), _ptr(v), _ptr(Dk), _ptr(Uk), _ptr(Dv), _ptr(Uv),
         float(scale), _ptr(out), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+    return out
+
+
+def dar_prefill_chunk_workspace_bytes(cache: DarCache, n: int) -> int:
+    return int(load_library().dar_prefill_chunk_workspace_bytes(cache.struct, int(n)))
+
+
+def dar_prefill_chunk(cache: DarCache, q, k_new, v_new, Dk, Uk, Dv, Uv, scale=0.0, out=None, workspace=None,
+                      stream=None):
+    """Chunked prefill over the cache: queries ``q [B,Hq,n,d]`` at positions
+    ``seq_lens[b] ..`` attend to the cache and causally within the chunk;
+    ``k_new, v_new [B,Hkv,n,d]`` are then appended.  Returns ``[B,Hq,n,d]``."""
+    _dev(q, "q", cache.dtype)
+    _dev(k_new, "k_new", cache.dtype)
+    _dev(v_new, "v_new", cache.dtype)
+    for name, t in (("Dk", Dk), ("Uk", Uk), ("Dv", Dv), ("Uv", Uv)):
+        _dev(t, name, torch.float32)
+    B, Hq, n, d = q.shape
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", cache.dtype)
+    if workspace is None:
+        workspace = torch.empty(max(1, dar_prefill_chunk_workspace_bytes(cache, n)), dtype=torch.uint8,
+                                device=q.device)
+    _dev(workspace, "workspace")
+    _check(load_library().dar_prefill_chunk(
+        cache.struct, Hq, n, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(Dk), _ptr(Uk), _ptr(Dv), _ptr(Uv),
+        float(scale), _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
     return out
