@@ -26,16 +26,16 @@
 // (x = s * scale * log2(e) - m), one conversion of the pair to bf16x2 and one
 // bf16x2 exp2, whose result is the packed bf16 P the PV product reads.
 //
-// Warp roles (224 threads): warp 0 issues TMA loads, warp 6 issues the S
-// products (and q~), warp 1 allocates TMEM and issues the PV products (one
-// thread each), warps 2-5 own one query row per thread (TMEM lane = row) for
-// the softmax and the epilogue.  The softmax releases an S buffer as soon as
-// it has loaded it (so S(t + NSB) is computed while it works on tile t) and
-// writes P into TMEM, where the PV products take it as their A operand.  The
-// issuing threads build their shared-memory descriptors once and only add
-// offsets per tile.  Two CTAs share an SM (256 TMEM columns and ~110 KB of
-// shared memory each), so one CTA's softmax overlaps the other's waits.  Every
-// wait is bounded; on a timeout the CTA flags *status and exits.
+// Warp roles (224 threads): warp 0 issues TMA loads, warp 6 the S products
+// (and q~), warp 1 allocates TMEM and issues the PV products (each issuing
+// warp runs its loop together; one elected lane issues), warps 2-5 own one
+// query row per thread (TMEM lane = row) for the softmax and the epilogue.
+// The softmax writes P into TMEM over the S it came from, where the PV
+// products take it as their A operand; with two, later three, S buffers the
+// S products run ahead of the softmax and only wait for the PV that last read
+// a buffer.  Two CTAs share an SM (256 TMEM columns and ~110 KB of shared
+// memory each), so one CTA's softmax overlaps the other's waits.  Every wait
+// is bounded; on a timeout the CTA flags *status and exits.
 #include <cuda.h>
 
 #include "dar_common.cuh"
@@ -83,23 +83,24 @@ __host__ __device__ constexpr Swizzle vd_swizzle()
 }
 
 // Tensor-memory columns of one CTA (256 of the SM's 512, two CTAs per SM):
-// S (fp32, BN columns; the softmax releases it as soon as it has loaded it,
-// and the S issuer, a thread of its own, computes S(t + 1) into it while tile
-// t's softmax runs), O_loc (64), O_glob (DP), the row sum (16 identical
-// columns) and P (bf16 pairs, BN / 2 columns; the A operand of the PV
-// products), in two buffers when they fit, so the softmax writes P(t + 1)
-// while PV(t) still reads P(t).  q~ passes through the O_loc columns before
-// the accumulators are cleared.
+// S buffers (fp32, BN columns each), O_loc (64), O_glob (DP) and the row sum
+// (16 identical columns).
+//  - d_down <= 32: two S buffers.  The softmax writes P(t) (bf16 pairs, BN / 2
+//    columns; the A operand of the PV products) over the first half of the S
+//    buffer it came from, and S(t + 2) goes into that buffer once PV(t) has
+//    read P(t), so the S products run a tile ahead of the softmax.
+//  - d_down = 64: one S buffer, released as soon as the softmax has loaded it,
+//    and P in 32 columns of its own.
+// q~ passes through the O_loc columns before the accumulators are cleared.
 template <int DP>
 struct Tmem {
-    static constexpr int NSB = 1;
-    static constexpr uint32_t S = 0;  // buffer b at S + b * BN
-    static constexpr uint32_t OL = NSB * BN;
+    static constexpr bool kAlias = 2 * BN + 64 + DP + 16 <= (int)kTmemCols;
+    static constexpr uint32_t S = 0;                      // buffer b at S + b * BN
+    static constexpr uint32_t OL = kAlias ? 2 * BN : BN;
     static constexpr uint32_t OG = OL + 64;
     static constexpr uint32_t SUM = OG + DP;
-    static constexpr uint32_t P = SUM + 16;  // buffer b at P + b * BN / 2
-    static constexpr int NPB = P + BN <= kTmemCols ? 2 : 1;
-    static_assert(P + NPB * BN / 2 <= kTmemCols, "tensor-memory columns overflow");
+    static constexpr uint32_t P = kAlias ? S : SUM + 16;  // alias: P of buffer b at S + b * BN
+    static_assert(SUM + 16 <= kTmemCols && (kAlias || P + BN / 2 <= kTmemCols), "tensor-memory columns overflow");
 };
 
 // Shared-memory layout (offsets from a 1024-byte aligned base).  A stage holds
@@ -207,12 +208,25 @@ __device__ __forceinline__ VTile vt_next(VTile v, int i0, int i_last, int w)
     return VTile{kt, k.loc, k.loc && k.glob};
 }
 
-__device__ __forceinline__ int vt_count(int i0, int i_last, int w)
+// Number of virtual tiles of query rows i0 .. i_last.  Key tile kt has local
+// pairs iff kt >= kt_loc_lo (w >= 1) and global pairs iff kt <= kt_glob_hi.
+__device__ __forceinline__ int vt_total(int i0, int i_last, int w)
 {
-    int n = 0;
-    for (VTile v = vt_first(i0, i_last, w); v.kt >= 0; v = vt_next(v, i0, i_last, w))
-        ++n;
-    return n;
+    const int kt_glob_hi = i_last >= w ? (i_last - w) / BN : -1;
+    if (w <= 0)
+        return kt_glob_hi + 1;
+    const int a = i0 - BN + 2 - w;  // local iff kt * BN >= a
+    const int kt_loc_lo = a > 0 ? (a + BN - 1) / BN : 0;
+    return i_last / BN - kt_loc_lo + 1 + kt_glob_hi + 1;
+}
+
+// S buffer b of virtual tile t and u = the number of earlier tiles that used
+// it (the phase of that buffer's barriers).
+template <bool ALIAS>
+__device__ __forceinline__ void buf_of(int t, int &b, int &u)
+{
+    b = ALIAS ? t & 1 : 0;
+    u = ALIAS ? t >> 1 : t;
 }
 
 // CH = false: the causal forward over positions 0..N-1 of q, k, v.  CH = true:
@@ -229,23 +243,23 @@ __global__ void __launch_bounds__(kThreads, 2)
 {
     using Ly = Layout<DP>;
     using Tm = Tmem<DP>;
+    constexpr bool ALIAS = Tm::kAlias;
     constexpr int NS = Ly::NS;
-    constexpr int NPB = Tm::NPB;
-    constexpr int NSB = Tm::NSB;
+    constexpr int NB = ALIAS ? 2 : 1;  // S buffers
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + Ly::BAR);
-    uint64_t *full = bars;                 // [NS] TMA -> MMA
-    uint64_t *empty = bars + NS;           // [NS] MMA -> TMA
-    uint64_t *s_full = bars + 2 * NS;      // [NSB] S of a virtual tile computed into buffer b
-    uint64_t *s_free = s_full + NSB;       // [NSB] S buffer b loaded by the softmax (one arrival per softmax warp)
-    uint64_t *p_full = s_free + NSB;       // [NPB] P written to TMEM buffer b (one arrival per softmax warp)
-    uint64_t *pv_done = p_full + NPB;      // [NPB] PV (and row sums) reading P buffer b finished
-    uint64_t *q_full = pv_done + NPB;      // Q landed
-    uint64_t *ukb_ready = q_full + 1;      // Uk (bf16) and the ones block written (every softmax thread)
-    uint64_t *qt_mma = q_full + 2;         // q~ = Q Uk^T computed into TMEM
-    uint64_t *qt_ready = q_full + 3;       // q~ in shared memory, accumulators zeroed (every softmax thread)
+    uint64_t *full = bars;              // [NS] TMA -> MMA
+    uint64_t *empty = bars + NS;        // [NS] last reader (the PV product) -> TMA
+    uint64_t *s_full = bars + 2 * NS;   // [NB] S computed into buffer b
+    uint64_t *p_full = s_full + NB;     // [NB] P of buffer b written (one arrival per softmax warp)
+    uint64_t *pv_done = p_full + NB;    // [NB] PV reading P of buffer b finished
+    uint64_t *s_free = pv_done + NB;    // single buffer: S loaded by the softmax (one arrival per softmax warp)
+    uint64_t *q_full = s_free + 1;      // Q landed
+    uint64_t *ukb_ready = q_full + 1;   // Uk (bf16) and the ones block written (every softmax thread)
+    uint64_t *qt_mma = q_full + 2;      // q~ = Q Uk^T computed into TMEM
+    uint64_t *qt_ready = q_full + 3;    // q~ in shared memory, accumulators zeroed (every softmax thread)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(q_full + 4);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -261,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int nqt = (nrows + BM - 1) / BM;
     const int qt = nqt - 1 - (int)blockIdx.y;  // longest rows first
     const int i0 = L0 + qt * BM, i_last = min(i0 + BM, N) - 1;
-    const int VT = vt_count(i0, i_last, w);
+    const int VT = vt_total(i0, i_last, w);
     // chunk mode: first positions of the window and tail buffers
     const int kb0 = CH ? max(0, L0 - w + 1) / BN * BN : 0;
     const int kt0 = CH ? max(0, L0 - w) / BN * BN : 0;
@@ -269,16 +283,16 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (threadIdx.x == 0) {
         for (int s = 0; s < NS; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], 2);  // the S and the PV issuer both release a stage
+            // released by the PV commit alone: PV(t) follows P(t), which follows
+            // the completion of S(t), so K and V have both been read by then
+            mbar_init(&empty[s], 1);
         }
-        for (int b2 = 0; b2 < NSB; ++b2) {
+        for (int b2 = 0; b2 < NB; ++b2) {
             mbar_init(&s_full[b2], 1);
-            mbar_init(&s_free[b2], kSoftmaxWarps);
-        }
-        for (int b2 = 0; b2 < NPB; ++b2) {
             mbar_init(&p_full[b2], kSoftmaxWarps);
             mbar_init(&pv_done[b2], 1);
         }
+        mbar_init(s_free, kSoftmaxWarps);
         mbar_init(q_full, 1);
         mbar_init(ukb_ready, kSoftmaxThreads);
         mbar_init(qt_mma, 1);
@@ -342,16 +356,20 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     } else if (warp == kWarpS || warp == kWarpPV) {
         // ------------------------------------------------------------ MMA issuers
-        // Two threads in two warps: S products (and q~) from one, PV products
-        // from the other.  A tensor-core instruction costs a thread ~50-150
-        // cycles to issue, independently of other issuing threads, so splitting
-        // the two streams lets each keep up with the softmax.  They write
-        // disjoint TMEM columns; each commit covers its own thread's products,
-        // and a stage is free once both have committed (empty[s] counts 2).
+        // Two warps: S products (and q~) from one, PV products from the other.
+        // Each warp runs its loop together and one elected lane issues the
+        // products and their commits, so descriptors and TMEM addresses stay
+        // warp-uniform.  They write disjoint TMEM columns; each commit covers
+        // the products of its tile, and the PV commit also frees the tile's
+        // stage.
         constexpr uint64_t kStageStep = Ly::STAGE >> 4;
         const uint64_t dStg = smem_desc(smem_u32(sm + Ly::STG), 16, 1024, kSw128);  // stage 0, K / V tile
+        auto wait_all = [&](uint64_t *bar, unsigned parity) {
+            const bool r = mbar_wait(bar, parity, abort_flag);
+            return __all_sync(0xffffffffu, r) != 0;
+        };
         bool ok = true;
-        if (lane == 0 && warp == kWarpS) {
+        if (warp == kWarpS) {
             constexpr uint32_t idS = idesc_bf16(BM, BN, false);
             constexpr uint32_t idQT = idesc_bf16(BM, DP, false);
             // Shared-memory descriptors, built once: a k-step of 16 elements adds
@@ -362,42 +380,62 @@ __global__ void __launch_bounds__(kThreads, 2)
             const uint64_t dStgD = smem_desc(smem_u32(sm + Ly::STG), 16, 8 * DP * 2, dp_swizzle<DP>());
             const uint32_t tS = tmem + Tm::S, tOL = tmem + Tm::OL;
             // q~ = Q Uk^T into the O_loc columns
-            ok = mbar_wait(q_full, 0, abort_flag) && mbar_wait(ukb_ready, 0, abort_flag);
+            ok = wait_all(q_full, 0) && wait_all(ukb_ready, 0);
             if (ok) {
                 tc_fence_after();
+                if (elect_one()) {
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk)
-                    mma_f16_ss(tOL, dQ + 2 * kk, dUKB + 2 * kk, idQT, kk > 0);
-                mma_commit(qt_mma);
-                ok = mbar_wait(qt_ready, 0, abort_flag);
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_f16_ss(tOL, dQ + 2 * kk, dUKB + 2 * kk, idQT, kk > 0);
+                    mma_commit(qt_mma);
+                }
+                __syncwarp();
+                ok = wait_all(qt_ready, 0);
                 tc_fence_after();
             }
-            // S(t) into buffer t % NSB once the buffer's previous S has been loaded
-            VTile vt = vt_first(i0, i_last, w);
-            for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
-                const int s = t % NS, sb = t % NSB;
-                if (!mbar_wait(&full[s], (t / NS) & 1, abort_flag) ||
-                    (t >= NSB && !mbar_wait(&s_free[sb], ((t / NSB) - 1) & 1, abort_flag))) {
+            // S(t) into buffer b once that buffer is free: PV(t - 2) has read the
+            // P written over it (two buffers), or the softmax has loaded S(t - 1)
+            // (one buffer)
+            // the next tile's key tile, S buffer and stage are computed at the top
+            // of each iteration, off the critical path
+            VTile nvt = vt_first(i0, i_last, w);
+            int nsb, nu, s = 0, sph = 0;
+            buf_of<ALIAS>(0, nsb, nu);
+            for (int t = 0; ok && t < VT; ++t) {
+                const VTile vt = nvt;
+                const int sb = nsb, u = nu;
+                nvt = vt_next(vt, i0, i_last, w);
+                buf_of<ALIAS>(t + 1, nsb, nu);
+                bool fine = wait_all(&full[s], sph);
+                if (fine && u > 0)
+                    fine = wait_all(ALIAS ? &pv_done[sb] : s_free, (u - 1) & 1);
+                if (!fine) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 const uint32_t tSb = tS + sb * BN;
-                if (vt.loc) {
-                    const uint64_t dK = dStg + s * kStageStep;
+                if (elect_one()) {
+                    if (vt.loc) {
+                        const uint64_t dK = dStg + s * kStageStep;
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        mma_f16_ss(tSb, dQ + 2 * kk, dK + 2 * kk, idS, kk > 0);
-                } else {
-                    const uint64_t dKD = dStgD + s * kStageStep;
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_f16_ss(tSb, dQ + 2 * kk, dK + 2 * kk, idS, kk > 0);
+                    } else {
+                        const uint64_t dKD = dStgD + s * kStageStep;
 #pragma unroll
-                    for (int kk = 0; kk < DP / 16; ++kk)
-                        mma_f16_ss(tSb, dQT + 2 * kk, dKD + 2 * kk, idS, kk > 0);
+                        for (int kk = 0; kk < DP / 16; ++kk)
+                            mma_f16_ss(tSb, dQT + 2 * kk, dKD + 2 * kk, idS, kk > 0);
+                    }
+                    mma_commit(&s_full[sb]);
                 }
-                mma_commit(&s_full[sb]);
-                mma_commit(&empty[s]);
+                __syncwarp();
+                if (++s == NS) {
+                    s = 0;
+                    sph ^= 1;
+                }
             }
-        } else if (lane == 0 && warp == kWarpPV) {
+        } else {
             constexpr uint32_t idPV = idesc_bf16(BM, 64, true);
             // global PV: N = DP + 16 when v^D rows carry the ones (O_glob, then the row sums)
             constexpr uint32_t idPVg = idesc_bf16(BM, kOnes ? DP + 16 : DP, true);
@@ -409,36 +447,48 @@ __global__ void __launch_bounds__(kThreads, 2)
             constexpr uint64_t kVStep = (16 * 128) >> 4, kVDStep = (16 * VR * 2) >> 4;
             // all-ones B operand (16 columns x 16 keys per k-step; every byte pair is 1.0)
             const uint64_t ones_desc = smem_desc(smem_u32(sm + Ly::ONES), 128, 256, kSwNone);
-            const uint32_t tOL = tmem + Tm::OL, tOG = tmem + Tm::OG, tSum = tmem + Tm::SUM, tP = tmem + Tm::P;
-            VTile vt = vt_first(i0, i_last, w);
-            for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
-                const int s = t % NS, pb = t % NPB;
-                if (!mbar_wait(&p_full[pb], (t / NPB) & 1, abort_flag)) {
+            const uint32_t tOL = tmem + Tm::OL, tOG = tmem + Tm::OG, tSum = tmem + Tm::SUM;
+            VTile nvt = vt_first(i0, i_last, w);
+            int npb, nu, s = 0;
+            buf_of<ALIAS>(0, npb, nu);
+            for (int t = 0; ok && t < VT; ++t) {
+                const VTile vt = nvt;
+                const int pb = npb, u = nu;
+                nvt = vt_next(vt, i0, i_last, w);
+                buf_of<ALIAS>(t + 1, npb, nu);
+                if (!wait_all(&p_full[pb], u & 1)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t aP = tP + pb * (BN / 2);
-                if (vt.loc) {
-                    const uint64_t dV = dStg + s * kStageStep + kVOff;
+                const uint32_t aP = tmem + Tm::P + (ALIAS ? pb * BN : 0);
+                if (elect_one()) {
+                    if (vt.loc) {
+                        const uint64_t dV = dStg + s * kStageStep + kVOff;
 #pragma unroll
-                    for (int kk = 0; kk < BN / 16; ++kk) {  // P (TMEM, 8 columns per 16 keys) times V
-                        mma_f16_ts(tOL, aP + kk * 8, dV + kk * kVStep, idPV, true);
-                        mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);  // row sums of P
-                    }
-                } else {
-                    const uint64_t dVD = dStgVD + s * kStageStep + kVDOff;
+                        for (int kk = 0; kk < BN / 16; ++kk) {  // P (TMEM, 8 columns per 16 keys) times V
+                            mma_f16_ts(tOL, aP + kk * 8, dV + kk * kVStep, idPV, true);
+                            mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);  // row sums of P
+                        }
+                    } else {
+                        const uint64_t dVD = dStgVD + s * kStageStep + kVDOff;
 #pragma unroll
-                    for (int kk = 0; kk < BN / 16; ++kk) {  // P times [V^D | ones]
-                        mma_f16_ts(tOG, aP + kk * 8, dVD + kk * kVDStep, idPVg, true);
-                        if constexpr (!kOnes)
-                            mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);
+                        for (int kk = 0; kk < BN / 16; ++kk) {  // P times [V^D | ones]
+                            mma_f16_ts(tOG, aP + kk * 8, dVD + kk * kVDStep, idPVg, true);
+                            if constexpr (!kOnes)
+                                mma_f16_ts(tSum, aP + kk * 8, ones_desc, idSum, true);
+                        }
                     }
+                    mma_commit(&pv_done[pb]);
+                    mma_commit(&empty[s]);
                 }
-                mma_commit(&pv_done[pb]);
-                mma_commit(&empty[s]);
+                __syncwarp();
+                if (++s == NS)
+                    s = 0;
             }
         }
+        if (!ok)
+            *abort_flag = 1;
     } else {  // warps 2 .. 2 + kSoftmaxWarps - 1
         // ------------------------------------------------------------ softmax warps
         // one query row per thread: warp w reads TMEM lanes 32 (w % 4) .. + 31
@@ -515,27 +565,37 @@ __global__ void __launch_bounds__(kThreads, 2)
 
         const float c2 = a.qscale;  // softmax scale * log2(e)
         float m_used = -INFINITY;
-        // highest PV(t') observed complete, per P buffer (t' even / odd)
-        int pv_seen0 = -NPB, pv_seen1 = 1 - NPB;
-        // wait until PV(u) (and so every tensor-core op issued before it) has completed
-        auto wait_pv = [&](int u) -> bool {
-            const bool odd = NPB == 2 && (u & 1);
-            if (u < 0 || (odd ? pv_seen1 : pv_seen0) >= u)
+        // last tile whose PV this thread has seen complete, per S buffer
+        int pv_seen0 = -1, pv_seen1 = -1;
+        // wait until PV(v) (its own products) has completed
+        auto wait_pv = [&](int v) -> bool {
+            if (v < 0)
                 return true;
-            if (!wait_uniform(&pv_done[odd ? 1 : 0], (u / NPB) & 1))
+            int pb, u;
+            buf_of<ALIAS>(v, pb, u);
+            const int seen = pb == 0 ? pv_seen0 : pv_seen1;
+            if (seen >= v)
+                return true;
+            if (!wait_uniform(&pv_done[pb], u & 1))
                 return false;
-            if (odd)
-                pv_seen1 = u;
+            if (pb == 0)
+                pv_seen0 = v;
             else
-                pv_seen0 = u;
+                pv_seen1 = v;
             tc_fence_after();
             return true;
         };
-        VTile vt = vt_first(i0, i_last, w);
-        for (int t = 0; ok && t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
+        VTile nvt = vt_first(i0, i_last, w);
+        int nsb, nu;
+        buf_of<ALIAS>(0, nsb, nu);
+        for (int t = 0; ok && t < VT; ++t) {
+            // this tile's parameters, and the next one's computed now, off the critical path
+            const VTile vt = nvt;
+            const int sb = nsb, u = nu;
+            nvt = vt_next(vt, i0, i_last, w);
+            buf_of<ALIAS>(t + 1, nsb, nu);
             const int j0 = vt.kt * BN;
-            const int sb = t % NSB;
-            if (!wait_uniform(&s_full[sb], (t / NSB) & 1)) {
+            if (!wait_uniform(&s_full[sb], u & 1)) {
                 ok = false;
                 break;
             }
@@ -548,15 +608,16 @@ __global__ void __launch_bounds__(kThreads, 2)
                 for (int e = 0; e < BN; ++e)
                     s[e] = __uint_as_float(r[e]);
             }
-            // this S buffer may be overwritten now (S(t + NSB))
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(&s_free[sb]);
+            if constexpr (!ALIAS) {  // the S buffer may be overwritten now (S(t + 1))
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(s_free);
+            }
 
             // masks: causal (tiles reaching past row i0), the other part of a
             // band tile, rows past the end; the kept columns form one range
-            if (j0 + BN - 1 > i0 || vt.band || i0 + BM > N) {
+            if (__builtin_expect(j0 + BN - 1 > i0 || vt.band || i0 + BM > N, 0)) {
                 int e_hi = i < N ? i - j0 : -1, e_lo = 0;
                 if (vt.band) {
                     if (vt.loc)
@@ -564,9 +625,17 @@ __global__ void __launch_bounds__(kThreads, 2)
                     else
                         e_hi = min(e_hi, i - w - j0);
                 }
+                // one bound at a time, each only where some row of the warp needs it
+                if (__any_sync(0xffffffffu, e_lo > 0)) {
 #pragma unroll
-                for (int e = 0; e < BN; ++e)
-                    s[e] = (e >= e_lo && e <= e_hi) ? s[e] : -INFINITY;
+                    for (int e = 0; e < BN; ++e)
+                        s[e] = e >= e_lo ? s[e] : -INFINITY;
+                }
+                if (__any_sync(0xffffffffu, e_hi < BN - 1)) {
+#pragma unroll
+                    for (int e = 0; e < BN; ++e)
+                        s[e] = e <= e_hi ? s[e] : -INFINITY;
+                }
             }
             const float mt = tree_max3(s) * c2;
             // raise the running max only when it grows by more than the threshold
@@ -585,10 +654,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                 ffma2(x0, x1, s[e], s[e + 1], c2, c2, mneg, mneg);
                 pk[e / 2] = ex2_bf16x2(cvt_bf16x2(x0, x1));
             }
-            if (__any_sync(0xffffffffu, scale_o)) {
-                // every earlier PV must have landed before O is rescaled (and PV(t),
+            if (__builtin_expect(__any_sync(0xffffffffu, scale_o), 0)) {
+                // every earlier PV must have landed before O is rescaled (PV(t),
                 // which needs P(t), cannot start before it is)
-                if (!wait_pv(t - 1)) {
+                if (!wait_pv(t - 1) || !wait_pv(t - 2)) {
                     ok = false;
                     break;
                 }
@@ -611,22 +680,23 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tmem_st16(tl + Tm::OG + c, r);
                 }
             }
-            // the PV that last read this P buffer (tile t - NPB) must be done with it
-            if (!wait_pv(t - NPB)) {
+            // one buffer: PV(t - 1) must be done with the P buffer (two buffers:
+            // P goes over S(t), whose buffer was free before S(t) was computed)
+            if (!ALIAS && !wait_pv(t - 1)) {
                 ok = false;
                 break;
             }
-            const int pb = t % NPB;
-            tmem_st32(tl + Tm::P + pb * (BN / 2), pk);
+            tmem_st32(tl + Tm::P + (ALIAS ? sb * BN : 0), pk);
             tmem_wait_st();
             tc_fence_before();
             __syncwarp();
             if (lane == 0)
-                mbar_arrive(&p_full[pb]);
+                mbar_arrive(&p_full[sb]);
         }
 
-        // ---- epilogue: o = (O_loc + O_glob Uv) / l
-        if (ok && wait_pv(VT - 1)) {
+        // ---- epilogue: o = (O_loc + O_glob Uv) / l (the last products may
+        // still be running on either buffer)
+        if (ok && wait_pv(VT - 1) && wait_pv(VT - 2)) {
             const float *sUv = reinterpret_cast<const float *>(sm + Ly::UV);
             float og[DP];
             float l;
@@ -646,22 +716,24 @@ __global__ void __launch_bounds__(kThreads, 2)
             bf16 *orow = static_cast<bf16 *>(a.out) + (((size_t)b * a.Hq + h) * nrows + (i - L0)) * 64;
 #pragma unroll
             for (int c = 0; c < 64; c += 16) {
-                uint32_t r[16];
-                tmem_ld16(tl + Tm::OL + c, r);
                 float o[16];
+                {
+                    uint32_t r[16];
+                    tmem_ld16(tl + Tm::OL + c, r);
 #pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    o[e] = __uint_as_float(r[e]);
+                    for (int e = 0; e < 16; ++e)
+                        o[e] = __uint_as_float(r[e]);
+                }
 #pragma unroll
                 for (int kk = 0; kk < DP; ++kk) {
                     const float4 *u4 = reinterpret_cast<const float4 *>(sUv + kk * 64 + c);
 #pragma unroll
                     for (int e4 = 0; e4 < 4; ++e4) {
-                        const float4 u = u4[e4];
-                        o[4 * e4 + 0] = fmaf(og[kk], u.x, o[4 * e4 + 0]);
-                        o[4 * e4 + 1] = fmaf(og[kk], u.y, o[4 * e4 + 1]);
-                        o[4 * e4 + 2] = fmaf(og[kk], u.z, o[4 * e4 + 2]);
-                        o[4 * e4 + 3] = fmaf(og[kk], u.w, o[4 * e4 + 3]);
+                        const float4 uu = u4[e4];
+                        o[4 * e4 + 0] = fmaf(og[kk], uu.x, o[4 * e4 + 0]);
+                        o[4 * e4 + 1] = fmaf(og[kk], uu.y, o[4 * e4 + 1]);
+                        o[4 * e4 + 2] = fmaf(og[kk], uu.z, o[4 * e4 + 2]);
+                        o[4 * e4 + 3] = fmaf(og[kk], uu.w, o[4 * e4 + 3]);
                     }
                 }
 #pragma unroll

@@ -300,6 +300,20 @@ __device__ __forceinline__ void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uin
 
 // Arrive once on the mbarrier when every tcgen05 operation issued so far by
 // this thread has completed.
+// True in exactly one lane of a fully active warp.  A warp that runs its
+// issue loop together and issues tcgen05.mma / commit under this predicate
+// keeps the operands (descriptors, TMEM addresses) warp-uniform, so they are
+// handed to the tensor core without a per-thread serialising loop: about half
+// the issue cost of a lone divergent thread (measured, M128 N32 from TMEM).
+__device__ __forceinline__ bool elect_one()
+{
+    uint32_t p;
+    asm volatile(
+        "{\n\t.reg .pred P;\n\telect.sync _|P, 0xffffffff;\n\tselp.u32 %0, 1, 0, P;\n\t}"
+        : "=r"(p));
+    return p != 0;
+}
+
 __device__ __forceinline__ void mma_commit(uint64_t *bar)
 {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
