@@ -125,19 +125,6 @@ struct Layout {
     static_assert(VD_OFF + BN * vd_row<DP>() * 2 <= STAGE, "a stage holds either part");
 };
 
-struct TileKind {
-    bool loc, glob;
-};
-
-__device__ __forceinline__ TileKind tile_kind(int i0, int i_last, int j0, int w)
-{
-    const int min_d = i0 - (j0 + BN - 1), max_d = i_last - j0;
-    TileKind k;
-    k.glob = max_d >= w;
-    k.loc = max(min_d, 0) <= min(max_d, w - 1);
-    return k;
-}
-
 __device__ __forceinline__ float max3(float a, float b, float c)
 {
     float d;
@@ -190,35 +177,38 @@ struct VTile {
     bool band; // the key tile also has the other part
 };
 
-__device__ __forceinline__ VTile vt_first(int i0, int i_last, int w)
-{
-    const int kt = i_last / BN;
-    const TileKind k = tile_kind(i0, i_last, kt * BN, w);
-    return VTile{kt, k.loc, k.loc && k.glob};
-}
-
-__device__ __forceinline__ VTile vt_next(VTile v, int i0, int i_last, int w)
-{
-    if (v.band && v.loc)
-        return VTile{v.kt, false, true};
-    const int kt = v.kt - 1;
-    if (kt < 0)
-        return VTile{-1, false, false};
-    const TileKind k = tile_kind(i0, i_last, kt * BN, w);
-    return VTile{kt, k.loc, k.loc && k.glob};
-}
-
-// Number of virtual tiles of query rows i0 .. i_last.  Key tile kt has local
-// pairs iff kt >= kt_loc_lo (w >= 1) and global pairs iff kt <= kt_glob_hi.
-__device__ __forceinline__ int vt_total(int i0, int i_last, int w)
-{
-    const int kt_glob_hi = i_last >= w ? (i_last - w) / BN : -1;
-    if (w <= 0)
-        return kt_glob_hi + 1;
-    const int a = i0 - BN + 2 - w;  // local iff kt * BN >= a
-    const int kt_loc_lo = a > 0 ? (a + BN - 1) / BN : 0;
-    return i_last / BN - kt_loc_lo + 1 + kt_glob_hi + 1;
-}
+// The sequence of query rows i0 .. i_last in closed form (Eq. 3: pair (i, j)
+// is local iff i - j < w).  Key tile kt has local pairs iff kt >= kt_l (none
+// when w = 0) and global pairs iff kt <= kt_g, so going down from
+// kt_hi = i_last / BN: nL local-only tiles, nB band tiles (two virtual tiles
+// each), then the global-only tiles.  at(t) depends on t alone, so a loop
+// computes it without a chain through the previous tile.
+struct TileMap {
+    int kt_hi, kt_b, kt_go, nL, nLB, VT;
+    __device__ __forceinline__ TileMap(int i0, int i_last, int w)
+    {
+        kt_hi = i_last / BN;
+        const int kt_g = i_last >= w ? (i_last - w) / BN : -1;
+        int kt_l = kt_hi + 1;  // no local pairs (w = 0)
+        if (w > 0) {
+            const int a = i0 - BN + 2 - w;  // local iff kt * BN >= a
+            kt_l = a > 0 ? (a + BN - 1) / BN : 0;
+        }
+        nL = kt_hi - max(kt_g, kt_l - 1);
+        kt_b = min(kt_hi, kt_g);
+        nLB = nL + 2 * max(0, kt_b - kt_l + 1);
+        kt_go = min(kt_g, kt_l - 1);
+        VT = nLB + max(0, kt_go + 1);
+    }
+    __device__ __forceinline__ VTile at(int t) const
+    {
+        if (t < nL)
+            return VTile{kt_hi - t, true, false};
+        if (t < nLB)
+            return VTile{kt_b - ((t - nL) >> 1), ((t - nL) & 1) == 0, true};
+        return VTile{kt_go - (t - nLB), false, false};
+    }
+};
 
 // S buffer b of virtual tile t and u = the number of earlier tiles that used
 // it (the phase of that buffer's barriers).
@@ -275,7 +265,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int nqt = (nrows + BM - 1) / BM;
     const int qt = nqt - 1 - (int)blockIdx.y;  // longest rows first
     const int i0 = L0 + qt * BM, i_last = min(i0 + BM, N) - 1;
-    const int VT = vt_total(i0, i_last, w);
+    const TileMap tiles(i0, i_last, w);
+    const int VT = tiles.VT;
     // chunk mode: first positions of the window and tail buffers
     const int kb0 = CH ? max(0, L0 - w + 1) / BN * BN : 0;
     const int kt0 = CH ? max(0, L0 - w) / BN * BN : 0;
@@ -323,8 +314,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             mbar_expect_tx(q_full, BM * 64 * 2);
             tma_load_2d(sm + Ly::Q, &tmQ, 0, (b * a.Hq + h) * nrows + qt * BM, q_full);
-            VTile vt = vt_first(i0, i_last, w);
-            for (int t = 0; t < VT; ++t, vt = vt_next(vt, i0, i_last, w)) {
+            for (int t = 0; t < VT; ++t) {
+                const VTile vt = tiles.at(t);
                 const int s = t % NS;
                 if (t >= NS && !mbar_wait(&empty[s], ((t / NS) - 1) & 1, abort_flag))
                     break;
@@ -396,16 +387,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             // S(t) into buffer b once that buffer is free: PV(t - 2) has read the
             // P written over it (two buffers), or the softmax has loaded S(t - 1)
             // (one buffer)
-            // the next tile's key tile, S buffer and stage are computed at the top
-            // of each iteration, off the critical path
-            VTile nvt = vt_first(i0, i_last, w);
-            int nsb, nu, s = 0, sph = 0;
-            buf_of<ALIAS>(0, nsb, nu);
+            int s = 0, sph = 0;
             for (int t = 0; ok && t < VT; ++t) {
-                const VTile vt = nvt;
-                const int sb = nsb, u = nu;
-                nvt = vt_next(vt, i0, i_last, w);
-                buf_of<ALIAS>(t + 1, nsb, nu);
+                const VTile vt = tiles.at(t);
+                int sb, u;
+                buf_of<ALIAS>(t, sb, u);
                 bool fine = wait_all(&full[s], sph);
                 if (fine && u > 0)
                     fine = wait_all(ALIAS ? &pv_done[sb] : s_free, (u - 1) & 1);
@@ -448,14 +434,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             // all-ones B operand (16 columns x 16 keys per k-step; every byte pair is 1.0)
             const uint64_t ones_desc = smem_desc(smem_u32(sm + Ly::ONES), 128, 256, kSwNone);
             const uint32_t tOL = tmem + Tm::OL, tOG = tmem + Tm::OG, tSum = tmem + Tm::SUM;
-            VTile nvt = vt_first(i0, i_last, w);
-            int npb, nu, s = 0;
-            buf_of<ALIAS>(0, npb, nu);
+            int s = 0;
             for (int t = 0; ok && t < VT; ++t) {
-                const VTile vt = nvt;
-                const int pb = npb, u = nu;
-                nvt = vt_next(vt, i0, i_last, w);
-                buf_of<ALIAS>(t + 1, npb, nu);
+                const VTile vt = tiles.at(t);
+                int pb, u;
+                buf_of<ALIAS>(t, pb, u);
                 if (!wait_all(&p_full[pb], u & 1)) {
                     ok = false;
                     break;
@@ -585,15 +568,10 @@ __global__ void __launch_bounds__(kThreads, 2)
             tc_fence_after();
             return true;
         };
-        VTile nvt = vt_first(i0, i_last, w);
-        int nsb, nu;
-        buf_of<ALIAS>(0, nsb, nu);
         for (int t = 0; ok && t < VT; ++t) {
-            // this tile's parameters, and the next one's computed now, off the critical path
-            const VTile vt = nvt;
-            const int sb = nsb, u = nu;
-            nvt = vt_next(vt, i0, i_last, w);
-            buf_of<ALIAS>(t + 1, nsb, nu);
+            const VTile vt = tiles.at(t);
+            int sb, u;
+            buf_of<ALIAS>(t, sb, u);
             const int j0 = vt.kt * BN;
             if (!wait_uniform(&s_full[sb], u & 1)) {
                 ok = false;
