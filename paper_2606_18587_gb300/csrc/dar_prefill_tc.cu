@@ -48,9 +48,9 @@ namespace tcp {
 using namespace sm100;
 
 constexpr int BM = 128, BN = 64;
-constexpr int kSoftmaxWarps = 4, kSoftmaxThreads = 32 * kSoftmaxWarps;  // one thread per query row
+constexpr int kSoftmaxWarps = 8, kSoftmaxThreads = 32 * kSoftmaxWarps;  // four threads per query row, two rows each
 constexpr int kThreads = 32 * (3 + kSoftmaxWarps);
-constexpr int kWarpPV = 1, kWarpS = 2 + kSoftmaxWarps;  // MMA issuers (warp 0: TMA, warps 2-5: softmax)
+constexpr int kWarpPV = 1, kWarpS = 2 + kSoftmaxWarps;  // MMA issuers (warp 0: TMA, warps 2-9: softmax)
 constexpr uint32_t kTmemCols = 256;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: p stays below 2^8 between rescales
 constexpr uint32_t kOnesBf16x2 = 0x3F803F80u;
@@ -132,25 +132,6 @@ __device__ __forceinline__ float max3(float a, float b, float c)
     return d;
 }
 
-// Maximum of N values (N = 64) with the 3-input max.f32, as a shallow tree:
-// 21 independent maxima of 3, then 7, then 3, then 1 (depth 4).
-template <int N>
-__device__ __forceinline__ float tree_max3(const float (&v)[N])
-{
-    static_assert(N == 64, "tree shaped for 64 values");
-    float a[22];
-#pragma unroll
-    for (int k = 0; k < 21; ++k)
-        a[k] = max3(v[3 * k], v[3 * k + 1], v[3 * k + 2]);
-    a[21] = v[63];
-    float b[8];
-#pragma unroll
-    for (int k = 0; k < 7; ++k)
-        b[k] = max3(a[3 * k], a[3 * k + 1], a[3 * k + 2]);
-    b[7] = a[21];
-    return max3(max3(b[0], b[1], b[2]), max3(b[3], b[4], b[5]), fmaxf(b[6], b[7]));
-}
-
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -165,6 +146,16 @@ __device__ __forceinline__ void st_swz(unsigned char *base, int r, int c, uint4 
     constexpr int mask = RB / 16 - 1;
     const int phys = c ^ ((r * RB >> 7) & mask);
     *reinterpret_cast<uint4 *>(base + (size_t)r * RB + phys * 16) = v;
+}
+
+// Write one 32-bit word (bf16 pair) at word q of 16-byte chunk c of row r of a
+// K-major operand whose rows are RB bytes, with the matching swizzle.
+template <int RB>
+__device__ __forceinline__ void st_swz4(unsigned char *base, int r, int c, int q, uint32_t v)
+{
+    constexpr int mask = RB / 16 - 1;
+    const int phys = c ^ ((r * RB >> 7) & mask);
+    *reinterpret_cast<uint32_t *>(base + (size_t)r * RB + phys * 16 + q * 4) = v;
 }
 
 // Virtual tiles: a key tile whose pairs are all local or all global is one
@@ -474,11 +465,17 @@ __global__ void __launch_bounds__(kThreads, 2)
             *abort_flag = 1;
     } else {  // warps 2 .. 2 + kSoftmaxWarps - 1
         // ------------------------------------------------------------ softmax warps
-        // one query row per thread: warp w reads TMEM lanes 32 (w % 4) .. + 31
+        // Warp w covers TMEM lanes 32 (w % 4) + 16 h .. + 15 (h = 0 for warps
+        // 2-5, 1 for warps 6-9) with the 16-lane load/store shapes: four
+        // threads per query row, each thread two rows (ra, ra + 8) and 16 of a
+        // tile's 64 columns, 8k + 2 q4 + {0, 1} (k = 0 .. 7, q4 = lane % 4).  A
+        // row's maximum is combined across its four threads with shuffles.
         const int quad = warp & 3;
-        const int row = 32 * quad + lane;
-        const int i = i0 + row;
-        const uint32_t tl = tmem + ((uint32_t)(32 * quad) << 16);
+        const int half = (warp - 2) >> 2;
+        const int q4 = lane & 3;
+        const int ra = 32 * quad + 16 * half + (lane >> 2);  // rows ra and ra + 8 of the 128
+        const int iA = i0 + ra, iB = iA + 8;
+        const uint32_t tl = tmem + ((uint32_t)(32 * quad + 16 * half) << 16);
         const int stid = threadIdx.x - 64;  // 0 .. kSoftmaxThreads - 1
         // ---- set-up: Uk as a bf16 operand, the ones block, Uv for the epilogue
         {
@@ -513,32 +510,29 @@ __global__ void __launch_bounds__(kThreads, 2)
         bool ok = wait_uniform(qt_mma, 0);
         if (ok) {
             tc_fence_after();
-            uint32_t z[16];
+            // q~ (fp32, TMEM) -> bf16 operand rows in shared memory; then clear the accumulators
+            unsigned char *qrow = sm + Ly::QT;
 #pragma unroll
-            for (int e = 0; e < 16; ++e)
-                z[e] = 0u;
-            {
-                // q~ (fp32, TMEM) -> bf16 operand rows in shared memory; then clear the accumulators
-                uint32_t r[16];
-                unsigned char *qrow = sm + Ly::QT;
+            for (int c = 0; c < DP; c += 16) {
+                uint32_t r[8];
+                tmem_ld_16x256b_x2(tl + Tm::OL + c, r);
 #pragma unroll
-                for (int c = 0; c < DP; c += 16) {
-                    tmem_ld16(tl + Tm::OL + c, r);
-#pragma unroll
-                    for (int k = 0; k < 2; ++k)
-                        st_swz<DP * 2>(qrow, row, c / 8 + k,
-                                       make_uint4(pack_bf16(__uint_as_float(r[8 * k + 0]), __uint_as_float(r[8 * k + 1])),
-                                                  pack_bf16(__uint_as_float(r[8 * k + 2]), __uint_as_float(r[8 * k + 3])),
-                                                  pack_bf16(__uint_as_float(r[8 * k + 4]), __uint_as_float(r[8 * k + 5])),
-                                                  pack_bf16(__uint_as_float(r[8 * k + 6]), __uint_as_float(r[8 * k + 7]))));
+                for (int k = 0; k < 2; ++k) {
+                    st_swz4<DP * 2>(qrow, ra, c / 8 + k, q4, pack_bf16(__uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1])));
+                    st_swz4<DP * 2>(qrow, ra + 8, c / 8 + k, q4,
+                                    pack_bf16(__uint_as_float(r[4 * k + 2]), __uint_as_float(r[4 * k + 3])));
                 }
-#pragma unroll
-                for (int c = 0; c < 64; c += 16)
-                    tmem_st16(tl + Tm::OL + c, z);
-#pragma unroll
-                for (int c = 0; c < DP + 16; c += 16)  // O_glob and the row-sum columns
-                    tmem_st16(tl + Tm::OG + c, z);
             }
+            uint32_t z[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                z[e] = 0u;
+#pragma unroll
+            for (int c = 0; c < 64; c += 16)
+                tmem_st_16x256b_x2(tl + Tm::OL + c, z);
+#pragma unroll
+            for (int c = 0; c < DP + 16; c += 16)  // O_glob and the row-sum columns
+                tmem_st_16x256b_x2(tl + Tm::OG + c, z);
             tmem_wait_st();
             fence_proxy_async_smem();
         }
@@ -547,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         mbar_arrive(qt_ready);
 
         const float c2 = a.qscale;  // softmax scale * log2(e)
-        float m_used = -INFINITY;
+        float mA = -INFINITY, mB = -INFINITY;  // running maxima (log2 units) of rows ra, ra + 8
         // last tile whose PV this thread has seen complete, per S buffer
         int pv_seen0 = -1, pv_seen1 = -1;
         // wait until PV(v) (its own products) has completed
@@ -568,6 +562,19 @@ __global__ void __launch_bounds__(kThreads, 2)
             tc_fence_after();
             return true;
         };
+        // scale 16 columns of both rows' accumulators
+        auto rescale16 = [&](uint32_t col, float alA, float alB) {
+            uint32_t r[8];
+            tmem_ld_16x256b_x2(tl + col, r);
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                r[4 * k + 0] = __float_as_uint(__uint_as_float(r[4 * k + 0]) * alA);
+                r[4 * k + 1] = __float_as_uint(__uint_as_float(r[4 * k + 1]) * alA);
+                r[4 * k + 2] = __float_as_uint(__uint_as_float(r[4 * k + 2]) * alB);
+                r[4 * k + 3] = __float_as_uint(__uint_as_float(r[4 * k + 3]) * alB);
+            }
+            tmem_st_16x256b_x2(tl + col, r);
+        };
         for (int t = 0; ok && t < VT; ++t) {
             const VTile vt = tiles.at(t);
             int sb, u;
@@ -578,13 +585,18 @@ __global__ void __launch_bounds__(kThreads, 2)
                 break;
             }
             tc_fence_after();
-            float s[BN];
+            // row ra: sa[2k + j], row ra + 8: sv[2k + j] = score column 8k + 2 q4 + j
+            float sa[16], sv[16];
             {
-                uint32_t r[BN];
-                tmem_ld64(tl + Tm::S + sb * BN, r);
+                uint32_t r[32];
+                tmem_ld_16x256b_x8(tl + Tm::S + sb * BN, r);
 #pragma unroll
-                for (int e = 0; e < BN; ++e)
-                    s[e] = __uint_as_float(r[e]);
+                for (int k = 0; k < 8; ++k) {
+                    sa[2 * k] = __uint_as_float(r[4 * k]);
+                    sa[2 * k + 1] = __uint_as_float(r[4 * k + 1]);
+                    sv[2 * k] = __uint_as_float(r[4 * k + 2]);
+                    sv[2 * k + 1] = __uint_as_float(r[4 * k + 3]);
+                }
             }
             if constexpr (!ALIAS) {  // the S buffer may be overwritten now (S(t + 1))
                 tc_fence_before();
@@ -594,45 +606,72 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
 
             // masks: causal (tiles reaching past row i0), the other part of a
-            // band tile, rows past the end; the kept columns form one range
+            // band tile, rows past the end; the kept columns of a row form one
+            // range, here relative to this thread's column offset 2 q4
             if (__builtin_expect(j0 + BN - 1 > i0 || vt.band || i0 + BM > N, 0)) {
-                int e_hi = i < N ? i - j0 : -1, e_lo = 0;
+                int hiA = iA < N ? iA - j0 : -1, hiB = iB < N ? iB - j0 : -1, loA = 0, loB = 0;
                 if (vt.band) {
-                    if (vt.loc)
-                        e_lo = i - w - j0 + 1;
-                    else
-                        e_hi = min(e_hi, i - w - j0);
+                    if (vt.loc) {
+                        loA = iA - w - j0 + 1;
+                        loB = iB - w - j0 + 1;
+                    } else {
+                        hiA = min(hiA, iA - w - j0);
+                        hiB = min(hiB, iB - w - j0);
+                    }
                 }
+                loA -= 2 * q4;
+                loB -= 2 * q4;
+                hiA -= 2 * q4;
+                hiB -= 2 * q4;
                 // one bound at a time, each only where some row of the warp needs it
-                if (__any_sync(0xffffffffu, e_lo > 0)) {
+                if (__any_sync(0xffffffffu, loA > -2 * q4 || loB > -2 * q4)) {
 #pragma unroll
-                    for (int e = 0; e < BN; ++e)
-                        s[e] = e >= e_lo ? s[e] : -INFINITY;
+                    for (int e = 0; e < 16; ++e) {
+                        const int col = 8 * (e >> 1) + (e & 1);
+                        sa[e] = col >= loA ? sa[e] : -INFINITY;
+                        sv[e] = col >= loB ? sv[e] : -INFINITY;
+                    }
                 }
-                if (__any_sync(0xffffffffu, e_hi < BN - 1)) {
+                if (__any_sync(0xffffffffu, hiA + 2 * q4 < BN - 1 || hiB + 2 * q4 < BN - 1)) {
 #pragma unroll
-                    for (int e = 0; e < BN; ++e)
-                        s[e] = e <= e_hi ? s[e] : -INFINITY;
+                    for (int e = 0; e < 16; ++e) {
+                        const int col = 8 * (e >> 1) + (e & 1);
+                        sa[e] = col <= hiA ? sa[e] : -INFINITY;
+                        sv[e] = col <= hiB ? sv[e] : -INFINITY;
+                    }
                 }
             }
-            const float mt = tree_max3(s) * c2;
-            // raise the running max only when it grows by more than the threshold
-            const bool raise = mt > m_used + kRescaleThreshold;
-            const bool scale_o = raise && m_used != -INFINITY;
-            // O's scale factor when the running max is raised (applied below, once P is computed)
-            const float alpha = scale_o ? ex2_approx(m_used - mt) : 1.f;
-            if (raise)
-                m_used = mt;
-            // P = 2^(s * c2 - m) in bf16 pairs (masked entries give 0)
-            const float mneg = m_used == -INFINITY ? 0.f : -m_used;
-            uint32_t pk[BN / 2];
+            // row maxima: this thread's 16 columns, then across the row's four threads
+            float xA = max3(max3(sa[0], sa[1], sa[2]), max3(sa[3], sa[4], sa[5]), max3(sa[6], sa[7], sa[8]));
+            float xB = max3(max3(sv[0], sv[1], sv[2]), max3(sv[3], sv[4], sv[5]), max3(sv[6], sv[7], sv[8]));
+            xA = max3(xA, max3(sa[9], sa[10], sa[11]), max3(sa[12], sa[13], fmaxf(sa[14], sa[15])));
+            xB = max3(xB, max3(sv[9], sv[10], sv[11]), max3(sv[12], sv[13], fmaxf(sv[14], sv[15])));
+            xA = fmaxf(xA, __shfl_xor_sync(0xffffffffu, xA, 1));
+            xB = fmaxf(xB, __shfl_xor_sync(0xffffffffu, xB, 1));
+            xA = fmaxf(xA, __shfl_xor_sync(0xffffffffu, xA, 2)) * c2;
+            xB = fmaxf(xB, __shfl_xor_sync(0xffffffffu, xB, 2)) * c2;
+            // raise a running max only when it grows by more than the threshold
+            const bool raiseA = xA > mA + kRescaleThreshold, raiseB = xB > mB + kRescaleThreshold;
+            const bool scaleA = raiseA && mA != -INFINITY, scaleB = raiseB && mB != -INFINITY;
+            // O's scale factors when a running max is raised (applied below, once P is computed)
+            const float alA = scaleA ? ex2_approx(mA - xA) : 1.f, alB = scaleB ? ex2_approx(mB - xB) : 1.f;
+            if (raiseA)
+                mA = xA;
+            if (raiseB)
+                mB = xB;
+            // P = 2^(s * c2 - m) in bf16 pairs (masked entries give 0): pw[2k] row
+            // ra, pw[2k + 1] row ra + 8, P column 4k + q4 (keys 8k + 2 q4, + 1)
+            const float nA = mA == -INFINITY ? 0.f : -mA, nB = mB == -INFINITY ? 0.f : -mB;
+            uint32_t pw[16];
 #pragma unroll
-            for (int e = 0; e < BN; e += 2) {
-                float x0, x1;
-                ffma2(x0, x1, s[e], s[e + 1], c2, c2, mneg, mneg);
-                pk[e / 2] = ex2_bf16x2(cvt_bf16x2(x0, x1));
+            for (int k = 0; k < 8; ++k) {
+                float x0, x1, y0, y1;
+                ffma2(x0, x1, sa[2 * k], sa[2 * k + 1], c2, c2, nA, nA);
+                ffma2(y0, y1, sv[2 * k], sv[2 * k + 1], c2, c2, nB, nB);
+                pw[2 * k] = ex2_bf16x2(cvt_bf16x2(x0, x1));
+                pw[2 * k + 1] = ex2_bf16x2(cvt_bf16x2(y0, y1));
             }
-            if (__builtin_expect(__any_sync(0xffffffffu, scale_o), 0)) {
+            if (__builtin_expect(__any_sync(0xffffffffu, scaleA || scaleB), 0)) {
                 // every earlier PV must have landed before O is rescaled (PV(t),
                 // which needs P(t), cannot start before it is)
                 if (!wait_pv(t - 1) || !wait_pv(t - 2)) {
@@ -640,23 +679,11 @@ __global__ void __launch_bounds__(kThreads, 2)
                     break;
                 }
 #pragma unroll
-                for (int c = 0; c < 64; c += 16) {
-                    uint32_t r[16];
-                    tmem_ld16(tl + Tm::OL + c, r);
+                for (int c = 0; c < 64; c += 16)
+                    rescale16(Tm::OL + c, alA, alB);
 #pragma unroll
-                    for (int e = 0; e < 16; ++e)
-                        r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-                    tmem_st16(tl + Tm::OL + c, r);
-                }
-#pragma unroll
-                for (int c = 0; c < DP + 16; c += 16) {  // O_glob and the row sums
-                    uint32_t r[16];
-                    tmem_ld16(tl + Tm::OG + c, r);
-#pragma unroll
-                    for (int e = 0; e < 16; ++e)
-                        r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-                    tmem_st16(tl + Tm::OG + c, r);
-                }
+                for (int c = 0; c < DP + 16; c += 16)  // O_glob and the row sums
+                    rescale16(Tm::OG + c, alA, alB);
             }
             // one buffer: PV(t - 1) must be done with the P buffer (two buffers:
             // P goes over S(t), whose buffer was free before S(t) was computed)
@@ -664,7 +691,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 ok = false;
                 break;
             }
-            tmem_st32(tl + Tm::P + (ALIAS ? sb * BN : 0), pk);
+            tmem_st_16x128b_x8(tl + Tm::P + (ALIAS ? sb * BN : 0), pw);
             tmem_wait_st();
             tc_fence_before();
             __syncwarp();
@@ -673,57 +700,67 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
 
         // ---- epilogue: o = (O_loc + O_glob Uv) / l (the last products may
-        // still be running on either buffer)
+        // still be running on either buffer).  O_glob rows go through shared
+        // memory (the stage area, idle by now), so each thread can take the
+        // whole d_down vector of its two rows.
         if (ok && wait_pv(VT - 1) && wait_pv(VT - 2)) {
             const float *sUv = reinterpret_cast<const float *>(sm + Ly::UV);
-            float og[DP];
-            float l;
-            {
-                uint32_t r[16];
+            constexpr int OGS = DP + 1;  // padded row stride (floats)
+            float *sOG = reinterpret_cast<float *>(sm + Ly::STG);
 #pragma unroll
-                for (int c = 0; c < DP; c += 16) {
-                    tmem_ld16(tl + Tm::OG + c, r);
+            for (int c = 0; c < DP; c += 16) {
+                uint32_t r[8];
+                tmem_ld_16x256b_x2(tl + Tm::OG + c, r);
 #pragma unroll
-                    for (int e = 0; e < 16; ++e)
-                        og[c + e] = __uint_as_float(r[e]);
-                }
-                tmem_ld16(tl + Tm::SUM, r);
-                l = __uint_as_float(r[0]);
-            }
-            const float inv = l > 0.f ? 1.f / l : 0.f;
-            bf16 *orow = static_cast<bf16 *>(a.out) + (((size_t)b * a.Hq + h) * nrows + (i - L0)) * 64;
+                for (int k = 0; k < 2; ++k)
 #pragma unroll
-            for (int c = 0; c < 64; c += 16) {
-                float o[16];
-                {
-                    uint32_t r[16];
-                    tmem_ld16(tl + Tm::OL + c, r);
-#pragma unroll
-                    for (int e = 0; e < 16; ++e)
-                        o[e] = __uint_as_float(r[e]);
-                }
-#pragma unroll
-                for (int kk = 0; kk < DP; ++kk) {
-                    const float4 *u4 = reinterpret_cast<const float4 *>(sUv + kk * 64 + c);
-#pragma unroll
-                    for (int e4 = 0; e4 < 4; ++e4) {
-                        const float4 uu = u4[e4];
-                        o[4 * e4 + 0] = fmaf(og[kk], uu.x, o[4 * e4 + 0]);
-                        o[4 * e4 + 1] = fmaf(og[kk], uu.y, o[4 * e4 + 1]);
-                        o[4 * e4 + 2] = fmaf(og[kk], uu.z, o[4 * e4 + 2]);
-                        o[4 * e4 + 3] = fmaf(og[kk], uu.w, o[4 * e4 + 3]);
+                    for (int j = 0; j < 2; ++j) {
+                        sOG[ra * OGS + c + 8 * k + 2 * q4 + j] = __uint_as_float(r[4 * k + j]);
+                        sOG[(ra + 8) * OGS + c + 8 * k + 2 * q4 + j] = __uint_as_float(r[4 * k + 2 + j]);
                     }
-                }
+            }
+            float lA, lB;
+            {
+                uint32_t r[8];
+                tmem_ld_16x256b_x2(tl + Tm::SUM, r);  // 16 identical columns
+                lA = __uint_as_float(r[0]);
+                lB = __uint_as_float(r[2]);
+            }
+            // O_loc: oa[2k + j] row ra, ov[2k + j] row ra + 8, output column 8k + 2 q4 + j
+            float oa[16], ov[16];
+            {
+                uint32_t r[32];
+                tmem_ld_16x256b_x8(tl + Tm::OL, r);
 #pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    o[e] *= inv;
-                if (i < N) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(orow + c);
-                    dst[0] = make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]),
-                                        pack_bf16(o[6], o[7]));
-                    dst[1] = make_uint4(pack_bf16(o[8], o[9]), pack_bf16(o[10], o[11]), pack_bf16(o[12], o[13]),
-                                        pack_bf16(o[14], o[15]));
+                for (int k = 0; k < 8; ++k) {
+                    oa[2 * k] = __uint_as_float(r[4 * k]);
+                    oa[2 * k + 1] = __uint_as_float(r[4 * k + 1]);
+                    ov[2 * k] = __uint_as_float(r[4 * k + 2]);
+                    ov[2 * k + 1] = __uint_as_float(r[4 * k + 3]);
                 }
+            }
+            __syncwarp();
+#pragma unroll 4
+            for (int kk = 0; kk < DP; ++kk) {
+                const float gA = sOG[ra * OGS + kk], gB = sOG[(ra + 8) * OGS + kk];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const float2 uu = *reinterpret_cast<const float2 *>(sUv + kk * 64 + 8 * k + 2 * q4);
+                    oa[2 * k] = fmaf(gA, uu.x, oa[2 * k]);
+                    oa[2 * k + 1] = fmaf(gA, uu.y, oa[2 * k + 1]);
+                    ov[2 * k] = fmaf(gB, uu.x, ov[2 * k]);
+                    ov[2 * k + 1] = fmaf(gB, uu.y, ov[2 * k + 1]);
+                }
+            }
+            const float invA = lA > 0.f ? 1.f / lA : 0.f, invB = lB > 0.f ? 1.f / lB : 0.f;
+            bf16 *orowA = static_cast<bf16 *>(a.out) + (((size_t)b * a.Hq + h) * nrows + (iA - L0)) * 64 + 2 * q4;
+            bf16 *orowB = orowA + 8 * 64;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                if (iA < N)
+                    *reinterpret_cast<uint32_t *>(orowA + 8 * k) = pack_bf16(oa[2 * k] * invA, oa[2 * k + 1] * invA);
+                if (iB < N)
+                    *reinterpret_cast<uint32_t *>(orowB + 8 * k) = pack_bf16(ov[2 * k] * invB, ov[2 * k + 1] * invB);
             }
         } else {
             ok = false;
