@@ -15,6 +15,9 @@ arrays.  Function-level citations:
 * :func:`prefill`, :func:`decode` -- the two row sets the method is used with:
   every position (training-mode forward), or the last position of each
   sequence (one inference step).
+* :func:`attention_rows_direct`, :func:`prefill_direct`, :func:`decode_direct`
+  -- Sec. 5, "Direct lower-dimensional global attention": the global path in
+  d_down with a query of its own and an output map of the global values.
 
 Storage types: ``"f32"`` arrays are float32; ``"bf16"`` arrays are uint16
 holding bfloat16 bit patterns.
@@ -60,6 +63,10 @@ def _load():
             [ctypes.c_int] * 8 + [P] * 7 + [ctypes.c_double, ctypes.c_long, P, P, P, P, ctypes.c_int]
         )
         lib.dar_oracle_attention.restype = ctypes.c_int
+        lib.dar_oracle_attention_direct.argtypes = (
+            [ctypes.c_int] * 8 + [P] * 7 + [ctypes.c_double, ctypes.c_double, ctypes.c_long, P, P, P, P, ctypes.c_int]
+        )
+        lib.dar_oracle_attention_direct.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -183,5 +190,83 @@ def decode(q_last, k_hist, v_hist, lens, Dk, Uk, Dv, Uv, w, dtype, scale=None, n
         rows = np.array([(0, h, L - 1) for h in hs], dtype=np.int32)
         q_rows = np.ascontiguousarray(q_last[b, hs])
         res = attention_rows(q_rows, Hq, kb, vb, kd, vd, Uk, Uv, w, dtype, rows, scale, nthreads)
+        out[b, hs] = res
+    return out
+
+
+def attention_rows_direct(q_rows, qd_rows, Hq, k, v, kd, vd, Wo, w, dtype, rows, scale=None, scale_down=None,
+                          nthreads=None):
+    """Sec. 5, direct lower-dimensional global attention, for explicit rows.
+
+    Local pairs (``i - j < w``, Eq. 3) score ``scale * q . k_j`` against the
+    full-dimension keys; global pairs score ``scale_down * q^D . k^D_j`` in
+    d_down, with ``qd_rows [R,dd]`` the d_down query of each row.  One softmax
+    over both (Eq. 4); global values are ``v^D_j Wo`` with ``Wo [Hkv,dd,d]``.
+    Defaults: ``scale = 1/sqrt(d)``, ``scale_down = 1/sqrt(dd)``.  Returns
+    float64 ``[R,d]``."""
+    q_rows, qd_rows, k, v, kd, vd = (_check(a, dtype) for a in (q_rows, qd_rows, k, v, kd, vd))
+    Wo = np.ascontiguousarray(Wo, dtype=np.float32)
+    B, Hkv, N, d = k.shape
+    dd = kd.shape[3]
+    rows = np.ascontiguousarray(rows, dtype=np.int32).reshape(-1, 3)
+    assert q_rows.shape == (rows.shape[0], d) and qd_rows.shape == (rows.shape[0], dd)
+    rb, rh, ri = (np.ascontiguousarray(rows[:, c]) for c in range(3))
+    out = np.zeros((rows.shape[0], d), dtype=np.float64)
+    scale = 1.0 / np.sqrt(d) if scale is None else scale
+    scale_down = 1.0 / np.sqrt(dd) if scale_down is None else scale_down
+    nthreads = (os.cpu_count() or 1) if nthreads is None else nthreads
+    rc = _load().dar_oracle_attention_direct(
+        _DTYPES[dtype], B, int(Hq), Hkv, N, d, dd, int(w),
+        _ptr(q_rows), _ptr(qd_rows), _ptr(k), _ptr(v), _ptr(kd), _ptr(vd), _ptr(Wo),
+        float(scale), float(scale_down), rows.shape[0], _ptr(rb), _ptr(rh), _ptr(ri), _ptr(out), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle rejected its arguments")
+    return out
+
+
+def prefill_direct(q, qd, k, v, Dk, Dv, Wo, w, dtype, scale=None, scale_down=None, nthreads=None, rows=None):
+    """Causal forward of the direct variant over positions 0..N-1.
+
+    ``q [B,Hq,N,d]``, ``qd [B,Hq,N,dd]`` (the d_down queries), ``k, v
+    [B,Hkv,N,d]``; ``k^D, v^D`` come from Eq. 1 with ``Dk, Dv``.  Rows as in
+    :func:`prefill`."""
+    B, Hq, N, d = q.shape
+    kd = down_project(k, Dk, dtype)
+    vd = down_project(v, Dv, dtype)
+    full = rows is None
+    if full:
+        bb, hh, ii = np.meshgrid(np.arange(B), np.arange(Hq), np.arange(N), indexing="ij")
+        rows = np.stack([bb.ravel(), hh.ravel(), ii.ravel()], axis=1)
+    rows = np.asarray(rows, dtype=np.int64).reshape(-1, 3)
+    q_rows = np.ascontiguousarray(q[rows[:, 0], rows[:, 1], rows[:, 2]])
+    qd_rows = np.ascontiguousarray(qd[rows[:, 0], rows[:, 1], rows[:, 2]])
+    out = attention_rows_direct(q_rows, qd_rows, Hq, k, v, kd, vd, Wo, w, dtype, rows, scale, scale_down,
+                                nthreads)
+    return out.reshape(B, Hq, N, d) if full else out
+
+
+def decode_direct(q_last, qd_last, k_hist, v_hist, lens, Dk, Dv, Wo, w, dtype, scale=None, scale_down=None,
+                  nthreads=None, heads=None):
+    """One inference step of the direct variant (query at ``lens[b]-1``).
+
+    ``q_last [B,Hq,d]``, ``qd_last [B,Hq,dd]``; otherwise as :func:`decode`."""
+    B, Hq, d = q_last.shape
+    lens = np.asarray(lens, dtype=np.int64)
+    out = np.zeros((B, Hq, d), dtype=np.float64)
+    if heads is None:
+        heads = [(b, h) for b in range(B) for h in range(Hq)]
+    by_seq = {}
+    for b, h in heads:
+        if lens[b] > 0:
+            by_seq.setdefault(int(b), []).append(int(h))
+    for b, hs in sorted(by_seq.items()):
+        L = int(lens[b])
+        kb = np.ascontiguousarray(k_hist[b:b + 1, :, :L])
+        vb = np.ascontiguousarray(v_hist[b:b + 1, :, :L])
+        kd = down_project(kb, Dk, dtype)
+        vd = down_project(vb, Dv, dtype)
+        rows = np.array([(0, h, L - 1) for h in hs], dtype=np.int32)
+        res = attention_rows_direct(np.ascontiguousarray(q_last[b, hs]), np.ascontiguousarray(qd_last[b, hs]), Hq,
+                                    kb, vb, kd, vd, Wo, w, dtype, rows, scale, scale_down, nthreads)
         out[b, hs] = res
     return out

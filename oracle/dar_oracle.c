@@ -246,3 +246,140 @@ int dar_oracle_attention(int dtype, int B, int Hq, int Hkv, int N, int d, int dd
     free(th);
     return 0;
 }
+
+/* ---- Sec. 5, "Direct lower-dimensional global attention" ------------------
+ * The global path runs in d_down: a query q^D_i of its own (d_down), scored
+ * against the d_down keys k^D_j of the distant tokens with scale_down
+ * (1/sqrt(d_down) by default), and the weighted d_down values mapped to d by
+ * an output map Wo (d_down x d, per KV head).  The local path is unchanged
+ * (Eq. 3 selection, scale 1/sqrt(d)), and one softmax covers both paths
+ * (Eq. 4 carried over).  Per token the mapped value v^D_j Wo is formed
+ * explicitly, in fp64, before the weighted sum. */
+
+typedef struct {
+    attn_job base;      /* k, v, kd, vd, q (local query), rows, out, threads */
+    const void *qd;     /* [nrows][dd] storage type: the d_down query of each row */
+    const float *Wo;    /* [Hkv][dd][d] fp32 */
+    double scale_down;
+} attn_direct_job;
+
+static void attn_unit_direct(const attn_direct_job *D, int b, int g)
+{
+    const attn_job *J = &D->base;
+    const int d = J->d, dd = J->dd, N = J->N, G = J->Hq / J->Hkv;
+    int jmax = -1;
+    for (long r = 0; r < J->nrows; ++r)
+        if (J->row_b[r] == b && J->row_h[r] / G == g && J->row_i[r] > jmax)
+            jmax = J->row_i[r];
+    if (jmax < 0)
+        return;
+    const int n = jmax + 1;
+
+    double *Kfull = malloc(sizeof(double) * (size_t)n * d);
+    double *Vfull = malloc(sizeof(double) * (size_t)n * d);
+    double *Kdown = malloc(sizeof(double) * (size_t)n * dd);
+    double *Vmap = malloc(sizeof(double) * (size_t)n * d);
+    double *s = malloc(sizeof(double) * (size_t)n);
+    const size_t base = ((size_t)b * J->Hkv + g) * N;
+
+    for (int j = 0; j < n; ++j) {
+        for (int t = 0; t < d; ++t) {
+            Kfull[(size_t)j * d + t] = load_as_f32(J->k, J->dtype, (base + j) * d + t);
+            Vfull[(size_t)j * d + t] = load_as_f32(J->v, J->dtype, (base + j) * d + t);
+        }
+        for (int c = 0; c < dd; ++c)
+            Kdown[(size_t)j * dd + c] = load_as_f32(J->kd, J->dtype, (base + j) * dd + c);
+        for (int t = 0; t < d; ++t) {
+            double va = 0.0;
+            for (int c = 0; c < dd; ++c)
+                va += (double)load_as_f32(J->vd, J->dtype, (base + j) * dd + c) *
+                      (double)D->Wo[((size_t)g * dd + c) * d + t];
+            Vmap[(size_t)j * d + t] = va;
+        }
+    }
+
+    for (long r = 0; r < J->nrows; ++r) {
+        if (J->row_b[r] != b || J->row_h[r] / G != g)
+            continue;
+        const int i = J->row_i[r];
+        double *o = J->out + (size_t)r * d;
+        double smax = -INFINITY;
+        for (int j = 0; j <= i; ++j) {
+            double dot = 0.0;
+            if (i - j < J->w) {
+                for (int t = 0; t < d; ++t)
+                    dot += (double)load_as_f32(J->q, J->dtype, (size_t)r * d + t) * Kfull[(size_t)j * d + t];
+                s[j] = J->scale * dot;
+            } else {
+                for (int c = 0; c < dd; ++c)
+                    dot += (double)load_as_f32(D->qd, J->dtype, (size_t)r * dd + c) * Kdown[(size_t)j * dd + c];
+                s[j] = D->scale_down * dot;
+            }
+            if (s[j] > smax)
+                smax = s[j];
+        }
+        double denom = 0.0;
+        for (int j = 0; j <= i; ++j)
+            denom += exp(s[j] - smax);
+        for (int t = 0; t < d; ++t)
+            o[t] = 0.0;
+        for (int j = 0; j <= i; ++j) {
+            const double p = exp(s[j] - smax) / denom;
+            const double *val = (i - j < J->w) ? &Vfull[(size_t)j * d] : &Vmap[(size_t)j * d];
+            for (int t = 0; t < d; ++t)
+                o[t] += p * val[t];
+        }
+    }
+    free(Kfull);
+    free(Vfull);
+    free(Kdown);
+    free(Vmap);
+    free(s);
+}
+
+static void *attn_direct_worker(void *arg)
+{
+    const attn_direct_job *D = (const attn_direct_job *)arg;
+    const int units = D->base.B * D->base.Hkv;
+    for (int u = D->base.tid; u < units; u += D->base.nthreads)
+        attn_unit_direct(D, u / D->base.Hkv, u % D->base.Hkv);
+    return NULL;
+}
+
+/* As dar_oracle_attention, with the global path of Sec. 5's direct variant:
+ * qd [nrows][dd] the d_down query of each row, Wo [Hkv][dd][d] the output map
+ * of the global path, scale_down the global scores' scale. */
+int dar_oracle_attention_direct(int dtype, int B, int Hq, int Hkv, int N, int d, int dd, int w,
+                                const void *q, const void *qd, const void *k, const void *v,
+                                const void *kd, const void *vd, const float *Wo, double scale,
+                                double scale_down, long nrows, const int *row_b, const int *row_h,
+                                const int *row_i, double *out, int nthreads)
+{
+    if (B < 1 || Hkv < 1 || Hq < Hkv || Hq % Hkv || N < 1 || d < 1 || dd < 1 || w < 0 ||
+        nrows < 0 || (dtype != ORC_F32 && dtype != ORC_BF16))
+        return -1;
+    for (long r = 0; r < nrows; ++r)
+        if (row_b[r] < 0 || row_b[r] >= B || row_h[r] < 0 || row_h[r] >= Hq ||
+            row_i[r] < 0 || row_i[r] >= N)
+            return -1;
+    if (nthreads < 1)
+        nthreads = 1;
+    attn_direct_job *jobs = malloc(sizeof(attn_direct_job) * (size_t)nthreads);
+    pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
+    for (int t = 0; t < nthreads; ++t) {
+        attn_job J = {dtype, B, Hq, Hkv, N, d, dd, w, q, k, v, kd, vd, NULL, NULL, scale,
+                      nrows, row_b, row_h, row_i, out, nthreads, t};
+        jobs[t].base = J;
+        jobs[t].qd = qd;
+        jobs[t].Wo = Wo;
+        jobs[t].scale_down = scale_down;
+    }
+    for (int t = 1; t < nthreads; ++t)
+        pthread_create(&th[t], NULL, attn_direct_worker, &jobs[t]);
+    attn_direct_worker(&jobs[0]);
+    for (int t = 1; t < nthreads; ++t)
+        pthread_join(th[t], NULL);
+    free(jobs);
+    free(th);
+    return 0;
+}
