@@ -15,6 +15,9 @@ arrays.  Function-level citations:
 * :func:`prefill`, :func:`decode` -- the two row sets the method is used with:
   every position (training-mode forward), or the last position of each
   sequence (one inference step).
+* :func:`backward` -- Sec. 2.3 (training): the gradients of the causal
+  forward with respect to q, k, v and the four projections, by the chain rule
+  through Eq. 4, 3, 2 and 1 in turn.
 * :func:`attention_rows_direct`, :func:`prefill_direct`, :func:`decode_direct`
   -- Sec. 5, "Direct lower-dimensional global attention": the global path in
   d_down with a query of its own and an output map of the global values.
@@ -67,6 +70,10 @@ def _load():
             [ctypes.c_int] * 8 + [P] * 7 + [ctypes.c_double, ctypes.c_double, ctypes.c_long, P, P, P, P, ctypes.c_int]
         )
         lib.dar_oracle_attention_direct.restype = ctypes.c_int
+        lib.dar_oracle_backward.argtypes = (
+            [ctypes.c_int] * 8 + [P] * 8 + [ctypes.c_double] + [P] * 7 + [ctypes.c_int]
+        )
+        lib.dar_oracle_backward.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -270,3 +277,29 @@ def decode_direct(q_last, qd_last, k_hist, v_hist, lens, Dk, Dv, Wo, w, dtype, s
                                     kb, vb, kd, vd, Wo, w, dtype, rows, scale, scale_down, nthreads)
         out[b, hs] = res
     return out
+
+
+def backward(q, k, v, Dk, Uk, Dv, Uv, dout, w, dtype, scale=None, nthreads=None):
+    """Sec. 2.3, training: gradients of the causal forward (:func:`prefill`)
+    for the output gradient ``dout [B,Hq,N,d]`` (storage type).
+
+    Returns a dict of float64 arrays: ``dq [B,Hq,N,d]``, ``dk, dv [B,Hkv,N,d]``,
+    ``dDk, dDv [Hkv,d,dd]``, ``dUk, dUv [Hkv,dd,d]``.  The rounding of the
+    stored ``k^D, v^D`` to the storage type is not differentiated."""
+    q, k, v, dout = (_check(a, dtype) for a in (q, k, v, dout))
+    Dk, Uk, Dv, Uv = (np.ascontiguousarray(a, dtype=np.float32) for a in (Dk, Uk, Dv, Uv))
+    B, Hq, N, d = q.shape
+    Hkv = k.shape[1]
+    dd = Dk.shape[2]
+    scale = 1.0 / np.sqrt(d) if scale is None else scale
+    nthreads = (os.cpu_count() or 1) if nthreads is None else nthreads
+    g = dict(dq=np.zeros((B, Hq, N, d)), dk=np.zeros((B, Hkv, N, d)), dv=np.zeros((B, Hkv, N, d)),
+             dDk=np.zeros((Hkv, d, dd)), dUk=np.zeros((Hkv, dd, d)), dDv=np.zeros((Hkv, d, dd)),
+             dUv=np.zeros((Hkv, dd, d)))
+    rc = _load().dar_oracle_backward(
+        _DTYPES[dtype], B, Hq, Hkv, N, d, dd, int(w), _ptr(q), _ptr(k), _ptr(v), _ptr(Dk), _ptr(Uk), _ptr(Dv),
+        _ptr(Uv), _ptr(dout), float(scale), _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]), _ptr(g["dDk"]),
+        _ptr(g["dUk"]), _ptr(g["dDv"]), _ptr(g["dUv"]), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle rejected its arguments")
+    return g

@@ -383,3 +383,232 @@ int dar_oracle_attention_direct(int dtype, int B, int Hq, int Hkv, int N, int d,
     free(th);
     return 0;
 }
+
+/* ---- Sec. 2.3, training: gradients of the DAR attention forward -----------
+ * The loss is any scalar whose gradient with respect to the outputs o_i is
+ * dO_i (given).  Backpropagation runs through the forward's steps in reverse,
+ * each written out as its plain derivative, in fp64:
+ *
+ *   Eq. 4   o_i = sum_j p_ij val_j,  p_i = softmax_j(s_ij),  s_ij = scale q_i . key_j
+ *           dP_ij = dO_i . val_j;  dS_ij = p_ij (dP_ij - sum_l p_il dP_il)
+ *           dq_i = scale sum_j dS_ij key_j;  dkey_j += scale dS_ij q_i;  dval_j += p_ij dO_i
+ *   Eq. 3   key_j / val_j is the full k_j / v_j (i - j < w) or the lifted k'_j / v'_j,
+ *           so each (i, j) pair sends its gradient to exactly one of the two
+ *   Eq. 2   k'_j = k^D_j Uk:  dk^D_j = dk'_j Uk^T,  dUk += (k^D_j)^T dk'_j   (same for v, Uv)
+ *   Eq. 1   k^D_j = k_j Dk:   dk_j += dk^D_j Dk^T,  dDk += k_j^T dk^D_j      (same for v, Dv)
+ *
+ * The forward stores k^D rounded to the storage type; its derivative is taken
+ * as that of the unrounded product (the rounding is not differentiated), so the
+ * bottleneck projections receive the gradient of every position that reaches
+ * a token through the global path, as Sec. 2.3 describes.  GQA: the gradients
+ * of a KV head sum over the query heads that read it. */
+
+typedef struct {
+    int dtype, B, Hq, Hkv, N, d, dd, w;
+    const void *q, *k, *v, *dout;             /* storage type */
+    const float *Dk, *Uk, *Dv, *Uv;           /* fp32 */
+    double scale;
+    double *dq, *dk, *dv;                     /* [B][Hq|Hkv][N][d] */
+    double *wpart;                            /* [B][Hkv][4][d * dd]: dDk, dUk, dDv, dUv of one unit */
+    int nthreads, tid;
+} bwd_job;
+
+static void bwd_unit(const bwd_job *J, int b, int g)
+{
+    const int d = J->d, dd = J->dd, N = J->N, G = J->Hq / J->Hkv, w = J->w;
+    const size_t base = ((size_t)b * J->Hkv + g) * N;
+    const float *Dk = J->Dk + (size_t)g * d * dd, *Dv = J->Dv + (size_t)g * d * dd;
+    const float *Uk = J->Uk + (size_t)g * dd * d, *Uv = J->Uv + (size_t)g * dd * d;
+    double *K = malloc(sizeof(double) * (size_t)N * d), *V = malloc(sizeof(double) * (size_t)N * d);
+    double *KD = malloc(sizeof(double) * (size_t)N * dd), *VD = malloc(sizeof(double) * (size_t)N * dd);
+    double *Kl = malloc(sizeof(double) * (size_t)N * d), *Vl = malloc(sizeof(double) * (size_t)N * d);
+    double *dKl = calloc((size_t)N * d, sizeof(double)), *dVl = calloc((size_t)N * d, sizeof(double));
+    double *p = malloc(sizeof(double) * (size_t)N), *dp = malloc(sizeof(double) * (size_t)N);
+    double *Q = malloc(sizeof(double) * (size_t)d), *dO = malloc(sizeof(double) * (size_t)d);
+    double *dk = J->dk + base * d, *dv = J->dv + base * d;
+    double *wp = J->wpart + ((size_t)b * J->Hkv + g) * 4 * (size_t)d * dd;
+    double *dDk = wp, *dUk = wp + (size_t)d * dd, *dDv = wp + 2 * (size_t)d * dd, *dUv = wp + 3 * (size_t)d * dd;
+
+    /* forward quantities: Eq. 1 (stored, rounded to T) and Eq. 2 (explicit lift) */
+    for (int j = 0; j < N; ++j) {
+        for (int t = 0; t < d; ++t) {
+            K[(size_t)j * d + t] = load_as_f32(J->k, J->dtype, (base + j) * d + t);
+            V[(size_t)j * d + t] = load_as_f32(J->v, J->dtype, (base + j) * d + t);
+        }
+        for (int c = 0; c < dd; ++c) {
+            float ka = 0.0f, va = 0.0f;
+            for (int t = 0; t < d; ++t) {
+                ka = fmaf(load_as_f32(J->k, J->dtype, (base + j) * d + t), Dk[(size_t)t * dd + c], ka);
+                va = fmaf(load_as_f32(J->v, J->dtype, (base + j) * d + t), Dv[(size_t)t * dd + c], va);
+            }
+            /* stored in the storage type, as the forward reads them */
+            KD[(size_t)j * dd + c] = J->dtype == ORC_BF16 ? bf16_bits_to_f32(f32_to_bf16_bits(ka)) : ka;
+            VD[(size_t)j * dd + c] = J->dtype == ORC_BF16 ? bf16_bits_to_f32(f32_to_bf16_bits(va)) : va;
+        }
+        for (int t = 0; t < d; ++t) {
+            double ka = 0.0, va = 0.0;
+            for (int c = 0; c < dd; ++c) {
+                ka += KD[(size_t)j * dd + c] * (double)Uk[(size_t)c * d + t];
+                va += VD[(size_t)j * dd + c] * (double)Uv[(size_t)c * d + t];
+            }
+            Kl[(size_t)j * d + t] = ka;
+            Vl[(size_t)j * d + t] = va;
+        }
+    }
+    memset(dk, 0, sizeof(double) * (size_t)N * d);
+    memset(dv, 0, sizeof(double) * (size_t)N * d);
+
+    /* Eq. 4 and Eq. 3 backwards, one query row at a time */
+    for (int hh = 0; hh < G; ++hh) {
+        const int h = g * G + hh;
+        const size_t qbase = ((size_t)b * J->Hq + h) * N;
+        for (int i = 0; i < N; ++i) {
+            for (int t = 0; t < d; ++t) {
+                Q[t] = load_as_f32(J->q, J->dtype, (qbase + i) * d + t);
+                dO[t] = load_as_f32(J->dout, J->dtype, (qbase + i) * d + t);
+            }
+            double smax = -INFINITY;
+            for (int j = 0; j <= i; ++j) {
+                const double *key = (i - j < w) ? &K[(size_t)j * d] : &Kl[(size_t)j * d];
+                double dot = 0.0;
+                for (int t = 0; t < d; ++t)
+                    dot += Q[t] * key[t];
+                p[j] = J->scale * dot;
+                if (p[j] > smax)
+                    smax = p[j];
+            }
+            double denom = 0.0;
+            for (int j = 0; j <= i; ++j) {
+                p[j] = exp(p[j] - smax);
+                denom += p[j];
+            }
+            double Di = 0.0;  /* sum_l p_il dP_il */
+            for (int j = 0; j <= i; ++j) {
+                p[j] /= denom;
+                const double *val = (i - j < w) ? &V[(size_t)j * d] : &Vl[(size_t)j * d];
+                double dot = 0.0;
+                for (int t = 0; t < d; ++t)
+                    dot += dO[t] * val[t];
+                dp[j] = dot;
+                Di += p[j] * dot;
+            }
+            double *dqi = J->dq + (qbase + i) * d;
+            for (int t = 0; t < d; ++t)
+                dqi[t] = 0.0;
+            for (int j = 0; j <= i; ++j) {
+                const int loc = i - j < w;
+                const double ds = p[j] * (dp[j] - Di);
+                const double *key = loc ? &K[(size_t)j * d] : &Kl[(size_t)j * d];
+                double *dkey = loc ? &dk[(size_t)j * d] : &dKl[(size_t)j * d];
+                double *dval = loc ? &dv[(size_t)j * d] : &dVl[(size_t)j * d];
+                for (int t = 0; t < d; ++t) {
+                    dqi[t] += J->scale * ds * key[t];
+                    dkey[t] += J->scale * ds * Q[t];
+                    dval[t] += p[j] * dO[t];
+                }
+            }
+        }
+    }
+
+    /* Eq. 2 and Eq. 1 backwards, per token */
+    memset(wp, 0, sizeof(double) * 4 * (size_t)d * dd);
+    double *dkd = malloc(sizeof(double) * (size_t)dd), *dvd = malloc(sizeof(double) * (size_t)dd);
+    for (int j = 0; j < N; ++j) {
+        for (int c = 0; c < dd; ++c) {
+            double a = 0.0, e = 0.0;
+            for (int t = 0; t < d; ++t) {
+                a += dKl[(size_t)j * d + t] * (double)Uk[(size_t)c * d + t];
+                e += dVl[(size_t)j * d + t] * (double)Uv[(size_t)c * d + t];
+                dUk[(size_t)c * d + t] += KD[(size_t)j * dd + c] * dKl[(size_t)j * d + t];
+                dUv[(size_t)c * d + t] += VD[(size_t)j * dd + c] * dVl[(size_t)j * d + t];
+            }
+            dkd[c] = a;
+            dvd[c] = e;
+        }
+        for (int t = 0; t < d; ++t)
+            for (int c = 0; c < dd; ++c) {
+                dk[(size_t)j * d + t] += dkd[c] * (double)Dk[(size_t)t * dd + c];
+                dv[(size_t)j * d + t] += dvd[c] * (double)Dv[(size_t)t * dd + c];
+                dDk[(size_t)t * dd + c] += K[(size_t)j * d + t] * dkd[c];
+                dDv[(size_t)t * dd + c] += V[(size_t)j * d + t] * dvd[c];
+            }
+    }
+    free(dkd);
+    free(dvd);
+    free(K);
+    free(V);
+    free(KD);
+    free(VD);
+    free(Kl);
+    free(Vl);
+    free(dKl);
+    free(dVl);
+    free(p);
+    free(dp);
+    free(Q);
+    free(dO);
+}
+
+static void *bwd_worker(void *arg)
+{
+    const bwd_job *J = (const bwd_job *)arg;
+    const int units = J->B * J->Hkv;
+    for (int u = J->tid; u < units; u += J->nthreads)
+        bwd_unit(J, u / J->Hkv, u % J->Hkv);
+    return NULL;
+}
+
+/*
+ * Gradients of the causal forward over positions 0..N-1 (the training forward
+ * of Sec. 2.3) for the output gradient dout [B][Hq][N][d] (storage type):
+ *   dq [B][Hq][N][d], dk, dv [B][Hkv][N][d], and per KV head
+ *   dDk, dDv [Hkv][d][dd], dUk, dUv [Hkv][dd][d], all fp64.
+ * Inputs as dar_oracle_attention with Dk, Dv (Eq. 1) in place of kd, vd.
+ * Returns 0, or -1 on a bad argument.  Threads run over (b, g) units; the
+ * projection gradients are summed over units in a fixed order.
+ */
+int dar_oracle_backward(int dtype, int B, int Hq, int Hkv, int N, int d, int dd, int w,
+                        const void *q, const void *k, const void *v, const float *Dk,
+                        const float *Uk, const float *Dv, const float *Uv, const void *dout,
+                        double scale, double *dq, double *dk, double *dv, double *dDk,
+                        double *dUk, double *dDv, double *dUv, int nthreads)
+{
+    if (B < 1 || Hkv < 1 || Hq < Hkv || Hq % Hkv || N < 1 || d < 1 || dd < 1 || w < 0 ||
+        (dtype != ORC_F32 && dtype != ORC_BF16))
+        return -1;
+    if (nthreads < 1)
+        nthreads = 1;
+    const size_t wd = (size_t)d * dd;
+    double *wpart = malloc(sizeof(double) * (size_t)B * Hkv * 4 * wd);
+    bwd_job *jobs = malloc(sizeof(bwd_job) * (size_t)nthreads);
+    pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
+    for (int t = 0; t < nthreads; ++t) {
+        bwd_job J = {dtype, B, Hq, Hkv, N, d, dd, w, q, k, v, dout, Dk, Uk, Dv, Uv, scale,
+                     dq, dk, dv, wpart, nthreads, t};
+        jobs[t] = J;
+    }
+    for (int t = 1; t < nthreads; ++t)
+        pthread_create(&th[t], NULL, bwd_worker, &jobs[t]);
+    bwd_worker(&jobs[0]);
+    for (int t = 1; t < nthreads; ++t)
+        pthread_join(th[t], NULL);
+    for (int g = 0; g < Hkv; ++g)
+        for (size_t e = 0; e < wd; ++e) {
+            double s0 = 0.0, s1 = 0.0, s2 = 0.0, s3 = 0.0;
+            for (int b = 0; b < B; ++b) {
+                const double *wp = wpart + ((size_t)b * Hkv + g) * 4 * wd;
+                s0 += wp[e];
+                s1 += wp[wd + e];
+                s2 += wp[2 * wd + e];
+                s3 += wp[3 * wd + e];
+            }
+            dDk[g * wd + e] = s0;
+            dUk[g * wd + e] = s1;
+            dDv[g * wd + e] = s2;
+            dUv[g * wd + e] = s3;
+        }
+    free(wpart);
+    free(jobs);
+    free(th);
+    return 0;
+}
