@@ -252,10 +252,11 @@ def time_graph(torch, g, stream, before=None):
     return a.elapsed_time(b)
 
 
-def decode_only_point(torch, dar, I, W, cfg, K, l2, dev, stream, hbm_peak):
+def decode_only_point(torch, dar, I, W, cfg, K, l2, dev, stream, hbm_peak, direct=False):
     """GB/s of graph-timed dar_attn_decode calls on one decode workload (the
     cache is read, never written, so replays are identical); caches rotate
-    over enough copies to exceed 4x L2."""
+    over enough copies to exceed 4x L2.  direct: dar_attn_decode_direct (the
+    global path of Sec. 5's direct variant; same cache bytes)."""
     wl = W.DecodeWorkload(cfg)
     lens = W.download(wl.cache.seq_lens).astype(np.int64)
     nbytes = W.decode_step_bytes(cfg, lens)
@@ -263,8 +264,13 @@ def decode_only_point(torch, dar, I, W, cfg, K, l2, dev, stream, hbm_peak):
     caches = [wl.cache] + [clone_cache(dar, wl.cache) for _ in range(R - 1)]
     outs = [torch.empty_like(wl.q) for _ in range(R)]
     ws = [wl.workspace] + [dar.decode_workspace(c, cfg.Hq) for c in caches[1:]]
-    g = graph_of(torch, lambda j: dar.dar_attn_decode(caches[j % R], wl.q, wl.Uk, wl.Uv, ws[j % R], out=outs[j % R]),
-                 K)
+    if direct:
+        qd = W.upload(I.direct_queries(cfg), cfg.dtype)
+        g = graph_of(torch, lambda j: dar.dar_attn_decode_direct(caches[j % R], wl.q, qd, wl.Uv, ws[j % R],
+                                                                 out=outs[j % R]), K)
+    else:
+        g = graph_of(torch, lambda j: dar.dar_attn_decode(caches[j % R], wl.q, wl.Uk, wl.Uv, ws[j % R],
+                                                          out=outs[j % R]), K)
     ms = time_graph(torch, g, stream, before=lambda: flush_l2(torch, dev, 2 * l2))
     us = 1e3 * ms / K
     gbs = nbytes / (us * 1e-6) / 1e9
@@ -345,6 +351,46 @@ def prefill_section(args, torch, dar, W, I, dev, stream, tc_peak, peak_src, loca
             "tensor": {"achieved": round(p_tflops, 2), "peak": tc_peak, "unit": "TFLOP/s",
                        "frac": round(p_tflops / tc_peak, 4), "peak_source": f"{peak_src} bf16 dense (burst)"},
             "clocks": clk.summary()}
+
+
+def direct_prefill_point(args, torch, dar, W, I, dev, stream):
+    """The 410M-like prefill with the direct global path of Sec. 5
+    (dar_attn_prefill_direct): median CUDA-event time of K calls, sampled rows
+    checked against the oracle."""
+    import oracle
+    pcfg = I.PREFILL_410M
+    pw = W.PrefillWorkload(pcfg)
+    qd_host = I.direct_queries(pcfg)
+    qd = W.upload(qd_host, pcfg.dtype)
+
+    def call():
+        dar.dar_attn_prefill_direct(pw.q, qd, pw.k, pw.v, pw.Dk, pw.Dv, pw.Uv, pcfg.w, out=pw.out,
+                                    workspace=pw.workspace, stream=stream)
+
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(max(3, min(args.steps, 10)))]
+    for a, b in ev:
+        a.record(stream)
+        call()
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms = float(np.median([a.elapsed_time(b) for a, b in ev]))
+    rng = np.random.default_rng(2)
+    rows = np.array([(int(rng.integers(pcfg.B)), int(rng.integers(pcfg.Hq)), int(i))
+                     for i in [0, pcfg.w - 1, pcfg.w, pcfg.N - 1] + list(rng.integers(0, pcfg.N, 4))])
+    x = pw.host
+    want = oracle.prefill_direct(x["q"], qd_host, x["k"], x["v"], x["Dk"], x["Dv"], x["Uv"], pcfg.w, pcfg.dtype,
+                                 rows=rows)
+    got = W.to_f64(W.download(pw.out), pcfg.dtype)[rows[:, 0], rows[:, 1], rows[:, 2]]
+    err = float(np.abs(got - want).max())
+    if not err <= TOL_BF16:
+        raise RuntimeError(f"direct prefill output differs from the oracle: max-abs {err}")
+    flops = W.prefill_flops(pcfg)  # the direct path does the same contractions, minus the q Uk^T lift
+    return {"workload": pcfg.name, "ms": round(ms, 4), "tflops": round(flops / (ms * 1e-3) / 1e12, 2),
+            "exps_per_call": W.prefill_exps(pcfg), "oracle_max_abs_err": round(err, 5)}
 
 
 def verify_steps(torch, dar, oracle, I, W, cfg, wls, outs, knew_host, vnew_host, n_appended, R):
@@ -567,7 +613,11 @@ def run_ours(args, world, rank, local):
         gqa = decode_only_point(torch, dar, I, W, I.DECODE_1B_GQA, K, l2, dev, stream, hbm_peak)
         sweep = [decode_only_point(torch, dar, I, W, I.sweep_point(k), K, l2, dev, stream, hbm_peak)
                  for k in range(len(I.SWEEP_W) * len(I.SWEEP_DD))]
-        extra = {"decode_1b_gqa": gqa, "sweep": sweep,
+        direct = {"decode": decode_only_point(torch, dar, I, W, cfg, K, l2, dev, stream, hbm_peak, direct=True),
+                  "prefill": direct_prefill_point(args, torch, dar, W, I, dev, stream),
+                  "what": "direct lower-dimensional global attention (Sec. 5): dar_attn_decode_direct, "
+                          "dar_attn_prefill_direct"}
+        extra = {"decode_1b_gqa": gqa, "sweep": sweep, "direct_variant": direct,
                  "note": "graph of K dar_attn_decode calls, rotating cache copies > 4x L2, L2 flushed before"}
 
     cpu = None

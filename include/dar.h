@@ -252,6 +252,40 @@ dar_status dar_prefill_chunk(const dar_cache *cache, int32_t Hq, int32_t n, cons
                              const float *Dv, const float *Uv, float scale, void *out, void *workspace,
                              size_t workspace_bytes, void *stream);
 
+/*
+ * Direct lower-dimensional global attention (Sec. 5, "Direct lower-dimensional
+ * global attention": the global path runs entirely in d_down instead of
+ * lifting h^D back to d).  Local pairs (i - j < w, Eq. 3) are unchanged:
+ * scale * q . k_j with full-d keys and values.  Global pairs score
+ * scale_down * q^D . k^D_j, where q^D is a d_down query of the row's own
+ * (qd) and k^D = k Dk is the cached bottleneck key (Eq. 1); their values
+ * v^D_j = v Dv enter as v^D_j Wo, Wo [Hkv][d_down][d] the global path's
+ * output map to d.  One softmax covers both paths (Eq. 4 carried over):
+ *   o_i = (sum_local p_j v_j + (sum_global p_j v^D_j) Wo) / sum_j p_j.
+ * scale_down <= 0 selects 1/sqrt(d_down).  The global path computes
+ * scale * (qd * scale_down / scale) . k^D, so on the bf16 tensor-core paths
+ * the rescaled qd is rounded to bf16 once, as q~ is in the standard form.
+ */
+
+/* As dar_attn_prefill with the direct global path: qd [B][Hq][N][d_down] T,
+ * Wo in place of Uv; no Uk.  Same workspace (dar_prefill_workspace_bytes),
+ * status and error behaviour. */
+dar_status dar_attn_prefill_direct(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
+                                   int32_t d, int32_t d_down, int32_t w, const void *q, const void *qd,
+                                   const void *k, const void *v, const float *Dk, const float *Dv,
+                                   const float *Wo, float scale, float scale_down, void *out,
+                                   void *workspace, size_t workspace_bytes, int32_t *status,
+                                   void *stream);
+
+/* As dar_attn_decode with the direct global path: qd [B][Hq][d_down] T (16-byte
+ * aligned), Wo in place of Uv; no Uk.  Same cache (the pages hold k^D, v^D of
+ * Eq. 1, written by dar_cache_append), workspace (dar_decode_workspace_bytes)
+ * and error behaviour; both kernels start after all earlier work on the
+ * stream has finished. */
+dar_status dar_attn_decode_direct(const dar_cache *cache, int32_t Hq, const void *q, const void *qd,
+                                  const float *Wo, float scale, float scale_down, void *out,
+                                  void *workspace, size_t workspace_bytes, void *stream);
+
 /* Message for the last non-OK return on this thread ("" if none). */
 const char *dar_last_error(void);
 

@@ -292,6 +292,27 @@ dar_status dar_attn_decode(const dar_cache *cache, int32_t Hq, const void *q, co
                      "dar_attn_decode launch");
 }
 
+dar_status dar_attn_decode_direct(const dar_cache *cache, int32_t Hq, const void *q, const void *qd,
+                                  const float *Wo, float scale, float scale_down, void *out,
+                                  void *workspace, size_t workspace_bytes, void *stream)
+{
+    dar::DecodeArgs a;
+    bool empty = false;
+    // Wo stands in for Uk in the shared checks; Uk is never read here
+    dar_status s = prepare_decode(cache, Hq, q, Wo, Wo, scale, out, workspace, workspace_bytes, &a, &empty);
+    if (s != DAR_OK || empty)
+        return s;
+    if (!qd)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(qd))
+        return fail(DAR_ERR_INVALID_ARG, "qd must be 16-byte aligned");
+    a.qd = qd;
+    a.qd_ratio = default_scale(scale_down, cache->d_down) / default_scale(scale, cache->d);
+    a.prep_overlaps_prev = 0;
+    return from_cuda(dar::launch_decode(cache->dtype, cache->d_down, a, static_cast<cudaStream_t>(stream)),
+                     "dar_attn_decode_direct launch");
+}
+
 dar_status dar_decode_step(const dar_cache *cache, const void *k_new, const void *v_new, int32_t n,
                            const int32_t *n_per_seq, const float *Dk, const float *Dv, int32_t Hq,
                            const void *q, const float *Uk, const float *Uv, float scale, void *out,
@@ -405,11 +426,17 @@ size_t dar_prefill_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hkv, int3
            align256(rows * dar::prefill_vd_stride(dtype, d_down) * esize(dtype));
 }
 
-dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
-                            int32_t d, int32_t d_down, int32_t w, const void *q, const void *k,
-                            const void *v, const float *Dk, const float *Uk, const float *Dv,
-                            const float *Uv, float scale, void *out, void *workspace,
-                            size_t workspace_bytes, int32_t *status, void *stream)
+}  // extern "C"
+
+namespace {
+
+// dar_attn_prefill (qd == NULL: q~ = q Uk^T) and dar_attn_prefill_direct
+// (qd given, Uk unused, global scores at scale_down).
+dar_status prefill_common(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N, int32_t d,
+                          int32_t d_down, int32_t w, const void *q, const void *qd, const void *k,
+                          const void *v, const float *Dk, const float *Uk, const float *Dv, const float *Uv,
+                          float scale, float scale_down, void *out, void *workspace, size_t workspace_bytes,
+                          int32_t *status, void *stream)
 {
     dar_status s = check_dims(dtype, d, d_down);
     if (s != DAR_OK)
@@ -420,11 +447,13 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
         return ok();
     if ((long long)B * Hq > 65535 || (long long)B * Hkv > 65535)
         return fail(DAR_ERR_UNSUPPORTED, "B*Hq=%lld > 65535", (long long)B * Hq);
+    if (!Uk)
+        Uk = Uv;  // the direct variant has no Uk; never read then
     if (!q || !k || !v || !Dk || !Uk || !Dv || !Uv || !out || !workspace)
         return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) ||
         !aligned16(workspace) || !aligned16(Dk) || !aligned16(Dv) || !aligned16(Uk) ||
-        !aligned16(Uv))
+        !aligned16(Uv) || (qd && !aligned16(qd)))
         return fail(DAR_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
     const size_t need = dar_prefill_workspace_bytes(dtype, B, Hkv, N, d_down);
     if (workspace_bytes < need)
@@ -457,9 +486,40 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
     a.kd_stride = kstride;
     a.vd_stride = vstride;
     a.qscale = default_scale(scale, d) * kLog2e;
+    a.qd = qd;
+    a.qd_ratio = qd ? default_scale(scale_down, d_down) / default_scale(scale, d) : 1.f;
     if (dtype == DAR_BF16)
         return from_cuda(dar::launch_prefill_tc(d_down, a, st), "dar_attn_prefill (tcgen05) launch");
     return from_cuda(dar::launch_prefill_simt(dtype, d_down, a, st), "dar_attn_prefill launch");
+}
+
+}  // namespace
+
+extern "C" {
+
+dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
+                            int32_t d, int32_t d_down, int32_t w, const void *q, const void *k,
+                            const void *v, const float *Dk, const float *Uk, const float *Dv,
+                            const float *Uv, float scale, void *out, void *workspace,
+                            size_t workspace_bytes, int32_t *status, void *stream)
+{
+    if (!Uk && B > 0 && N > 0)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    return prefill_common(dtype, B, Hq, Hkv, N, d, d_down, w, q, nullptr, k, v, Dk, Uk, Dv, Uv, scale, 0.f, out,
+                          workspace, workspace_bytes, status, stream);
+}
+
+dar_status dar_attn_prefill_direct(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
+                                   int32_t d, int32_t d_down, int32_t w, const void *q, const void *qd,
+                                   const void *k, const void *v, const float *Dk, const float *Dv,
+                                   const float *Wo, float scale, float scale_down, void *out,
+                                   void *workspace, size_t workspace_bytes, int32_t *status,
+                                   void *stream)
+{
+    if (!qd && B > 0 && N > 0)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    return prefill_common(dtype, B, Hq, Hkv, N, d, d_down, w, q, qd, k, v, Dk, nullptr, Dv, Wo, scale, scale_down,
+                          out, workspace, workspace_bytes, status, stream);
 }
 
 }  // extern "C"

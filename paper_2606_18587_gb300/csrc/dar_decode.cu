@@ -158,7 +158,9 @@ constexpr size_t decode_smem_bytes(int B)
 // --------------------------------------------------------------------- prep
 
 // q~ = q Uk^T for every (b, h) row, one row per warp (fp32, four partial sums
-// over t mod 4), and zeroed group counters.  Neither depends on the cache, so
+// over t mod 4), and zeroed group counters.  In the direct variant of Sec. 5
+// (a.qd set) q~ is the row's own d_down query times scale_down / scale, so the
+// stream kernel's global scores scale * q~ . k^D are scale_down * q^D . k^D.  Neither depends on the cache, so
 // when launched programmatically after the cache append (which writes neither
 // q nor Uk) this kernel runs while the append finishes; it waits for the
 // kernel before it before exiting, so the stream kernel, which waits for this
@@ -172,6 +174,11 @@ __global__ void __launch_bounds__(kPrepThreads) decode_prep_kernel(DecodeArgs a)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int rows = a.B * a.Hq;
     for (int row = blockIdx.x * kWarps + warp; row < rows; row += gridDim.x * kWarps) {
+        if (a.qd) {  // direct variant: the row's own d_down query, rescaled to the local scale
+            for (int c = lane; c < DD; c += 32)
+                a.qt[(size_t)row * DD + c] = to_f32(static_cast<const T *>(a.qd)[(size_t)row * DD + c]) * a.qd_ratio;
+            continue;
+        }
         const T *qrow = static_cast<const T *>(a.q) + (size_t)row * kHeadDim;
         const float q0 = to_f32(qrow[lane]), q1 = to_f32(qrow[lane + 32]);
         const int g = (row % a.Hq) / a.G;

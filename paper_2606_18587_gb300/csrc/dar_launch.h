@@ -38,6 +38,11 @@ struct DecodeArgs {
     int32_t *counters;  // [B][Hkv][HS] finished stages per group, then the pool's claim counter
     int B, Hq, Hkv, G, GH, HS, w, maxp, num_pages;
     float qscale;  // scale * log2(e)
+    // direct lower-dimensional global attention (Sec. 5): the d_down query of
+    // each row [B][Hq][dd] T, used as q~ after multiplying by qd_ratio =
+    // scale_down / scale (nullptr: q~ = q Uk^T)
+    const void *qd = nullptr;
+    float qd_ratio = 1.f;
     // the kernel before the decode on the stream is this library's cache
     // append (which writes neither q nor Uk): the decode's query-side set-up
     // may overlap it
@@ -52,6 +57,11 @@ struct PrefillArgs {
     int32_t *status;        // device error word or nullptr
     int B, Hq, Hkv, N, w, dd, kd_stride, vd_stride;
     float qscale;  // scale * log2(e)
+    // direct lower-dimensional global attention (Sec. 5): the d_down query of
+    // each row [B][Hq][N][dd] T, used as q~ after multiplying by qd_ratio =
+    // scale_down / scale (nullptr: q~ = q Uk^T)
+    const void *qd = nullptr;
+    float qd_ratio = 1.f;
     // chunked prefill over a cache (dar_prefill_chunk): query b sits at
     // position pos0[b] + r, r < n; local keys come from a window buffer of NW
     // rows per (b, KV head), starting at the 64-aligned position below

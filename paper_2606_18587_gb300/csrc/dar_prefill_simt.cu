@@ -6,7 +6,8 @@
 // all-global (every pair has i - j >= w), all-local (every pair i - j < w) or a
 // band tile that holds both kinds; the element rule is Eq. 3 (local iff
 // i - j < w).  Local pairs score q . k (d = 64); global pairs score
-// q~ . k^D with q~ = q Uk^T (d_down).  One online softmax covers both kinds,
+// q~ . k^D with q~ = q Uk^T (d_down; in the direct variant of Sec. 5, q~ is
+// the row's own d_down query times scale_down / scale).  One online softmax covers both kinds,
 // values accumulate in d (local) and d_down (global) and the global part is
 // lifted once with Uv in the epilogue:  o = (o_loc + o_glob Uv) / l.
 #include "dar_common.cuh"
@@ -57,6 +58,13 @@ __global__ void __launch_bounds__(256) prefill_simt_kernel(PrefillArgs a)
     __syncthreads();
     for (int idx = tid; idx < kSimtRows * DD; idx += 256) {
         const int rr = idx / DD, c = idx % DD;
+        if (a.qd) {  // direct variant (Sec. 5): the row's own d_down query, at the global scale
+            Qt[rr * LDD + c] = (i0 + rr < N)
+                ? to_f32(static_cast<const T *>(a.qd)[(((size_t)b * a.Hq + h) * N + i0 + rr) * DD + c]) *
+                      a.qd_ratio * a.qscale
+                : 0.f;
+            continue;
+        }
         float acc = 0.f;
         for (int t = 0; t < kHeadDim; ++t)
             acc = fmaf(Qs[rr * kSimtLd + t], Uk[c * kHeadDim + t], acc);

@@ -249,6 +249,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     constexpr int VR = kOnes ? vd_row<DP>() : DP;  // elements per v^D row in a stage
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int w = a.w;
+    const bool direct = a.qd != nullptr;  // Sec. 5 direct variant: q~ given, not absorbed
     const int bh = blockIdx.x, b = bh / a.Hq, h = bh % a.Hq, g = h / (a.Hq / a.Hkv);
     const int L0 = CH ? __ldg(a.pos0 + b) : 0;  // position of query row 0
     const int nrows = CH ? a.n : a.N;            // query rows per (b, h)
@@ -361,17 +362,20 @@ __global__ void __launch_bounds__(kThreads, 2)
             const uint64_t dUKB = smem_desc(smem_u32(sm + Ly::UKB), 16, 1024, kSw128);
             const uint64_t dStgD = smem_desc(smem_u32(sm + Ly::STG), 16, 8 * DP * 2, dp_swizzle<DP>());
             const uint32_t tS = tmem + Tm::S, tOL = tmem + Tm::OL;
-            // q~ = Q Uk^T into the O_loc columns
+            // q~ = Q Uk^T into the O_loc columns (the direct variant reads its
+            // d_down queries from memory instead)
             ok = wait_all(q_full, 0) && wait_all(ukb_ready, 0);
             if (ok) {
                 tc_fence_after();
-                if (elect_one()) {
+                if (!direct) {
+                    if (elect_one()) {
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        mma_f16_ss(tOL, dQ + 2 * kk, dUKB + 2 * kk, idQT, kk > 0);
-                    mma_commit(qt_mma);
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_f16_ss(tOL, dQ + 2 * kk, dUKB + 2 * kk, idQT, kk > 0);
+                        mma_commit(qt_mma);
+                    }
+                    __syncwarp();
                 }
-                __syncwarp();
                 ok = wait_all(qt_ready, 0);
                 tc_fence_after();
             }
@@ -480,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         // ---- set-up: Uk as a bf16 operand, the ones block, Uv for the epilogue
         {
             const float *Ukg = a.Uk + (size_t)g * a.dd * 64;
-            for (int idx = stid; idx < DP * 8; idx += kSoftmaxThreads) {  // row c, chunk ch of 8 values
+            for (int idx = direct ? DP * 8 : stid; idx < DP * 8; idx += kSoftmaxThreads) {  // row c, chunk ch of 8 values
                 const int c = idx / 8, ch = idx % 8;
                 uint4 v = make_uint4(0u, 0u, 0u, 0u);
                 if (c < a.dd) {
@@ -507,20 +511,40 @@ __global__ void __launch_bounds__(kThreads, 2)
             const bool r = mbar_wait(bar, parity, abort_flag);
             return __all_sync(0xffffffffu, r) != 0;
         };
-        bool ok = wait_uniform(qt_mma, 0);
+        bool ok = direct || wait_uniform(qt_mma, 0);
+        if (ok && direct) {
+            // the direct variant's d_down queries, times scale_down / scale, as
+            // bf16 operand rows (zero past the end and past d_down)
+            unsigned char *qrow = sm + Ly::QT;
+            const bf16 *qdh = static_cast<const bf16 *>(a.qd) + ((size_t)b * a.Hq + h) * nrows * a.dd;
+            auto pair = [&](int i, int e) -> uint32_t {
+                if (i >= N || e >= a.dd)
+                    return 0u;
+                const bf16 *p = qdh + (size_t)(i - L0) * a.dd + e;
+                return pack_bf16(__bfloat162float(p[0]) * a.qd_ratio, __bfloat162float(p[1]) * a.qd_ratio);
+            };
+#pragma unroll
+            for (int ch = 0; ch < DP / 8; ++ch) {
+                st_swz4<DP * 2>(qrow, ra, ch, q4, pair(iA, 8 * ch + 2 * q4));
+                st_swz4<DP * 2>(qrow, ra + 8, ch, q4, pair(iB, 8 * ch + 2 * q4));
+            }
+        }
         if (ok) {
             tc_fence_after();
             // q~ (fp32, TMEM) -> bf16 operand rows in shared memory; then clear the accumulators
             unsigned char *qrow = sm + Ly::QT;
+            if (!direct) {
 #pragma unroll
-            for (int c = 0; c < DP; c += 16) {
-                uint32_t r[8];
-                tmem_ld_16x256b_x2(tl + Tm::OL + c, r);
+                for (int c = 0; c < DP; c += 16) {
+                    uint32_t r[8];
+                    tmem_ld_16x256b_x2(tl + Tm::OL + c, r);
 #pragma unroll
-                for (int k = 0; k < 2; ++k) {
-                    st_swz4<DP * 2>(qrow, ra, c / 8 + k, q4, pack_bf16(__uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1])));
-                    st_swz4<DP * 2>(qrow, ra + 8, c / 8 + k, q4,
-                                    pack_bf16(__uint_as_float(r[4 * k + 2]), __uint_as_float(r[4 * k + 3])));
+                    for (int k = 0; k < 2; ++k) {
+                        st_swz4<DP * 2>(qrow, ra, c / 8 + k, q4,
+                                        pack_bf16(__uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1])));
+                        st_swz4<DP * 2>(qrow, ra + 8, c / 8 + k, q4,
+                                        pack_bf16(__uint_as_float(r[4 * k + 2]), __uint_as_float(r[4 * k + 3])));
+                    }
                 }
             }
             uint32_t z[8];

@@ -70,6 +70,9 @@ def load_library(path: str = LIB_PATH):
         "dar_prefill_chunk": ([CP, I32, I32, P, P, P, P, P, P, P, F, P, P, SZ, P], ctypes.c_int),
         "dar_attn_prefill": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, P, P,
                               SZ, P, P], ctypes.c_int),
+        "dar_attn_prefill_direct": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, F,
+                                     P, P, SZ, P, P], ctypes.c_int),
+        "dar_attn_decode_direct": ([CP, I32, P, P, P, F, F, P, P, SZ, P], ctypes.c_int),
         "dar_last_error": ([], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -294,6 +297,58 @@ def dar_attn_prefill(q, k, v, Dk, Uk, Dv, Uv, w, scale=0.0, out=None, workspace=
     _check(load_library().dar_attn_prefill(
         _code(q), B, Hq, Hkv, N, d, dd, int(w), _ptr(q), _ptr(k), _ptr(v), _ptr(Dk), _ptr(Uk), _ptr(Dv), _ptr(Uv),
         float(scale), _ptr(out), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+    return out
+
+
+def dar_attn_prefill_direct(q, qd, k, v, Dk, Dv, Wo, w, scale=0.0, scale_down=0.0, out=None, workspace=None,
+                            status=None, stream=None):
+    """Causal forward with the direct lower-dimensional global path (Sec. 5):
+    ``qd [B,Hq,N,d_down]`` the global path's queries, ``Wo [Hkv,d_down,d]`` its
+    output map; otherwise as :func:`dar_attn_prefill`."""
+    _dev(q, "q")
+    _dev(qd, "qd", q.dtype)
+    _dev(k, "k", q.dtype)
+    _dev(v, "v", q.dtype)
+    for name, t in (("Dk", Dk), ("Dv", Dv), ("Wo", Wo)):
+        _dev(t, name, torch.float32)
+    B, Hq, N, d = q.shape
+    Hkv = k.shape[1]
+    dd = Dk.shape[2]
+    if tuple(qd.shape) != (B, Hq, N, dd):
+        raise ValueError(f"qd has shape {tuple(qd.shape)}, expected {(B, Hq, N, dd)}")
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", q.dtype)
+    if workspace is None:
+        workspace = torch.empty(max(1, dar_prefill_workspace_bytes(q.dtype, B, Hkv, N, dd)),
+                                dtype=torch.uint8, device=q.device)
+    _dev(workspace, "workspace")
+    if status is not None:
+        _dev(status, "status", torch.int32)
+    _check(load_library().dar_attn_prefill_direct(
+        _code(q), B, Hq, Hkv, N, d, dd, int(w), _ptr(q), _ptr(qd), _ptr(k), _ptr(v), _ptr(Dk), _ptr(Dv), _ptr(Wo),
+        float(scale), float(scale_down), _ptr(out), _ptr(workspace), workspace.numel(), _ptr(status),
+        _stream(stream)))
+    return out
+
+
+def dar_attn_decode_direct(cache: DarCache, q, qd, Wo, workspace, scale=0.0, scale_down=0.0, out=None,
+                           stream=None):
+    """One decode step with the direct lower-dimensional global path (Sec. 5):
+    ``qd [B,Hq,d_down]`` the global path's queries, ``Wo [Hkv,d_down,d]`` its
+    output map; otherwise as :func:`dar_attn_decode`."""
+    _dev(q, "q", cache.dtype)
+    _dev(qd, "qd", cache.dtype)
+    _dev(Wo, "Wo", torch.float32)
+    _dev(workspace, "workspace")
+    if tuple(qd.shape) != (q.shape[0], q.shape[1], cache.d_down):
+        raise ValueError(f"qd has shape {tuple(qd.shape)}, expected {(q.shape[0], q.shape[1], cache.d_down)}")
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", cache.dtype)
+    _check(load_library().dar_attn_decode_direct(
+        cache.struct, q.shape[1], _ptr(q), _ptr(qd), _ptr(Wo), float(scale), float(scale_down), _ptr(out),
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
     return out
 
 

@@ -30,7 +30,7 @@ _GEN_LIB = os.path.join(_HERE, "libdar_inputs.so")
 _gen = None
 
 # tensor stream ids
-S_Q, S_K, S_V, S_DK, S_DV, S_UK, S_UV, S_LENS, S_PAGES, S_QDEC, S_KNEW, S_VNEW = range(1, 13)
+S_Q, S_K, S_V, S_DK, S_DV, S_UK, S_UV, S_LENS, S_PAGES, S_QDEC, S_KNEW, S_VNEW, S_QD = range(1, 14)
 _KIND = {"f32": 0, "bf16": 1, "f64": 2, "uniform": 3}
 _NP = {"f32": np.float32, "bf16": np.uint16, "f64": np.float64, "uniform": np.float64}
 
@@ -158,6 +158,15 @@ def prefill_inputs(cfg: Prefill):
     v = normal_array(s, S_V, (cfg.B, cfg.Hkv, cfg.N, cfg.d), dtype=cfg.dtype)
     Dk, Uk, Dv, Uv = projections(s, cfg.Hkv, cfg.d, cfg.dd)
     return dict(q=q, k=k, v=v, Dk=Dk, Uk=Uk, Dv=Dv, Uv=Uv)
+
+
+def direct_queries(cfg, step: int = 0) -> np.ndarray:
+    """The d_down queries of the direct global path (Sec. 5), N(0, 1) in the
+    storage type: [B, Hq, N, dd] for a prefill config, [B, Hq, dd] for a decode
+    config (at one decode step)."""
+    if isinstance(cfg, Prefill):
+        return normal_array(cfg.seed, S_QD, (cfg.B, cfg.Hq, cfg.N, cfg.dd), dtype=cfg.dtype)
+    return normal_array(cfg.seed, S_QD, (cfg.B, cfg.Hq, cfg.dd), dtype=cfg.dtype, sub=step)
 
 
 def decode_lengths(cfg: Decode) -> np.ndarray:
