@@ -393,6 +393,43 @@ def direct_prefill_point(args, torch, dar, W, I, dev, stream):
             "exps_per_call": W.prefill_exps(pcfg), "oracle_max_abs_err": round(err, 5)}
 
 
+def backward_point(args, torch, dar, W, I, dev, stream):
+    """The backward pass (Sec. 2.3 training) of the 410M-like prefill:
+    dar_attn_backward after one forward, median CUDA-event time of a few calls,
+    against the CUDA cores' fp32 FMA peak (the kernels use no tensor cores).
+    The gradients must be finite and bit-identical across calls; their values
+    are checked against the oracle in the GPU tests."""
+    pcfg = I.PREFILL_410M
+    pw = W.PrefillWorkload(pcfg)
+    pw.run()
+    dout = W.upload(I.normal_array(pcfg.seed, I.S_QD, (pcfg.B, pcfg.Hq, pcfg.N, pcfg.d), dtype=pcfg.dtype, sub=1),
+                    pcfg.dtype)
+    ws = torch.empty(dar.dar_attn_backward_workspace_bytes(pw.q.dtype, pcfg.B, pcfg.Hq, pcfg.Hkv, pcfg.N, pcfg.dd),
+                     dtype=torch.uint8, device=dev)
+    grads = dar.dar_attn_backward(pw.q, pw.k, pw.v, pw.Dk, pw.Uk, pw.Dv, pw.Uv, pw.out, dout, pcfg.w, workspace=ws,
+                                  stream=stream)
+    first = {n: t.clone() for n, t in grads.items()}
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(3)]
+    for a, b in ev:
+        a.record(stream)
+        dar.dar_attn_backward(pw.q, pw.k, pw.v, pw.Dk, pw.Uk, pw.Dv, pw.Uv, pw.out, dout, pcfg.w, workspace=ws,
+                              grads=grads, stream=stream)
+        b.record(stream)
+    torch.cuda.synchronize()
+    ms = float(np.median([a.elapsed_time(b) for a, b in ev]))
+    for n, t in grads.items():
+        if not bool(torch.isfinite(t.float()).all()) or not torch.equal(t, first[n]):
+            raise RuntimeError(f"backward gradient {n} is not finite or not repeatable")
+    flops = W.prefill_backward_flops(pcfg)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak = sms * 128 * 2 * SM_MAX_MHZ * 1e6 / 1e12
+    tf = flops / (ms * 1e-3) / 1e12
+    return {"workload": pcfg.name, "ms": round(ms, 3), "tflops": round(tf, 2), "flops_per_call": flops,
+            "roofline": {"bound": "alu", "achieved": round(tf, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
+                         "frac": round(tf / peak, 4),
+                         "peak_source": f"{sms} SMs x 128 fp32 FMA/clk x 2 x {SM_MAX_MHZ:.0f} MHz (nominal)"}}
+
+
 def verify_steps(torch, dar, oracle, I, W, cfg, wls, outs, knew_host, vnew_host, n_appended, R):
     """The timed graph's outputs: for every rotating copy, the last step's
     output equals an eager decode of the same state bit for bit, and sequence
@@ -618,6 +655,7 @@ def run_ours(args, world, rank, local):
                   "what": "direct lower-dimensional global attention (Sec. 5): dar_attn_decode_direct, "
                           "dar_attn_prefill_direct"}
         extra = {"decode_1b_gqa": gqa, "sweep": sweep, "direct_variant": direct,
+                 "backward": backward_point(args, torch, dar, W, I, dev, stream),
                  "note": "graph of K dar_attn_decode calls, rotating cache copies > 4x L2, L2 flushed before"}
 
     cpu = None

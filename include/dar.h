@@ -286,6 +286,32 @@ dar_status dar_attn_decode_direct(const dar_cache *cache, int32_t Hq, const void
                                   const float *Wo, float scale, float scale_down, void *out,
                                   void *workspace, size_t workspace_bytes, void *stream);
 
+/*
+ * Gradients of the causal forward of dar_attn_prefill (training, Sec. 2.3:
+ * the standard next-token objective; backpropagation updates W_down and W_up
+ * from the positions whose queries reach a token through the global path).
+ * Given the forward's inputs, its output `out` and the loss gradient `dout`
+ * [B][Hq][N][d] T, writes
+ *   dq [B][Hq][N][d], dk, dv [B][Hkv][N][d] (T),
+ *   dDk, dDv [Hkv][d][d_down], dUk, dUv [Hkv][d_down][d] (fp32),
+ * each overwritten (not accumulated).  The derivative is that of Eq. 1-4 with
+ * the stored k^D, v^D's rounding to T not differentiated (the bottleneck
+ * projections get the gradient of the unrounded product), and D_i = dout_i .
+ * out_i taken from the given forward output.  fp32 arithmetic on the CUDA
+ * cores for both storage types; no tensor cores.  The workspace
+ * (dar_attn_backward_workspace_bytes, no initialisation) holds per-row and
+ * per-token intermediates; outputs must not overlap inputs.  Deterministic:
+ * every sum runs in a fixed order.  Shapes as dar_attn_prefill; B*Hq <= 65535.
+ */
+size_t dar_attn_backward_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
+                                         int32_t N, int32_t d_down);
+dar_status dar_attn_backward(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N, int32_t d,
+                             int32_t d_down, int32_t w, const void *q, const void *k, const void *v,
+                             const float *Dk, const float *Uk, const float *Dv, const float *Uv,
+                             const void *out, const void *dout, float scale, void *dq, void *dk, void *dv,
+                             float *dDk, float *dUk, float *dDv, float *dUv, void *workspace,
+                             size_t workspace_bytes, void *stream);
+
 /* Message for the last non-OK return on this thread ("" if none). */
 const char *dar_last_error(void);
 

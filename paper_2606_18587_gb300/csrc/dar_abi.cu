@@ -509,6 +509,66 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
                           workspace, workspace_bytes, status, stream);
 }
 
+size_t dar_attn_backward_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
+                                         int32_t d_down)
+{
+    if (!dtype_valid(dtype) || B < 0 || Hkv < 1 || Hq < Hkv || Hq % Hkv || N < 0 || !dd_supported(d_down))
+        return 0;
+    return dar::backward_workspace_bytes(dtype, B, Hq, Hkv, N, d_down);
+}
+
+dar_status dar_attn_backward(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N, int32_t d,
+                             int32_t d_down, int32_t w, const void *q, const void *k, const void *v,
+                             const float *Dk, const float *Uk, const float *Dv, const float *Uv,
+                             const void *out, const void *dout, float scale, void *dq, void *dk, void *dv,
+                             float *dDk, float *dUk, float *dDv, float *dUv, void *workspace,
+                             size_t workspace_bytes, void *stream)
+{
+    dar_status s = check_dims(dtype, d, d_down);
+    if (s != DAR_OK)
+        return s;
+    if (B < 0 || Hkv < 1 || Hq < Hkv || Hq % Hkv || N < 0 || w < 0)
+        return fail(DAR_ERR_INVALID_ARG, "B=%d Hq=%d Hkv=%d N=%d w=%d", B, Hq, Hkv, N, w);
+    if ((long long)B * Hq > 65535 || (long long)B * Hkv > 65535)
+        return fail(DAR_ERR_UNSUPPORTED, "B*Hq=%lld > 65535", (long long)B * Hq);
+    const void *ptrs[] = {q, k, v, Dk, Uk, Dv, Uv, out, dout, dq, dk, dv, dDk, dUk, dDv, dUv, workspace};
+    for (const void *p : ptrs)
+        if (!p)
+            return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    for (const void *p : ptrs)
+        if (!aligned16(p))
+            return fail(DAR_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
+    const size_t need = dar::backward_workspace_bytes(dtype, B, Hq, Hkv, N, d_down);
+    if (workspace_bytes < need)
+        return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, need);
+    dar::BackwardArgs a;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.out = out;
+    a.dout = dout;
+    a.Dk = Dk;
+    a.Uk = Uk;
+    a.Dv = Dv;
+    a.Uv = Uv;
+    a.dq = dq;
+    a.dk = dk;
+    a.dv = dv;
+    a.dDk = dDk;
+    a.dUk = dUk;
+    a.dDv = dDv;
+    a.dUv = dUv;
+    a.B = B;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.N = N;
+    a.w = w;
+    a.dd = d_down;
+    a.scale = default_scale(scale, d);
+    return from_cuda(dar::launch_backward(dtype, a, workspace, static_cast<cudaStream_t>(stream)),
+                     "dar_attn_backward launch");
+}
+
 dar_status dar_attn_prefill_direct(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
                                    int32_t d, int32_t d_down, int32_t w, const void *q, const void *qd,
                                    const void *k, const void *v, const float *Dk, const float *Dv,

@@ -110,6 +110,20 @@ cudaError_t launch_decode(dar_dtype dt, int dd, const DecodeArgs &a, cudaStream_
 cudaError_t launch_prefill_simt(dar_dtype dt, int dd, const PrefillArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_tc(int dd, const PrefillArgs &a, cudaStream_t s);
 
+// Gradients of the causal forward (dar_backward.cu); the workspace holds the
+// Eq. 1 vectors, per-row q~, dO~, D, log-sum-exp, dq~, O^D, per-key dk^D,
+// dv^D and the projection gradients' partial sums.
+struct BackwardArgs {
+    const void *q, *k, *v, *out, *dout;
+    const float *Dk, *Uk, *Dv, *Uv;
+    void *dq, *dk, *dv;
+    float *dDk, *dUk, *dDv, *dUv;
+    int B, Hq, Hkv, N, w, dd;
+    float scale;
+};
+size_t backward_workspace_bytes(dar_dtype dt, int B, int Hq, int Hkv, int N, int dd);
+cudaError_t launch_backward(dar_dtype dt, const BackwardArgs &a, void *workspace, cudaStream_t s);
+
 // Chunked prefill over a cache: gather kernel, attention (chunk mode), then
 // the cache append of the chunk.  Buffers of the workspace (see dar_abi.cu).
 struct ChunkArgs {

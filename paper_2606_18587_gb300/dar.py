@@ -73,6 +73,9 @@ def load_library(path: str = LIB_PATH):
         "dar_attn_prefill_direct": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32, P, P, P, P, P, P, P, F, F,
                                      P, P, SZ, P, P], ctypes.c_int),
         "dar_attn_decode_direct": ([CP, I32, P, P, P, F, F, P, P, SZ, P], ctypes.c_int),
+        "dar_attn_backward_workspace_bytes": ([ctypes.c_int, I32, I32, I32, I32, I32], SZ),
+        "dar_attn_backward": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32] + [P] * 9 + [F] + [P] * 8 + [SZ, P],
+                              ctypes.c_int),
         "dar_last_error": ([], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -350,6 +353,40 @@ def dar_attn_decode_direct(cache: DarCache, q, qd, Wo, workspace, scale=0.0, sca
         cache.struct, q.shape[1], _ptr(q), _ptr(qd), _ptr(Wo), float(scale), float(scale_down), _ptr(out),
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
     return out
+
+
+def dar_attn_backward_workspace_bytes(dtype, B, Hq, Hkv, N, d_down) -> int:
+    return int(load_library().dar_attn_backward_workspace_bytes(_CODE[dtype], B, Hq, Hkv, N, d_down))
+
+
+def dar_attn_backward(q, k, v, Dk, Uk, Dv, Uv, out, dout, w, scale=0.0, workspace=None, grads=None,
+                      stream=None):
+    """Gradients of the causal forward (Sec. 2.3 training) for the output
+    gradient ``dout``; ``out`` is the forward's output.  Returns a dict with
+    ``dq, dk, dv`` (storage type) and ``dDk, dUk, dDv, dUv`` (fp32); ``grads``
+    may hold preallocated tensors under those names."""
+    _dev(q, "q")
+    for name, t in (("k", k), ("v", v), ("out", out), ("dout", dout)):
+        _dev(t, name, q.dtype)
+    for name, t in (("Dk", Dk), ("Uk", Uk), ("Dv", Dv), ("Uv", Uv)):
+        _dev(t, name, torch.float32)
+    B, Hq, N, d = q.shape
+    Hkv = k.shape[1]
+    dd = Dk.shape[2]
+    g = dict(grads or {})
+    for name, like in (("dq", q), ("dk", k), ("dv", v), ("dDk", Dk), ("dUk", Uk), ("dDv", Dv), ("dUv", Uv)):
+        if name not in g:
+            g[name] = torch.empty_like(like)
+        _dev(g[name], name, like.dtype)
+    if workspace is None:
+        workspace = torch.empty(max(1, dar_attn_backward_workspace_bytes(q.dtype, B, Hq, Hkv, N, dd)),
+                                dtype=torch.uint8, device=q.device)
+    _dev(workspace, "workspace")
+    _check(load_library().dar_attn_backward(
+        _code(q), B, Hq, Hkv, N, d, dd, int(w), _ptr(q), _ptr(k), _ptr(v), _ptr(Dk), _ptr(Uk), _ptr(Dv), _ptr(Uv),
+        _ptr(out), _ptr(dout), float(scale), *(_ptr(g[n]) for n in ("dq", "dk", "dv", "dDk", "dUk", "dDv", "dUv")),
+        _ptr(workspace), workspace.numel(), _stream(stream)))
+    return g
 
 
 def dar_prefill_chunk_workspace_bytes(cache: DarCache, n: int) -> int:

@@ -151,6 +151,21 @@ def prefill_flops(cfg: I.Prefill) -> float:
     return float(heads * (local * 4 * cfg.d + glob * 4 * cfg.dd + cfg.N * 4 * cfg.d * cfg.dd))
 
 
+def prefill_backward_flops(cfg: I.Prefill) -> float:
+    """Algorithmic FLOPs of the backward pass: per local pair five d-wide
+    contractions (scores recomputed, dP, dq, dk, dv: 10 d), per global pair the
+    same five in d_down plus the global value sum the Uv gradient needs
+    (12 d_down); per query row q Uk^T, dO Uv^T, the dq lift and the two
+    projection-gradient outer products; per key the dk, dv lifts and two more
+    outer products (each 2 d d_down)."""
+    local, glob = prefill_pairs(cfg.N, cfg.w)
+    heads = cfg.B * cfg.Hq
+    rows = heads * cfg.N
+    keys = cfg.B * cfg.Hkv * cfg.N
+    dd2 = 2 * cfg.d * cfg.dd
+    return float(heads * (local * 10 * cfg.d + glob * 12 * cfg.dd) + rows * 5 * dd2 + keys * 4 * dd2)
+
+
 def prefill_exps(cfg: I.Prefill) -> int:
     local, glob = prefill_pairs(cfg.N, cfg.w)
     return cfg.B * cfg.Hq * (local + glob)

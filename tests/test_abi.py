@@ -145,3 +145,51 @@ def test_bounded_wait_check_rejects_bad_arguments(lib):
     assert L.dar_check_bounded_wait(4096, 0, None) == 1
     assert L.dar_check_bounded_wait(4096, 2000001, None) == 1
     assert "limit_us" in L.dar_last_error().decode()
+
+
+def _declared_param_counts(header):
+    """Parameter count of every function declared in the header (C text)."""
+    import re
+    text = re.sub(r"/\*.*?\*/", "", open(header).read(), flags=re.S)
+    counts = {}
+    for m in re.finditer(r"\b(dar_\w+)\s*\(([^;{]*?)\)\s*;", text, re.S):
+        params = m.group(2).strip()
+        counts[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    return counts
+
+
+def test_binding_argument_counts_match_the_header(lib):
+    """Every ctypes signature in the Python binding has as many arguments as
+    the C declaration it wraps."""
+    L = lib.load_library()
+    counts = _declared_param_counts(lib.HEADER)
+    assert set(counts) == set(lib.declared_symbols())
+    for name, n in counts.items():
+        assert len(getattr(L, name).argtypes) == n, name
+
+
+def test_direct_and_backward_reject_bad_arguments(lib):
+    L = lib.load_library()
+    P = 4096
+    c = _cache(lib)
+    # direct decode: NULL qd, misaligned qd, Hq not a multiple of Hkv
+    assert L.dar_attn_decode_direct(ctypes.byref(c), 4, P, None, P, 0.0, 0.0, P, P, 1 << 30, None) == 1
+    assert L.dar_attn_decode_direct(ctypes.byref(c), 4, P, P + 4, P, 0.0, 0.0, P, P, 1 << 30, None) == 1
+    assert L.dar_attn_decode_direct(ctypes.byref(c), 3, P, P, P, 0.0, 0.0, P, P, 1 << 30, None) == 1
+    # direct prefill: NULL qd, unsupported d_down
+    pre = lambda qd=P, dd=16: L.dar_attn_prefill_direct(lib.DAR_BF16, 1, 4, 2, 16, 64, dd, 4, P, qd, P, P, P, P, P,  # noqa
+                                                         0.0, 0.0, P, P, 1 << 20, None, None)
+    assert pre(qd=None) == 1
+    assert pre(dd=12) == 2
+
+    # backward: workspace too small, NULL gradient, misaligned input
+    def bwd(dq=P, k=P, wsb=1 << 40, Hq=4):
+        return L.dar_attn_backward(lib.DAR_BF16, 1, Hq, 2, 16, 64, 16, 4, P, k, P, P, P, P, P, P, P, 0.0,
+                                   dq, P, P, P, P, P, P, P, wsb, None)
+    assert bwd(wsb=16) == 3
+    assert bwd(dq=None) == 1
+    assert bwd(k=P + 2) == 1
+    assert bwd(Hq=3) == 1
+    n = L.dar_attn_backward_workspace_bytes(lib.DAR_BF16, 1, 4, 2, 16, 16)
+    assert n > 0 and n % 256 == 0
+    assert L.dar_attn_backward_workspace_bytes(lib.DAR_BF16, 1, 3, 2, 16, 16) == 0
