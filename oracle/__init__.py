@@ -18,6 +18,10 @@ arrays.  Function-level citations:
 * :func:`backward` -- Sec. 2.3 (training): the gradients of the causal
   forward with respect to q, k, v and the four projections, by the chain rule
   through Eq. 4, 3, 2 and 1 in turn.
+* :func:`latent_rows`, :func:`latent_prefill`, :func:`latent_decode` -- Eq. 1-4
+  in the paper's own form on hidden states with one bottleneck per token
+  shared by every head, keys and values (``c = h W_down``, ``h' = c W_up``,
+  distant keys/values ``h' W_K``, ``h' W_V``), the cache scheme of Sec. 5.
 * :func:`attention_rows_direct`, :func:`prefill_direct`, :func:`decode_direct`
   -- Sec. 5, "Direct lower-dimensional global attention": the global path in
   d_down with a query of its own and an output map of the global values.
@@ -74,6 +78,10 @@ def _load():
             [ctypes.c_int] * 8 + [P] * 8 + [ctypes.c_double] + [P] * 7 + [ctypes.c_int]
         )
         lib.dar_oracle_backward.restype = ctypes.c_int
+        lib.dar_oracle_attention_latent.argtypes = (
+            [ctypes.c_int] * 9 + [P] * 7 + [ctypes.c_double, ctypes.c_long, P, P, P, P, ctypes.c_int]
+        )
+        lib.dar_oracle_attention_latent.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -303,3 +311,75 @@ def backward(q, k, v, Dk, Uk, Dv, Uv, dout, w, dtype, scale=None, nthreads=None)
     if rc != 0:
         raise ValueError("oracle rejected its arguments")
     return g
+
+
+def latent_rows(q_rows, Hq, k, v, c, Wup, WK, WV, w, dtype, rows, scale=None, nthreads=None):
+    """Eq. 2-4 in the latent form for explicit rows ``(b, h, i)``.
+
+    ``k, v [B,Hkv,N,d]`` the full keys/values (window branch of Eq. 3), ``c
+    [B,N,dl]`` the stored bottleneck of every token (Eq. 1), ``Wup [dl,D]``,
+    ``WK, WV [Hkv,D,d]``: distant keys/values are ``(c_j Wup) WK``, ``(c_j Wup)
+    WV``, formed explicitly.  Returns float64 ``[R,d]``."""
+    q_rows, k, v, c = (_check(a, dtype) for a in (q_rows, k, v, c))
+    Wup, WK, WV = (np.ascontiguousarray(a, dtype=np.float32) for a in (Wup, WK, WV))
+    B, Hkv, N, d = k.shape
+    dl, D = Wup.shape
+    assert c.shape == (B, N, dl) and WK.shape == (Hkv, D, d) and WV.shape == (Hkv, D, d)
+    rows = np.ascontiguousarray(rows, dtype=np.int32).reshape(-1, 3)
+    rb, rh, ri = (np.ascontiguousarray(rows[:, j]) for j in range(3))
+    out = np.zeros((rows.shape[0], d), dtype=np.float64)
+    scale = 1.0 / np.sqrt(d) if scale is None else scale
+    nthreads = (os.cpu_count() or 1) if nthreads is None else nthreads
+    rc = _load().dar_oracle_attention_latent(
+        _DTYPES[dtype], B, int(Hq), Hkv, N, d, D, dl, int(w), _ptr(q_rows), _ptr(k), _ptr(v), _ptr(c), _ptr(Wup),
+        _ptr(WK), _ptr(WV), float(scale), rows.shape[0], _ptr(rb), _ptr(rh), _ptr(ri), _ptr(out), int(nthreads))
+    if rc != 0:
+        raise ValueError("oracle rejected its arguments")
+    return out
+
+
+def latent_bottleneck(h, Wdown, dtype):
+    """Eq. 1 on hidden states: ``h [B,n,D]`` times ``Wdown [D,dl]`` -> ``c [B,n,dl]``,
+    each element one fp32 FMA chain over the D inputs, rounded to the storage
+    type (the same chain as :func:`down_project`, with one shared bottleneck)."""
+    return down_project(np.ascontiguousarray(h[:, None]), np.ascontiguousarray(Wdown[None]), dtype)[:, 0]
+
+
+def latent_prefill(q, k, v, h, Wdown, Wup, WK, WV, w, dtype, scale=None, nthreads=None, rows=None):
+    """Causal forward of the latent form over positions 0..N-1; ``h [B,N,D]``
+    the hidden states the bottleneck is taken from (Eq. 1)."""
+    B, Hq, N, d = q.shape
+    c = latent_bottleneck(h, Wdown, dtype)
+    full = rows is None
+    if full:
+        bb, hh, ii = np.meshgrid(np.arange(B), np.arange(Hq), np.arange(N), indexing="ij")
+        rows = np.stack([bb.ravel(), hh.ravel(), ii.ravel()], axis=1)
+    rows = np.asarray(rows, dtype=np.int64).reshape(-1, 3)
+    q_rows = np.ascontiguousarray(q[rows[:, 0], rows[:, 1], rows[:, 2]])
+    out = latent_rows(q_rows, Hq, k, v, c, Wup, WK, WV, w, dtype, rows, scale, nthreads)
+    return out.reshape(B, Hq, N, d) if full else out
+
+
+def latent_decode(q_last, k_hist, v_hist, h_hist, lens, Wdown, Wup, WK, WV, w, dtype, scale=None, nthreads=None,
+                  heads=None):
+    """One inference step of the latent form (query at ``lens[b]-1``):
+    ``q_last [B,Hq,d]``, histories ``k_hist, v_hist [B,Hkv,Nmax,d]`` and
+    ``h_hist [B,Nmax,D]`` (first ``lens[b]`` tokens read)."""
+    B, Hq, d = q_last.shape
+    lens = np.asarray(lens, dtype=np.int64)
+    out = np.zeros((B, Hq, d), dtype=np.float64)
+    if heads is None:
+        heads = [(b, h) for b in range(B) for h in range(Hq)]
+    by_seq = {}
+    for b, h in heads:
+        if lens[b] > 0:
+            by_seq.setdefault(int(b), []).append(int(h))
+    for b, hs in sorted(by_seq.items()):
+        L = int(lens[b])
+        c = latent_bottleneck(np.ascontiguousarray(h_hist[b:b + 1, :L]), Wdown, dtype)
+        rows = np.array([(0, h, L - 1) for h in hs], dtype=np.int32)
+        res = latent_rows(np.ascontiguousarray(q_last[b, hs]), Hq, np.ascontiguousarray(k_hist[b:b + 1, :, :L]),
+                          np.ascontiguousarray(v_hist[b:b + 1, :, :L]), c, Wup, WK, WV, w, dtype, rows, scale,
+                          nthreads)
+        out[b, hs] = res
+    return out

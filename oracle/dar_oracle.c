@@ -612,3 +612,142 @@ int dar_oracle_backward(int dtype, int B, int Hq, int Hkv, int N, int d, int dd,
     free(th);
     return 0;
 }
+
+/* ---- Sec. 2 in its latent form, with the cache scheme of Sec. 5 -----------
+ * The paper's own form of Eq. 1-3 on hidden states (model width D), with one
+ * bottleneck per token shared by every head and by keys and values:
+ *   Eq. 1  c_j  = h_j W_down                  (d_lat; given here as stored, c)
+ *   Eq. 2  h'_j = c_j W_up                    (back to D, explicitly, fp64)
+ *   Eq. 3  k_j = h_j W_K^g,  v_j = h_j W_V^g  inside the window (given: k, v)
+ *          k_j = h'_j W_K^g, v_j = h'_j W_V^g beyond it (computed here, fp64)
+ *   Eq. 4  one softmax over all j <= i.
+ * Positions are already encoded (no RoPE), as in the per-head form.
+ *   q    [nrows][d] T        the query of each row
+ *   k, v [B][Hkv][N][d] T    full keys / values of every token
+ *   c    [B][N][dl] T        the stored bottleneck of every token
+ *   Wup  [dl][D] fp32;  WK, WV [Hkv][D][d] fp32 */
+typedef struct {
+    int dtype, B, Hq, Hkv, N, d, D, dl, w;
+    const void *q, *k, *v, *c;
+    const float *Wup, *WK, *WV;
+    double scale;
+    long nrows;
+    const int *row_b, *row_h, *row_i;
+    double *out;
+    int nthreads, tid;
+} latent_job;
+
+static void latent_unit(const latent_job *J, int b, int g)
+{
+    const int d = J->d, D = J->D, dl = J->dl, N = J->N, G = J->Hq / J->Hkv;
+    int jmax = -1;
+    for (long r = 0; r < J->nrows; ++r)
+        if (J->row_b[r] == b && J->row_h[r] / G == g && J->row_i[r] > jmax)
+            jmax = J->row_i[r];
+    if (jmax < 0)
+        return;
+    const int n = jmax + 1;
+    const size_t base = ((size_t)b * J->Hkv + g) * N;
+    double *Kf = malloc(sizeof(double) * (size_t)n * d), *Vf = malloc(sizeof(double) * (size_t)n * d);
+    double *Kl = malloc(sizeof(double) * (size_t)n * d), *Vl = malloc(sizeof(double) * (size_t)n * d);
+    double *hl = malloc(sizeof(double) * (size_t)D), *s = malloc(sizeof(double) * (size_t)n);
+    for (int j = 0; j < n; ++j) {
+        for (int t = 0; t < d; ++t) {
+            Kf[(size_t)j * d + t] = load_as_f32(J->k, J->dtype, (base + j) * d + t);
+            Vf[(size_t)j * d + t] = load_as_f32(J->v, J->dtype, (base + j) * d + t);
+        }
+        /* Eq. 2: h'_j = c_j W_up */
+        for (int e = 0; e < D; ++e) {
+            double acc = 0.0;
+            for (int a = 0; a < dl; ++a)
+                acc += (double)load_as_f32(J->c, J->dtype, ((size_t)b * N + j) * dl + a) *
+                       (double)J->Wup[(size_t)a * D + e];
+            hl[e] = acc;
+        }
+        /* Eq. 3, distant branch: k'_j = h'_j W_K^g, v'_j = h'_j W_V^g */
+        for (int t = 0; t < d; ++t) {
+            double ka = 0.0, va = 0.0;
+            for (int e = 0; e < D; ++e) {
+                ka += hl[e] * (double)J->WK[((size_t)g * D + e) * d + t];
+                va += hl[e] * (double)J->WV[((size_t)g * D + e) * d + t];
+            }
+            Kl[(size_t)j * d + t] = ka;
+            Vl[(size_t)j * d + t] = va;
+        }
+    }
+    for (long r = 0; r < J->nrows; ++r) {
+        if (J->row_b[r] != b || J->row_h[r] / G != g)
+            continue;
+        const int i = J->row_i[r];
+        double *o = J->out + (size_t)r * d;
+        double smax = -INFINITY;
+        for (int j = 0; j <= i; ++j) {
+            const double *key = (i - j < J->w) ? &Kf[(size_t)j * d] : &Kl[(size_t)j * d];
+            double dot = 0.0;
+            for (int t = 0; t < d; ++t)
+                dot += (double)load_as_f32(J->q, J->dtype, (size_t)r * d + t) * key[t];
+            s[j] = J->scale * dot;
+            if (s[j] > smax)
+                smax = s[j];
+        }
+        double denom = 0.0;
+        for (int j = 0; j <= i; ++j)
+            denom += exp(s[j] - smax);
+        for (int t = 0; t < d; ++t)
+            o[t] = 0.0;
+        for (int j = 0; j <= i; ++j) {
+            const double p = exp(s[j] - smax) / denom;
+            const double *val = (i - j < J->w) ? &Vf[(size_t)j * d] : &Vl[(size_t)j * d];
+            for (int t = 0; t < d; ++t)
+                o[t] += p * val[t];
+        }
+    }
+    free(Kf);
+    free(Vf);
+    free(Kl);
+    free(Vl);
+    free(hl);
+    free(s);
+}
+
+static void *latent_worker(void *arg)
+{
+    const latent_job *J = (const latent_job *)arg;
+    const int units = J->B * J->Hkv;
+    for (int u = J->tid; u < units; u += J->nthreads)
+        latent_unit(J, u / J->Hkv, u % J->Hkv);
+    return NULL;
+}
+
+/* Rows of the latent form (the row list as in dar_oracle_attention). */
+int dar_oracle_attention_latent(int dtype, int B, int Hq, int Hkv, int N, int d, int D, int dl, int w,
+                                const void *q, const void *k, const void *v, const void *c,
+                                const float *Wup, const float *WK, const float *WV, double scale,
+                                long nrows, const int *row_b, const int *row_h, const int *row_i,
+                                double *out, int nthreads)
+{
+    if (B < 1 || Hkv < 1 || Hq < Hkv || Hq % Hkv || N < 1 || d < 1 || D < 1 || dl < 1 || w < 0 ||
+        nrows < 0 || (dtype != ORC_F32 && dtype != ORC_BF16))
+        return -1;
+    for (long r = 0; r < nrows; ++r)
+        if (row_b[r] < 0 || row_b[r] >= B || row_h[r] < 0 || row_h[r] >= Hq ||
+            row_i[r] < 0 || row_i[r] >= N)
+            return -1;
+    if (nthreads < 1)
+        nthreads = 1;
+    latent_job *jobs = malloc(sizeof(latent_job) * (size_t)nthreads);
+    pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
+    for (int t = 0; t < nthreads; ++t) {
+        latent_job J = {dtype, B, Hq, Hkv, N, d, D, dl, w, q, k, v, c, Wup, WK, WV, scale,
+                        nrows, row_b, row_h, row_i, out, nthreads, t};
+        jobs[t] = J;
+    }
+    for (int t = 1; t < nthreads; ++t)
+        pthread_create(&th[t], NULL, latent_worker, &jobs[t]);
+    latent_worker(&jobs[0]);
+    for (int t = 1; t < nthreads; ++t)
+        pthread_join(th[t], NULL);
+    free(jobs);
+    free(th);
+    return 0;
+}

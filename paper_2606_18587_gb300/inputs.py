@@ -31,6 +31,7 @@ _gen = None
 
 # tensor stream ids
 S_Q, S_K, S_V, S_DK, S_DV, S_UK, S_UV, S_LENS, S_PAGES, S_QDEC, S_KNEW, S_VNEW, S_QD = range(1, 14)
+S_H, S_WDOWN, S_WUP, S_WK, S_WV, S_HNEW = range(14, 20)
 _KIND = {"f32": 0, "bf16": 1, "f64": 2, "uniform": 3}
 _NP = {"f32": np.float32, "bf16": np.uint16, "f64": np.float64, "uniform": np.float64}
 
@@ -98,6 +99,17 @@ def projections(seed: int, Hkv: int, d: int, dd: int):
     Uk = normal_array(seed, S_UK, (Hkv, dd, d), std=1.0 / np.sqrt(dd))
     Uv = normal_array(seed, S_UV, (Hkv, dd, d), std=1.0 / np.sqrt(dd))
     return Dk, Uk, Dv, Uv
+
+
+def latent_projections(seed: int, Hkv: int, D: int, dl: int, d: int):
+    """The latent form's matrices, float32: Wdown [D,dl] ~ N(0, 1/D), Wup [dl,D]
+    ~ N(0, 1/dl), WK, WV [Hkv,D,d] ~ N(0, 1/D) (unit-variance bottlenecks,
+    lifted states and distant keys/values for unit-variance hidden states)."""
+    Wdown = normal_array(seed, S_WDOWN, (D, dl), std=1.0 / np.sqrt(D))
+    Wup = normal_array(seed, S_WUP, (dl, D), std=1.0 / np.sqrt(dl))
+    WK = normal_array(seed, S_WK, (Hkv, D, d), std=1.0 / np.sqrt(D))
+    WV = normal_array(seed, S_WV, (Hkv, D, d), std=1.0 / np.sqrt(D))
+    return Wdown, Wup, WK, WV
 
 
 # --------------------------------------------------------------------------- workloads
