@@ -353,6 +353,50 @@ def prefill_section(args, torch, dar, W, I, dev, stream, tc_peak, peak_src, loca
             "clocks": clk.summary()}
 
 
+def latent_point(torch, dar, I, W, cfg, K, l2, dev, stream, hbm_peak):
+    """GB/s of graph-timed dar_latent_decode calls on a latent-form workload
+    (one bottleneck per token shared by every head); cache copies rotate so
+    the bytes between two uses of one copy exceed 4x L2.  The first call's
+    output is checked against the oracle on two sequences."""
+    import oracle
+    wl = W.LatentDecodeWorkload(cfg, keep_history=True)
+    nbytes = W.latent_decode_bytes(cfg, wl.lens)
+    R = 1 if nbytes > 4 * l2 else int(math.ceil(4 * l2 / nbytes)) + 1
+    caches = [wl.cache]
+    for _ in range(R - 1):
+        c = dar.DarLatentCache(cfg.B, cfg.Hkv, cfg.D, cfg.dl, cfg.w, wl.cache.max_pages_per_seq,
+                               wl.cache.num_pages, block_table=wl.cache.block_table, device=dev)
+        for name in ("win_k", "win_v", "pool_c", "seq_lens"):
+            getattr(c, name).copy_(getattr(wl.cache, name))
+        caches.append(c)
+    outs = [torch.empty_like(wl.q) for _ in range(R)]
+    ws = [wl.workspace] + [dar.latent_decode_workspace(c, cfg.Hq) for c in caches[1:]]
+    g = graph_of(torch, lambda j: dar.dar_latent_decode(caches[j % R], wl.q, wl.A_K, wl.A_V, ws[j % R],
+                                                        out=outs[j % R]), K)
+    ms = time_graph(torch, g, stream, before=lambda: flush_l2(torch, dev, 2 * l2))
+    us = 1e3 * ms / K
+    gbs = nbytes / (us * 1e-6) / 1e9
+    status = sum(c.device_status() for c in caches)
+    seqs = [0, cfg.B - 1]
+    k, v, h = wl.history_arrays(seqs)
+    Wdown, Wup, WK, WV = wl.proj_host
+    heads = [(i, hq) for i in range(2) for hq in range(cfg.Hq)]
+    want = oracle.latent_decode(np.ascontiguousarray(wl.q_host[seqs]), k, v, h, wl.lens[seqs], Wdown, Wup, WK, WV,
+                                cfg.w, "bf16", heads=heads)
+    got = W.to_f64(W.download(outs[0]), "bf16")[seqs]
+    err = float(np.abs(got - want).max())
+    res = {"workload": cfg.name, "bytes_per_call": int(nbytes), "us_per_call": round(us, 3), "gbs": round(gbs, 1),
+           "frac_measured": round(gbs / hbm_peak, 4), "frac_nominal": round(gbs / NOMINAL_HBM_GBS, 4),
+           "copies": R, "oracle_max_abs_err": round(err, 5)}
+    del g, caches, outs, ws, wl
+    torch.cuda.empty_cache()
+    if status:
+        raise RuntimeError(f"device status {status} on {cfg.name}")
+    if not err <= TOL_BF16:
+        raise RuntimeError(f"latent decode output differs from the oracle: max-abs {err}")
+    return res
+
+
 def direct_prefill_point(args, torch, dar, W, I, dev, stream):
     """The 410M-like prefill with the direct global path of Sec. 5
     (dar_attn_prefill_direct): median CUDA-event time of K calls, sampled rows
@@ -471,6 +515,12 @@ def run_ours(args, world, rank, local):
     hbm_peak, tc_peak, tc_sus, peak_src = load_peaks()
     stream = torch.cuda.current_stream()
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    if args.only == "latent":  # profiling aid: the latent-form decode alone
+        res = [latent_point(torch, dar, I, W, c, args.steps, l2, dev, stream, hbm_peak)
+               for c in (I.DECODE_160M_LATENT, I.DECODE_1B_LATENT)]
+        if rank == 0:
+            print(json.dumps({"metric": "latent decode (profiling run)", "latent_form": res}), flush=True)
+        return
     if args.only == "prefill":  # profiling aid: the prefill alone
         pre = prefill_section(args, torch, dar, W, I, dev, stream, tc_peak, peak_src, local)
         if rank == 0:
@@ -656,6 +706,8 @@ def run_ours(args, world, rank, local):
                           "dar_attn_prefill_direct"}
         extra = {"decode_1b_gqa": gqa, "sweep": sweep, "direct_variant": direct,
                  "backward": backward_point(args, torch, dar, W, I, dev, stream),
+                 "latent_form": [latent_point(torch, dar, I, W, c, K, l2, dev, stream, hbm_peak)
+                                 for c in (I.DECODE_160M_LATENT, I.DECODE_1B_LATENT)],
                  "note": "graph of K dar_attn_decode calls, rotating cache copies > 4x L2, L2 flushed before"}
 
     cpu = None
@@ -755,7 +807,7 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle time for the CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true", help="skip the GQA and sweep decode workloads")
-    ap.add_argument("--only", choices=["all", "decode", "prefill"], default="all",
+    ap.add_argument("--only", choices=["all", "decode", "prefill", "latent"], default="all",
                     help="profiling aid: run only the decode step or only the prefill")
     ap.add_argument("--prefill-batch", type=int, default=8, help="batch of the prefill workload")
     ap.add_argument("--soak-seconds", type=float, default=1.0,

@@ -312,6 +312,70 @@ dar_status dar_attn_backward(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv
                              float *dDk, float *dUk, float *dDv, float *dUv, void *workspace,
                              size_t workspace_bytes, void *stream);
 
+/*
+ * The latent form (the paper's own Eq. 1-3 on hidden states, with the cache
+ * scheme of Sec. 5 "Compute and memory efficiency"): every token keeps ONE
+ * bottleneck c_j = h_j W_down (Eq. 1, h_j the layer's hidden state of width D),
+ * shared by every head and by keys and values; the last w tokens also keep
+ * their full per-KV-head keys and values.  A distant token reaches head g as
+ * k'_j = (c_j W_up) W_K^g, v'_j = (c_j W_up) W_V^g (Eq. 2-3); with W_up
+ * absorbed (A_K^g = W_up W_K^g, A_V^g = W_up W_V^g) the decode scores
+ * q . k'_j = (q A_K^gT) . c_j and lifts the weighted sum of the c_j once with
+ * A_V^g.  Cache memory is O(T d_lat + w d) for all heads together.
+ * Positions are already encoded (no RoPE in the library).  bf16 only;
+ * d = 64; d_lat in {64, 128, 192, 256}; Hq <= 32; D <= 8192.
+ *
+ *  win_k, win_v  [B][Hkv][w][d] bf16, ring slot p % w (as dar_cache)
+ *  pool_c        [num_pages][DAR_PAGE_SIZE][d_lat] bf16: c of the token at
+ *                position p in page block_table[b][p / 64], row p % 64 --
+ *                for EVERY position (window tokens too), so nothing migrates
+ *  block_table   [B][max_pages_per_seq] int32; seq_lens [B]; status as dar_cache.
+ * Capacity: max_pages_per_seq * 64 tokens per sequence.
+ */
+typedef struct dar_latent_cache {
+    int32_t B, Hkv, d, D, d_lat, w;
+    int32_t max_pages_per_seq;
+    int32_t num_pages;
+    void *win_k, *win_v;
+    void *pool_c;
+    int32_t *block_table;
+    int32_t *seq_lens;
+    int32_t *status;
+} dar_latent_cache;
+
+/* Append n tokens per sequence (n_b = n_per_seq[b] when given, a device
+ * int32[B] with 0 <= n_b <= n): h_new [B][n][D] bf16 their hidden states,
+ * k_new, v_new [B][Hkv][n][d] bf16 their keys and values, W_down [D][d_lat]
+ * fp32.  Writes c = round_bf16(fp32 FMA chain over e = 0..D-1 of
+ * h[e] W_down[e][c], from +0) into each new token's page row (Eq. 1, the same
+ * chain order as dar_down_project), ring rows for the tokens that remain in
+ * the window, then seq_lens[b] += n_b.  A length beyond capacity or a needed
+ * block-table entry outside [0, num_pages) sets *status = DAR_ERR_CAPACITY. */
+dar_status dar_latent_append(const dar_latent_cache *cache, const void *h_new, const void *k_new,
+                             const void *v_new, int32_t n, const int32_t *n_per_seq,
+                             const float *W_down, void *stream);
+
+/* The absorbed maps of Sec. 5: A_K[g] = W_up W_K[g], A_V[g] = W_up W_V[g]
+ * (fp32 FMA chains over D).  W_up [d_lat][D], W_K, W_V [Hkv][D][d] fp32.
+ * Written: A_K [Hkv][d][d_lat] (stored transposed: element (c, t) of
+ * W_up W_K[g] at A_K[g][t][c]) and A_V [Hkv][d_lat][d], both fp32. */
+dar_status dar_latent_absorb(int32_t Hkv, int32_t D, int32_t d, int32_t d_lat, const float *W_up,
+                             const float *W_K, const float *W_V, float *A_K, float *A_V, void *stream);
+
+/* One decode step of the latent form for the query at position L_b - 1:
+ * q [B][Hq][d] bf16, A_K [Hkv][d][d_lat], A_V [Hkv][d_lat][d] fp32 (as
+ * dar_latent_absorb writes them),
+ * out [B][Hq][d] bf16.  Local keys (the last min(L_b, w) tokens) at full d,
+ * distant ones through c, one softmax over both (Eq. 3-4).  Three kernels in
+ * order on `stream` (q~ = q A_K^T; split-K over pages of the latent pool and
+ * the window; merge and lift).  Workspace of
+ * dar_latent_decode_workspace_bytes(cache, Hq) bytes, no initialisation.
+ * L_b == 0 gives a zero output. */
+size_t dar_latent_decode_workspace_bytes(const dar_latent_cache *cache, int32_t Hq);
+dar_status dar_latent_decode(const dar_latent_cache *cache, int32_t Hq, const void *q, const float *A_K,
+                             const float *A_V, float scale, void *out, void *workspace,
+                             size_t workspace_bytes, void *stream);
+
 /* Message for the last non-OK return on this thread ("" if none). */
 const char *dar_last_error(void);
 

@@ -509,6 +509,142 @@ dar_status dar_attn_prefill(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv,
                           workspace, workspace_bytes, status, stream);
 }
 
+}  // extern "C"
+
+namespace {
+
+dar_status check_latent(const dar_latent_cache *c)
+{
+    if (!c)
+        return fail(DAR_ERR_INVALID_ARG, "cache is NULL");
+    if (c->d != dar::kHeadDim)
+        return fail(DAR_ERR_UNSUPPORTED, "head dimension d=%d (only d=64 is built)", c->d);
+    if (c->d_lat != 64 && c->d_lat != 128 && c->d_lat != 192 && c->d_lat != 256)
+        return fail(DAR_ERR_UNSUPPORTED, "d_lat=%d (built: 64, 128, 192, 256)", c->d_lat);
+    if (c->B < 0 || c->Hkv < 1 || c->w < 1 || c->D < 1 || c->max_pages_per_seq < 1 || c->num_pages < 1)
+        return fail(DAR_ERR_INVALID_ARG, "latent cache shape B=%d Hkv=%d w=%d D=%d max_pages_per_seq=%d "
+                    "num_pages=%d", c->B, c->Hkv, c->w, c->D, c->max_pages_per_seq, c->num_pages);
+    if (c->D > 8192)
+        return fail(DAR_ERR_UNSUPPORTED, "hidden width D=%d > 8192", c->D);
+    if (c->B > 65535)
+        return fail(DAR_ERR_UNSUPPORTED, "batch %d > 65535", c->B);
+    if (c->B == 0)
+        return DAR_OK;
+    if (!c->win_k || !c->win_v || !c->pool_c || !c->block_table || !c->seq_lens || !c->status)
+        return fail(DAR_ERR_INVALID_ARG, "latent cache pointer is NULL");
+    if (!aligned16(c->win_k) || !aligned16(c->win_v) || !aligned16(c->pool_c))
+        return fail(DAR_ERR_INVALID_ARG, "latent cache buffers must be 16-byte aligned");
+    if ((double)c->num_pages * DAR_PAGE_SIZE >= 2147483647.0 || (double)c->max_pages_per_seq * 64 >= 2147483647.0)
+        return fail(DAR_ERR_UNSUPPORTED, "latent pool rows beyond int32");
+    return DAR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+dar_status dar_latent_append(const dar_latent_cache *cache, const void *h_new, const void *k_new,
+                             const void *v_new, int32_t n, const int32_t *n_per_seq,
+                             const float *W_down, void *stream)
+{
+    dar_status s = check_latent(cache);
+    if (s != DAR_OK)
+        return s;
+    if (n < 0)
+        return fail(DAR_ERR_INVALID_ARG, "n=%d", n);
+    if (cache->B == 0 || n == 0)
+        return ok();
+    if (!h_new || !k_new || !v_new || !W_down)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(h_new) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(W_down))
+        return fail(DAR_ERR_INVALID_ARG, "h_new, k_new, v_new and W_down must be 16-byte aligned");
+    dar::LatentAppendArgs a;
+    a.h = h_new;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.Wdown = W_down;
+    a.win_k = cache->win_k;
+    a.win_v = cache->win_v;
+    a.pool_c = cache->pool_c;
+    a.block_table = cache->block_table;
+    a.n_per_seq = n_per_seq;
+    a.seq_lens = cache->seq_lens;
+    a.status = cache->status;
+    a.B = cache->B;
+    a.Hkv = cache->Hkv;
+    a.n = n;
+    a.D = cache->D;
+    a.DL = cache->d_lat;
+    a.w = cache->w;
+    a.maxp = cache->max_pages_per_seq;
+    a.num_pages = cache->num_pages;
+    return from_cuda(dar::launch_latent_append(a, static_cast<cudaStream_t>(stream)), "dar_latent_append launch");
+}
+
+dar_status dar_latent_absorb(int32_t Hkv, int32_t D, int32_t d, int32_t d_lat, const float *W_up,
+                             const float *W_K, const float *W_V, float *A_K, float *A_V, void *stream)
+{
+    if (d != dar::kHeadDim)
+        return fail(DAR_ERR_UNSUPPORTED, "head dimension d=%d (only d=64 is built)", d);
+    if (Hkv < 1 || D < 1 || d_lat < 1 || Hkv > 65535 || d_lat > 65535)
+        return fail(DAR_ERR_INVALID_ARG, "Hkv=%d D=%d d_lat=%d", Hkv, D, d_lat);
+    if (!W_up || !W_K || !W_V || !A_K || !A_V)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    return from_cuda(dar::launch_latent_absorb(W_up, W_K, W_V, A_K, A_V, Hkv, D, d_lat,
+                                               static_cast<cudaStream_t>(stream)),
+                     "dar_latent_absorb launch");
+}
+
+size_t dar_latent_decode_workspace_bytes(const dar_latent_cache *cache, int32_t Hq)
+{
+    if (check_latent(cache) != DAR_OK || Hq < cache->Hkv || Hq % cache->Hkv || Hq > 32)
+        return 0;
+    return dar::latent_decode_workspace_bytes(cache->B, Hq, cache->d_lat, cache->max_pages_per_seq);
+}
+
+dar_status dar_latent_decode(const dar_latent_cache *cache, int32_t Hq, const void *q, const float *A_K,
+                             const float *A_V, float scale, void *out, void *workspace,
+                             size_t workspace_bytes, void *stream)
+{
+    dar_status s = check_latent(cache);
+    if (s != DAR_OK)
+        return s;
+    if (Hq < cache->Hkv || Hq % cache->Hkv)
+        return fail(DAR_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", Hq, cache->Hkv);
+    if (Hq > 32)
+        return fail(DAR_ERR_UNSUPPORTED, "Hq=%d > 32", Hq);
+    if (cache->B == 0)
+        return ok();
+    if (!q || !A_K || !A_V || !out || !workspace)
+        return fail(DAR_ERR_INVALID_ARG, "NULL pointer");
+    if (!aligned16(q) || !aligned16(out) || !aligned16(A_K) || !aligned16(A_V) || !aligned16(workspace))
+        return fail(DAR_ERR_INVALID_ARG, "q, out, A_K, A_V and workspace must be 16-byte aligned");
+    const size_t need = dar::latent_decode_workspace_bytes(cache->B, Hq, cache->d_lat, cache->max_pages_per_seq);
+    if (workspace_bytes < need)
+        return fail(DAR_ERR_CAPACITY, "workspace %zu bytes < %zu needed", workspace_bytes, need);
+    dar::LatentDecodeArgs a;
+    a.q = q;
+    a.out = out;
+    a.win_k = cache->win_k;
+    a.win_v = cache->win_v;
+    a.pool_c = cache->pool_c;
+    a.block_table = cache->block_table;
+    a.seq_lens = cache->seq_lens;
+    a.status = cache->status;
+    a.Ak = A_K;
+    a.Av = A_V;
+    a.B = cache->B;
+    a.Hq = Hq;
+    a.Hkv = cache->Hkv;
+    a.DL = cache->d_lat;
+    a.w = cache->w;
+    a.maxp = cache->max_pages_per_seq;
+    a.num_pages = cache->num_pages;
+    a.scale = default_scale(scale, cache->d);
+    return from_cuda(dar::launch_latent_decode(a, workspace, static_cast<cudaStream_t>(stream)),
+                     "dar_latent_decode launch");
+}
+
 size_t dar_attn_backward_workspace_bytes(dar_dtype dtype, int32_t B, int32_t Hq, int32_t Hkv, int32_t N,
                                          int32_t d_down)
 {

@@ -1,0 +1,812 @@
+// dar_latent.cu -- DAR attention in the paper's own latent form (Sec. 2,
+// Eq. 1-4 on hidden states, with the cache scheme of Sec. 5 "Compute and
+// memory efficiency"): every token keeps ONE bottleneck c_j = h_j W_down,
+// shared by all heads and by keys and values; a head g reaches a distant token
+// through k'_j = (c_j W_up) W_K^g and v'_j = (c_j W_up) W_V^g.  With W_up
+// absorbed (A_K^g = W_up W_K^g, A_V^g = W_up W_V^g, d_lat x d each):
+//   global score   scale * q_i . k'_j = scale * (q_i A_K^gT) . c_j = scale * q~_i . c_j
+//   global value   sum_j p_ij v'_j  = (sum_j p_ij c_j) A_V^g
+// so a decode step streams each distant token's d_lat-vector once for all Hq
+// heads (an MLA-like contraction: heads x d_lat against tokens x d_lat),
+// while the last w tokens keep full keys and values per KV head.
+//
+// Kernels:
+//  - latent_append: Eq. 1 (c = h W_down, one fp32 FMA chain over the D
+//    inputs per element, rounded once to bf16) into the page of every new
+//    token; new keys/values into the ring; then the lengths.
+//  - latent_absorb: A_K, A_V (fp32 chains over D).
+//  - decode: prep (q~ = q A_K^T, bf16), main (latent splits of four pages
+//    each: TMA-staged pages, S = Q~ C^T and O += P C on mma.sync tensor
+//    cores, one online softmax per head; plus one CTA per KV head for the
+//    window on the CUDA cores), merge (exact log-sum-exp combination of the
+//    partial results, then o = (O_loc + O_lat A_V) / l).
+#include <cuda.h>
+
+#include <mutex>
+
+#include "dar_common.cuh"
+#include "dar_launch.h"
+#include "dar_sm100.cuh"
+
+namespace dar {
+namespace lat {
+
+using namespace sm100;
+
+constexpr int kTok = DAR_PAGE_SIZE;  // tokens per page
+constexpr int kPagesPerSplit = 4;
+constexpr int kSplitTok = kTok * kPagesPerSplit;
+constexpr int kMainThreads = 128;
+constexpr int kWinChunk = 64;  // window tokens staged at a time
+constexpr int kWinLd = 65;
+
+struct Args {
+    const void *q;  // [B][Hq][64]
+    void *out;      // [B][Hq][64]
+    const void *win_k, *win_v;
+    const int32_t *block_table, *seq_lens;
+    int32_t *status;
+    const float *Ak, *Av;  // [Hkv][64][DL] (transposed), [Hkv][DL][64]
+    bf16 *qt;              // [B][Hq][DL]
+    float *rec_lat;        // [B][nspl][Hq][DL + 2]
+    float *rec_win;        // [B][Hq][66]
+    int B, Hq, Hkv, G, w, maxp, num_pages, nspl;
+    float c2;  // scale * log2(e)
+};
+
+// ---------------------------------------------------------------- append
+
+struct AppendArgs {
+    const void *h;  // [B][n][D]
+    const void *k_new, *v_new;  // [B][Hkv][n][64]
+    const float *Wdown;         // [D][DL]
+    void *win_k, *win_v, *pool_c;
+    const int32_t *block_table, *n_per_seq;
+    int32_t *seq_lens, *status;
+    int B, Hkv, n, D, DL, w, maxp, num_pages;
+};
+
+constexpr int kAppTok = 4;  // tokens per block
+
+// Block (token group, b): c = round_bf16(chain_e h[e] Wdown[e][a]) for the
+// group's tokens, written to their pages; ring rows of the tokens that stay in
+// the window.  The lengths are read here and advanced by latent_lens_kernel.
+__global__ void __launch_bounds__(256) latent_append_kernel(AppendArgs a)
+{
+    extern __shared__ float hs[];  // [kAppTok][D]
+    const int b = blockIdx.y, r0 = blockIdx.x * kAppTok;
+    const int nb = a.n_per_seq ? __ldg(a.n_per_seq + b) : a.n;
+    if (nb < 0 || nb > a.n) {
+        if (threadIdx.x == 0 && blockIdx.x == 0)
+            report(a.status, DAR_ERR_INVALID_ARG);
+        return;
+    }
+    if (r0 >= nb)
+        return;
+    const int L = __ldg(a.seq_lens + b);
+    const int Lnew = L + nb;
+    if (Lnew > a.maxp * kTok) {
+        if (threadIdx.x == 0)
+            report(a.status, DAR_ERR_CAPACITY);
+        return;
+    }
+    const int nt = min(kAppTok, nb - r0);
+    const bf16 *h = static_cast<const bf16 *>(a.h) + ((size_t)b * a.n + r0) * a.D;
+    for (int i = threadIdx.x; i < nt * a.D; i += blockDim.x)
+        hs[i] = __bfloat162float(h[i]);
+    // ring rows of the tokens that are still inside the window after the append
+    for (int i = threadIdx.x; i < nt * a.Hkv * 8; i += blockDim.x) {  // 16-byte chunks of 64-wide rows
+        const int t = i / (a.Hkv * 8), g = (i / 8) % a.Hkv, ch = i % 8;
+        const int p = L + r0 + t;
+        if (p < Lnew - a.w)
+            continue;
+        const size_t src = (((size_t)b * a.Hkv + g) * a.n + r0 + t) * 64 + ch * 8;
+        const size_t dst = (((size_t)b * a.Hkv + g) * a.w + p % a.w) * 64 + ch * 8;
+        reinterpret_cast<uint4 *>(a.win_k)[dst / 8] = reinterpret_cast<const uint4 *>(a.k_new)[src / 8];
+        reinterpret_cast<uint4 *>(a.win_v)[dst / 8] = reinterpret_cast<const uint4 *>(a.v_new)[src / 8];
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nt * a.DL; i += blockDim.x) {
+        const int t = i / a.DL, c = i % a.DL;
+        const int p = L + r0 + t;
+        const int pid = __ldg(a.block_table + (size_t)b * a.maxp + p / kTok);
+        if (pid < 0 || pid >= a.num_pages) {
+            report(a.status, DAR_ERR_CAPACITY);
+            continue;
+        }
+        float acc = 0.f;  // Eq. 1: one fp32 chain over e = 0..D-1 from +0
+        for (int e = 0; e < a.D; ++e)
+            acc = fmaf(hs[t * a.D + e], __ldg(a.Wdown + (size_t)e * a.DL + c), acc);
+        static_cast<bf16 *>(a.pool_c)[((size_t)pid * kTok + p % kTok) * a.DL + c] = __float2bfloat16_rn(acc);
+    }
+}
+
+__global__ void latent_lens_kernel(AppendArgs a)
+{
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= a.B)
+        return;
+    const int nb = a.n_per_seq ? a.n_per_seq[b] : a.n;
+    if (nb < 0 || nb > a.n)
+        return;
+    if (a.seq_lens[b] + nb <= a.maxp * kTok)
+        a.seq_lens[b] += nb;
+}
+
+// A[g][c][t] = chain_e Wup[c][e] W[g][e][t] (fp32), for A_K (stored as
+// [g][t][c]) and A_V (stored as [g][c][t]).
+__global__ void latent_absorb_kernel(const float *Wup, const float *WK, const float *WV, float *Ak, float *Av, int D,
+                                     int DL)
+{
+    const int g = blockIdx.y, c = blockIdx.x, t = threadIdx.x;  // 64 threads
+    const float *wk = WK + (size_t)g * D * 64, *wv = WV + (size_t)g * D * 64;
+    float ak = 0.f, av = 0.f;
+    for (int e = 0; e < D; ++e) {
+        const float u = __ldg(Wup + (size_t)c * D + e);
+        ak = fmaf(u, __ldg(wk + (size_t)e * 64 + t), ak);
+        av = fmaf(u, __ldg(wv + (size_t)e * 64 + t), av);
+    }
+    Ak[((size_t)g * 64 + t) * DL + c] = ak;  // [Hkv][d][d_lat]: the prep kernel reads rows of d_lat
+    Av[((size_t)g * DL + c) * 64 + t] = av;  // [Hkv][d_lat][d]: the merge reads rows of d
+}
+
+// ---------------------------------------------------------------- decode: prep
+
+// q~[b][h][c] = sum_t q[b][h][t] A_K[g][t][c] (fp32, stored as bf16), one
+// warp per row, lanes over c (coalesced rows of A_K).  It starts the main
+// kernel's launch at once: that kernel stages its first pages before it waits
+// for q~.
+template <int DL>
+__global__ void __launch_bounds__(256) latent_prep_kernel(Args a)
+{
+    grid_dep_launch();
+    const int lane = threadIdx.x & 31;
+    const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (row >= a.B * a.Hq)
+        return;
+    const int g = (row % a.Hq) / a.G;
+    const bf16 *qr = static_cast<const bf16 *>(a.q) + (size_t)row * 64;
+    const float q0 = __bfloat162float(qr[lane]), q1 = __bfloat162float(qr[lane + 32]);
+    const float *ak = a.Ak + (size_t)g * 64 * DL + lane;
+    float s[DL / 32];
+#pragma unroll
+    for (int e = 0; e < DL / 32; ++e)
+        s[e] = 0.f;
+#pragma unroll 16
+    for (int t = 0; t < 64; ++t) {
+        const float qv = __shfl_sync(0xffffffffu, t < 32 ? q0 : q1, t & 31);
+#pragma unroll
+        for (int e = 0; e < DL / 32; ++e)
+            s[e] = fmaf(qv, __ldg(ak + (size_t)t * DL + 32 * e), s[e]);
+    }
+#pragma unroll
+    for (int e = 0; e < DL / 32; ++e)
+        a.qt[(size_t)row * DL + 32 * e + lane] = __float2bfloat16_rn(s[e]);
+}
+
+// ---------------------------------------------------------------- decode: main
+
+// Shared-memory tiles are rows of 128 bytes (64 bf16) with the 16-byte chunk
+// index XOR (row % 8), the layout the 128-byte TMA swizzle writes; a d_lat-wide
+// row is DL / 64 such blocks of rows.
+__device__ __forceinline__ uint32_t swz(uint32_t base, int row, int chunk)
+{
+    return base + (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+template <int DL, int MT>
+struct MainLayout {
+    static constexpr uint32_t QT = 0;                              // [DL/64][MT*16][128 B]
+    static constexpr uint32_t CB = (DL * MT * 16 * 2 + 1023) / 1024 * 1024;  // two page buffers
+    static constexpr uint32_t CSTAGE = DL / 64 * 8192;             // [DL/64][64][128 B]
+    static constexpr uint32_t P = CB + 2 * CSTAGE;                 // [MT*16][128 B]
+    static constexpr uint32_t RED = P + MT * 16 * 128;             // [4][MT*16] floats
+    static constexpr uint32_t BAR = RED + 4 * MT * 16 * 4;
+    static constexpr uint32_t TOTAL = BAR + 64;
+};
+
+template <int DL, int MT>
+__global__ void __launch_bounds__(kMainThreads) latent_main_kernel(const __grid_constant__ CUtensorMap tmC, Args a)
+{
+    using Ly = MainLayout<DL, MT>;
+    constexpr int NT = DL / 32;  // n-tiles of 8 columns per warp in O
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                          ~uintptr_t(1023));
+    const uint32_t sbase = smem_u32(sm);
+    uint64_t *full = reinterpret_cast<uint64_t *>(sm + Ly::BAR);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Ly::BAR + 16);
+    float *red = reinterpret_cast<float *>(sm + Ly::RED);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int b = blockIdx.y;
+    const int L = __ldg(a.seq_lens + b);
+    grid_dep_launch();  // the merge kernel may launch; it waits for this grid to finish
+
+    if ((int)blockIdx.x >= a.nspl) {
+        // (reads q, the ring and the lengths, which the work before the prep
+        // kernel wrote: this CTA needs nothing from the prep kernel)
+        // ------------------------------------------------ window CTA: KV head g
+        const int g = blockIdx.x - a.nspl;
+        float *Ks = reinterpret_cast<float *>(sm);      // [kWinChunk][65]
+        float *Vs = Ks + kWinChunk * kWinLd;            // [kWinChunk][65]
+        float *Pw = Vs + kWinChunk * kWinLd;            // [4 warps][kWinChunk]
+        float *Qs = Pw + 4 * kWinChunk;                 // [4 warps][64]
+        if (L < 0 || L > a.maxp * kTok) {
+            if (tid == 0)
+                report(a.status, DAR_ERR_CAPACITY);
+            return;
+        }
+        const int nwin = min(L, a.w), p0 = L - nwin;
+        for (int hh0 = 0; hh0 < a.G; hh0 += 4) {
+            const int hh = hh0 + warp, h = g * a.G + hh;
+            const bool active = hh < a.G;
+            float m = -INFINITY, l = 0.f, acc0 = 0.f, acc1 = 0.f;
+            if (active) {
+                const bf16 *qr = static_cast<const bf16 *>(a.q) + ((size_t)b * a.Hq + h) * 64;
+                Qs[warp * 64 + lane] = __bfloat162float(qr[lane]) * a.c2;
+                Qs[warp * 64 + lane + 32] = __bfloat162float(qr[lane + 32]) * a.c2;
+            }
+            for (int c0 = 0; c0 < nwin; c0 += kWinChunk) {
+                const int nc = min(kWinChunk, nwin - c0);
+                __syncthreads();
+                for (int i = tid; i < nc * 8; i += kMainThreads) {  // 16-byte chunks
+                    const int j = i / 8, ch = i % 8;
+                    const int p = p0 + c0 + j;
+                    const size_t row = ((size_t)b * a.Hkv + g) * a.w + p % a.w;
+                    const uint4 kv = reinterpret_cast<const uint4 *>(a.win_k)[row * 8 + ch];
+                    const uint4 vv = reinterpret_cast<const uint4 *>(a.win_v)[row * 8 + ch];
+                    float kf[8], vf[8];
+                    unpack(kv, kf, bf16());
+                    unpack(vv, vf, bf16());
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        Ks[j * kWinLd + ch * 8 + e] = kf[e];
+                        Vs[j * kWinLd + ch * 8 + e] = vf[e];
+                    }
+                }
+                __syncthreads();
+                if (!active)
+                    continue;
+                float s[kWinChunk / 32];
+                float mx = -INFINITY;
+#pragma unroll
+                for (int u = 0; u < kWinChunk / 32; ++u) {
+                    const int j = lane + 32 * u;
+                    float acc = -INFINITY;
+                    if (j < nc) {
+                        acc = 0.f;
+#pragma unroll 16
+                        for (int t = 0; t < 64; ++t)
+                            acc = fmaf(Qs[warp * 64 + t], Ks[j * kWinLd + t], acc);
+                    }
+                    s[u] = acc;
+                    mx = fmaxf(mx, acc);
+                }
+#pragma unroll
+                for (int o = 16; o; o >>= 1)
+                    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+                const float mnew = fmaxf(m, mx);
+                const float alpha = m == -INFINITY ? 0.f : ex2_approx(m - mnew);
+                float ps = 0.f;
+#pragma unroll
+                for (int u = 0; u < kWinChunk / 32; ++u) {
+                    const float p = s[u] == -INFINITY ? 0.f : ex2_approx(s[u] - mnew);
+                    Pw[warp * kWinChunk + lane + 32 * u] = p;
+                    ps += p;
+                }
+#pragma unroll
+                for (int o = 16; o; o >>= 1)
+                    ps += __shfl_xor_sync(0xffffffffu, ps, o);
+                l = l * alpha + ps;
+                m = mnew;
+                acc0 *= alpha;
+                acc1 *= alpha;
+                __syncwarp();
+                for (int j = 0; j < nc; ++j) {
+                    const float p = Pw[warp * kWinChunk + j];
+                    acc0 = fmaf(p, Vs[j * kWinLd + lane], acc0);
+                    acc1 = fmaf(p, Vs[j * kWinLd + lane + 32], acc1);
+                }
+                __syncwarp();
+            }
+            if (active) {
+                float *rec = a.rec_win + ((size_t)b * a.Hq + h) * 66;
+                rec[lane] = acc0;
+                rec[lane + 32] = acc1;
+                if (lane == 0) {
+                    rec[64] = m;
+                    rec[65] = l;
+                }
+            }
+        }
+        return;
+    }
+
+    // ---------------------------------------------------- latent CTA: 4 pages
+    const int split = blockIdx.x;
+    const int Lg = L > a.w ? L - a.w : 0;
+    if (L > a.maxp * kTok) {
+        if (tid == 0 && split == 0)
+            report(a.status, DAR_ERR_CAPACITY);
+        return;
+    }
+    const int t0 = split * kSplitTok, t1 = min(Lg, t0 + kSplitTok);
+    if (t0 >= t1)
+        return;  // the merge reads only the splits that hold tokens
+    const int npg = (t1 - t0 + kTok - 1) / kTok;
+    if (tid == 0) {
+        mbar_init(&full[0], 1);
+        mbar_init(&full[1], 1);
+        *abort_flag = 0;
+        mbar_init_fence();
+        prefetch_tensormap(&tmC);
+    }
+    __syncthreads();
+    auto issue = [&](int pi) {  // thread 0: page pi of the split into buffer pi % 2
+        int pid = __ldg(a.block_table + (size_t)b * a.maxp + t0 / kTok + pi);
+        if (pid < 0 || pid >= a.num_pages) {
+            report(a.status, DAR_ERR_CAPACITY);
+            pid = 0;
+        }
+        uint64_t *bar = &full[pi & 1];
+        mbar_expect_tx(bar, kTok * DL * 2);
+#pragma unroll
+        for (int cb = 0; cb < DL / 64; ++cb)
+            tma_load_2d(sm + Ly::CB + (pi & 1) * Ly::CSTAGE + cb * 8192, &tmC, cb * 64, pid * kTok, bar);
+    };
+    if (tid == 0) {
+        issue(0);
+        if (npg > 1)
+            issue(1);
+    }
+    grid_dep_wait();  // q~ comes from the prep kernel
+    // q~ rows (zero past Hq) into the swizzled operand tile
+    for (int i = tid; i < MT * 16 * (DL / 8); i += kMainThreads) {
+        const int r = i / (DL / 8), ch = i % (DL / 8);
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (r < a.Hq)
+            v = *reinterpret_cast<const uint4 *>(a.qt + ((size_t)b * a.Hq + r) * DL + ch * 8);
+        *reinterpret_cast<uint4 *>(sm + Ly::QT + (ch / 8) * (MT * 16 * 128) + r * 128 +
+                                   (((ch % 8) ^ (r & 7)) << 4)) = v;
+    }
+    __syncthreads();
+
+    float o[MT][NT][4];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+            o[mt][nt][0] = o[mt][nt][1] = o[mt][nt][2] = o[mt][nt][3] = 0.f;
+    float mrun[MT][2], lpart[MT][2];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+        mrun[mt][0] = mrun[mt][1] = -INFINITY, lpart[mt][0] = lpart[mt][1] = 0.f;
+    const int grp = lane >> 2, tig = lane & 3;
+    bool ok = true;
+
+    for (int pi = 0; pi < npg; ++pi) {
+        const int s = pi & 1;
+        if (!mbar_wait(&full[s], (pi >> 1) & 1, abort_flag))
+            ok = false;
+        if (__syncthreads_or(!ok)) {
+            ok = false;
+            break;
+        }
+        const uint32_t cbuf = sbase + Ly::CB + s * Ly::CSTAGE;
+        const int ntok = min(kTok, t1 - (t0 + pi * kTok));
+        if (ntok < kTok) {  // rows past the last distant token: zero (their P is 0; 0 * NaN must not arise)
+            for (int i = tid; i < (kTok - ntok) * (DL / 8); i += kMainThreads) {
+                const int r = ntok + i / (DL / 8), ch = i % (DL / 8);
+                *reinterpret_cast<uint4 *>(sm + Ly::CB + s * Ly::CSTAGE + (ch / 8) * 8192 + r * 128 +
+                                           (((ch % 8) ^ (r & 7)) << 4)) = make_uint4(0u, 0u, 0u, 0u);
+            }
+            __syncthreads();
+        }
+        // S = Q~ C^T: this warp's 16 tokens (two n-tiles) for every head row
+        float sc[MT][2][4];
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+                sc[mt][nt][0] = sc[mt][nt][1] = sc[mt][nt][2] = sc[mt][nt][3] = 0.f;
+        {
+            const int tok = 16 * warp + (lane & 7) + ((lane >> 4) << 3);
+            const int khalf = (lane >> 3) & 1;
+#pragma unroll
+            for (int kk = 0; kk < DL / 16; ++kk) {
+                const int ch = 2 * kk + khalf;  // 16-byte chunk along d_lat
+                uint32_t bfr[4];
+                ldsm_x4(swz(cbuf + (ch / 8) * 8192, tok, ch % 8), bfr);
+#pragma unroll
+                for (int mt = 0; mt < MT; ++mt) {
+                    const int row = mt * 16 + (lane & 15), ach = 2 * kk + (lane >> 4);
+                    uint32_t afr[4];
+                    ldsm_x4(swz(sbase + Ly::QT + (ach / 8) * (MT * 16 * 128), row, ach % 8), afr);
+                    mma_bf16_16816(sc[mt][0], afr, bfr[0], bfr[1]);
+                    mma_bf16_16816(sc[mt][1], afr, bfr[2], bfr[3]);
+                }
+            }
+        }
+        // masks and per-warp row maxima
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+            float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int col = 16 * warp + 8 * nt + 2 * tig + e;
+                    if (col >= ntok)
+                        sc[mt][nt][e] = sc[mt][nt][2 + e] = -INFINITY;
+                    mx0 = fmaxf(mx0, sc[mt][nt][e]);
+                    mx1 = fmaxf(mx1, sc[mt][nt][2 + e]);
+                }
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+            if (tig == 0) {
+                red[warp * MT * 16 + mt * 16 + grp] = mx0;
+                red[warp * MT * 16 + mt * 16 + grp + 8] = mx1;
+            }
+        }
+        __syncthreads();
+        // running maxima (log2 units), P = 2^(s c2 - m) into shared memory, rescale O
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+                const int row = mt * 16 + grp + 8 * hr;
+                float tmax = red[row];
+#pragma unroll
+                for (int w2 = 1; w2 < 4; ++w2)
+                    tmax = fmaxf(tmax, red[w2 * MT * 16 + row]);
+                const float mnew = fmaxf(mrun[mt][hr], tmax * a.c2);
+                const float alpha = mrun[mt][hr] == -INFINITY ? 0.f : ex2_approx(mrun[mt][hr] - mnew);
+                mrun[mt][hr] = mnew;
+                lpart[mt][hr] *= alpha;
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                    o[mt][nt][2 * hr] *= alpha;
+                    o[mt][nt][2 * hr + 1] *= alpha;
+                }
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt) {
+                    const float x0 = sc[mt][nt][2 * hr], x1 = sc[mt][nt][2 * hr + 1];
+                    const float p0 = x0 == -INFINITY ? 0.f : ex2_approx(fmaf(x0, a.c2, -mnew));
+                    const float p1 = x1 == -INFINITY ? 0.f : ex2_approx(fmaf(x1, a.c2, -mnew));
+                    const uint32_t pk = cvt_bf16x2(p0, p1);
+                    lpart[mt][hr] += bf16lo(pk) + bf16hi(pk);  // the weights the PV product uses
+                    const int col = 16 * warp + 8 * nt + 2 * tig;
+                    *reinterpret_cast<uint32_t *>(sm + Ly::P + row * 128 + (((col >> 3) ^ (row & 7)) << 4) +
+                                                  4 * tig) = pk;
+                }
+            }
+        __syncthreads();
+        // O += P C: this warp's DL/4 columns, K = the page's 64 tokens
+#pragma unroll
+        for (int kk = 0; kk < kTok / 16; ++kk) {
+            uint32_t afr[MT][4];
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt)
+                ldsm_x4(swz(sbase + Ly::P, mt * 16 + (lane & 15), 2 * kk + (lane >> 4)), afr[mt]);
+            const int krow = 16 * kk + (lane & 7) + (((lane >> 3) & 1) << 3);
+#pragma unroll
+            for (int np = 0; np < NT / 2; ++np) {
+                const int n0 = warp * (DL / 4) + 16 * np + ((lane >> 4) << 3);  // column of this lane's matrix
+                uint32_t bfr[4];
+                ldsm_x4_t(swz(cbuf + (n0 / 64) * 8192, krow, (n0 % 64) / 8), bfr);
+#pragma unroll
+                for (int mt = 0; mt < MT; ++mt) {
+                    mma_bf16_16816(o[mt][2 * np], afr[mt], bfr[0], bfr[1]);
+                    mma_bf16_16816(o[mt][2 * np + 1], afr[mt], bfr[2], bfr[3]);
+                }
+            }
+        }
+        __syncthreads();  // buffer s and P are free again
+        if (tid == 0 && pi + 2 < npg) {
+            fence_proxy_async_smem();
+            issue(pi + 2);
+        }
+    }
+    if (!ok) {
+        // let copies still in flight land before the CTA exits
+        if (tid == 0) {
+            for (int pi = 0; pi < npg && pi < 2; ++pi)
+                mbar_wait(&full[pi & 1], 0, nullptr);
+            report(a.status, DAR_ERR_DEVICE);
+        }
+        return;
+    }
+
+    // row sums: across the quad, then across the four warps
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int hr = 0; hr < 2; ++hr) {
+            float ls = lpart[mt][hr];
+            ls += __shfl_xor_sync(0xffffffffu, ls, 1);
+            ls += __shfl_xor_sync(0xffffffffu, ls, 2);
+            lpart[mt][hr] = ls;
+        }
+    __syncthreads();
+    if (tig == 0)
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+            red[warp * MT * 16 + mt * 16 + grp] = lpart[mt][0];
+            red[warp * MT * 16 + mt * 16 + grp + 8] = lpart[mt][1];
+        }
+    __syncthreads();
+    const size_t rbase = ((size_t)b * a.nspl + split) * a.Hq;
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int hr = 0; hr < 2; ++hr) {
+            const int row = mt * 16 + grp + 8 * hr;
+            if (row >= a.Hq)
+                continue;
+            float *rec = a.rec_lat + (rbase + row) * (DL + 2);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                const int col = warp * (DL / 4) + 8 * nt + 2 * tig;
+                *reinterpret_cast<float2 *>(rec + col) = make_float2(o[mt][nt][2 * hr], o[mt][nt][2 * hr + 1]);
+            }
+            if (warp == 0 && tig == 0) {
+                rec[DL] = mrun[mt][hr];
+                rec[DL + 1] = red[row] + red[MT * 16 + row] + red[2 * MT * 16 + row] + red[3 * MT * 16 + row];
+            }
+        }
+}
+
+// ---------------------------------------------------------------- decode: merge
+
+// One warp per (b, h): combine the window record and the sequence's latent
+// splits (log-sum-exp), lift the latent sum with A_V, divide.
+template <int DL>
+__global__ void __launch_bounds__(128) latent_merge_kernel(Args a)
+{
+    __shared__ float olat[4][DL];
+    __shared__ float fs[4][32];
+    grid_dep_wait();  // the main kernel's records
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int row = blockIdx.x * 4 + warp;
+    const bool active = row < a.B * a.Hq;
+    const int b = active ? row / a.Hq : 0, h = active ? row % a.Hq : 0, g = h / a.G;
+    int L = active ? __ldg(a.seq_lens + b) : 0;
+    if (L < 0 || L > a.maxp * kTok)
+        L = 0;  // reported by the main kernel; the output is undefined then
+    const int Lg = L > a.w ? L - a.w : 0;
+    const int ns = (Lg + kSplitTok - 1) / kSplitTok;
+    const float *rw = a.rec_win + (size_t)row * 66;
+    const float *rl0 = a.rec_lat + ((size_t)b * a.nspl * a.Hq + h) * (DL + 2);  // split s at + s * Hq * (DL + 2)
+    const size_t sstride = (size_t)a.Hq * (DL + 2);
+    const float mw = L > 0 ? rw[64] : -INFINITY;
+    // the splits' maxima and sums, one split per lane (32 at a time)
+    float M = mw;
+    for (int s = lane; s < ns; s += 32)
+        M = fmaxf(M, rl0[s * sstride + DL]);
+#pragma unroll
+    for (int o = 16; o; o >>= 1)
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    float l = 0.f;
+    float acc[DL / 32];
+#pragma unroll
+    for (int e = 0; e < DL / 32; ++e)
+        acc[e] = 0.f;
+    for (int s0 = 0; s0 < ns; s0 += 32) {
+        float f = 0.f;
+        if (s0 + lane < ns) {
+            const float *rl = rl0 + (s0 + lane) * sstride;
+            f = ex2_approx(rl[DL] - M);
+            l += f * rl[DL + 1];
+        }
+        fs[warp][lane] = f;
+        __syncwarp();
+        const int n = min(32, ns - s0);
+#pragma unroll 4
+        for (int j = 0; j < n; ++j) {
+            const float *rl = rl0 + (s0 + j) * sstride;
+            const float fj = fs[warp][j];
+#pragma unroll
+            for (int e = 0; e < DL / 32; ++e)
+                acc[e] = fmaf(fj, rl[lane + 32 * e], acc[e]);
+        }
+        __syncwarp();
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1)
+        l += __shfl_xor_sync(0xffffffffu, l, o);
+    const float fw = L > 0 ? ex2_approx(mw - M) : 0.f;
+    if (L > 0)
+        l += fw * rw[65];
+#pragma unroll
+    for (int e = 0; e < DL / 32; ++e)
+        olat[warp][lane + 32 * e] = acc[e];
+    __syncwarp();
+    if (!active)
+        return;
+    float o0 = L > 0 ? fw * rw[lane] : 0.f, o1 = L > 0 ? fw * rw[lane + 32] : 0.f;
+    const float *av = a.Av + (size_t)g * DL * 64;
+#pragma unroll 16
+    for (int c = 0; c < DL; ++c) {
+        const float x = olat[warp][c];
+        o0 = fmaf(x, __ldg(av + c * 64 + lane), o0);
+        o1 = fmaf(x, __ldg(av + c * 64 + lane + 32), o1);
+    }
+    const float inv = l > 0.f ? 1.f / l : 0.f;
+    bf16 *out = static_cast<bf16 *>(a.out) + (size_t)row * 64;
+    out[lane] = __float2bfloat16_rn(o0 * inv);
+    out[lane + 32] = __float2bfloat16_rn(o1 * inv);
+}
+
+// ---------------------------------------------------------------- host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+template <int DL, int MT>
+static cudaError_t decode_t(const Args &a, const void *pool_c, cudaStream_t s)
+{
+    using Ly = MainLayout<DL, MT>;
+    constexpr size_t win_smem = (2 * kWinChunk * kWinLd + 4 * kWinChunk + 4 * 64) * sizeof(float);
+    const size_t smem = 1024 + (Ly::TOTAL > win_smem ? Ly::TOTAL : win_smem);
+    static PerDeviceOnce once;
+    cudaError_t e = per_device_once(once, [&](int) {
+        return cudaFuncSetAttribute(latent_main_kernel<DL, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)smem);
+    });
+    if (e != cudaSuccess)
+        return e;
+    EncodeTiledFn enc = encode_fn();
+    if (!enc)
+        return cudaErrorNotSupported;
+    CUtensorMap tm;
+    const cuuint64_t dims[2] = {(cuuint64_t)DL, (cuuint64_t)a.num_pages * kTok};
+    const cuuint64_t strides[1] = {(cuuint64_t)DL * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)kTok};
+    const cuuint32_t estr[2] = {1, 1};
+    if (enc(&tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(pool_c), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+    const int rows = a.B * a.Hq;
+    // prep starts after all earlier work on the stream; main and merge are
+    // launched programmatically (each waits in-kernel for what it reads)
+    latent_prep_kernel<DL><<<(rows + 7) / 8, 256, 0, s>>>(a);
+    cudaLaunchAttribute pdl[1];
+    pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    pdl[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.stream = s;
+    cfg.attrs = pdl;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(a.nspl + a.Hkv, a.B);
+    cfg.blockDim = dim3(kMainThreads);
+    cfg.dynamicSmemBytes = smem;
+    e = cudaLaunchKernelEx(&cfg, latent_main_kernel<DL, MT>, tm, a);
+    if (e != cudaSuccess)
+        return e;
+    cfg.gridDim = dim3((rows + 3) / 4);
+    cfg.blockDim = dim3(128);
+    cfg.dynamicSmemBytes = 0;
+    e = cudaLaunchKernelEx(&cfg, latent_merge_kernel<DL>, a);
+    if (e != cudaSuccess)
+        return e;
+    return cudaGetLastError();
+}
+
+template <int DL>
+static cudaError_t decode_dl(const Args &a, const void *pool_c, cudaStream_t s)
+{
+    return a.Hq <= 16 ? decode_t<DL, 1>(a, pool_c, s) : decode_t<DL, 2>(a, pool_c, s);
+}
+
+}  // namespace lat
+
+size_t latent_decode_workspace_bytes(int B, int Hq, int DL, int maxp)
+{
+    auto al = [](size_t x) { return (x + 255) & ~size_t(255); };
+    const size_t nspl = (size_t)(maxp + lat::kPagesPerSplit - 1) / lat::kPagesPerSplit;
+    return al((size_t)B * Hq * DL * 2) + al((size_t)B * nspl * Hq * (DL + 2) * 4) + al((size_t)B * Hq * 66 * 4);
+}
+
+cudaError_t launch_latent_decode(const LatentDecodeArgs &x, void *workspace, cudaStream_t s)
+{
+    if (x.B == 0)
+        return cudaSuccess;
+    auto al = [](size_t v) { return (v + 255) & ~size_t(255); };
+    lat::Args a;
+    a.q = x.q;
+    a.out = x.out;
+    a.win_k = x.win_k;
+    a.win_v = x.win_v;
+    a.block_table = x.block_table;
+    a.seq_lens = x.seq_lens;
+    a.status = x.status;
+    a.Ak = x.Ak;
+    a.Av = x.Av;
+    a.B = x.B;
+    a.Hq = x.Hq;
+    a.Hkv = x.Hkv;
+    a.G = x.Hq / x.Hkv;
+    a.w = x.w;
+    a.maxp = x.maxp;
+    a.num_pages = x.num_pages;
+    a.nspl = (x.maxp + lat::kPagesPerSplit - 1) / lat::kPagesPerSplit;
+    a.c2 = x.scale * 1.4426950408889634f;
+    char *p = static_cast<char *>(workspace);
+    a.qt = reinterpret_cast<bf16 *>(p);
+    p += al((size_t)x.B * x.Hq * x.DL * 2);
+    a.rec_lat = reinterpret_cast<float *>(p);
+    p += al((size_t)x.B * a.nspl * x.Hq * (x.DL + 2) * 4);
+    a.rec_win = reinterpret_cast<float *>(p);
+    switch (x.DL) {
+    case 64: return lat::decode_dl<64>(a, x.pool_c, s);
+    case 128: return lat::decode_dl<128>(a, x.pool_c, s);
+    case 192: return lat::decode_dl<192>(a, x.pool_c, s);
+    case 256: return lat::decode_dl<256>(a, x.pool_c, s);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_latent_append(const LatentAppendArgs &x, cudaStream_t s)
+{
+    if (x.B == 0 || x.n == 0)
+        return cudaSuccess;
+    lat::AppendArgs a;
+    a.h = x.h;
+    a.k_new = x.k_new;
+    a.v_new = x.v_new;
+    a.Wdown = x.Wdown;
+    a.win_k = x.win_k;
+    a.win_v = x.win_v;
+    a.pool_c = x.pool_c;
+    a.block_table = x.block_table;
+    a.n_per_seq = x.n_per_seq;
+    a.seq_lens = x.seq_lens;
+    a.status = x.status;
+    a.B = x.B;
+    a.Hkv = x.Hkv;
+    a.n = x.n;
+    a.D = x.D;
+    a.DL = x.DL;
+    a.w = x.w;
+    a.maxp = x.maxp;
+    a.num_pages = x.num_pages;
+    const size_t smem = (size_t)lat::kAppTok * x.D * sizeof(float);
+    static PerDeviceOnce once;
+    cudaError_t e = per_device_once(once, [&](int) {
+        return cudaFuncSetAttribute(lat::latent_append_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)(lat::kAppTok * 8192 * sizeof(float)));
+    });
+    if (e != cudaSuccess)
+        return e;
+    lat::latent_append_kernel<<<dim3((x.n + lat::kAppTok - 1) / lat::kAppTok, x.B), 256, smem, s>>>(a);
+    lat::latent_lens_kernel<<<(x.B + 255) / 256, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_latent_absorb(const float *Wup, const float *WK, const float *WV, float *Ak, float *Av, int Hkv,
+                                 int D, int DL, cudaStream_t s)
+{
+    lat::latent_absorb_kernel<<<dim3(DL, Hkv), 64, 0, s>>>(Wup, WK, WV, Ak, Av, D, DL);
+    return cudaGetLastError();
+}
+
+}  // namespace dar

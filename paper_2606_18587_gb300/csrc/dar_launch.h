@@ -124,6 +124,31 @@ struct BackwardArgs {
 size_t backward_workspace_bytes(dar_dtype dt, int B, int Hq, int Hkv, int N, int dd);
 cudaError_t launch_backward(dar_dtype dt, const BackwardArgs &a, void *workspace, cudaStream_t s);
 
+// The latent form (dar_latent.cu): one bottleneck per token shared by all heads.
+struct LatentAppendArgs {
+    const void *h, *k_new, *v_new;
+    const float *Wdown;
+    void *win_k, *win_v, *pool_c;
+    const int32_t *block_table, *n_per_seq;
+    int32_t *seq_lens, *status;
+    int B, Hkv, n, D, DL, w, maxp, num_pages;
+};
+struct LatentDecodeArgs {
+    const void *q;
+    void *out;
+    const void *win_k, *win_v, *pool_c;
+    const int32_t *block_table, *seq_lens;
+    int32_t *status;
+    const float *Ak, *Av;
+    int B, Hq, Hkv, DL, w, maxp, num_pages;
+    float scale;
+};
+size_t latent_decode_workspace_bytes(int B, int Hq, int DL, int maxp);
+cudaError_t launch_latent_append(const LatentAppendArgs &a, cudaStream_t s);
+cudaError_t launch_latent_absorb(const float *Wup, const float *WK, const float *WV, float *Ak, float *Av, int Hkv,
+                                 int D, int DL, cudaStream_t s);
+cudaError_t launch_latent_decode(const LatentDecodeArgs &a, void *workspace, cudaStream_t s);
+
 // Chunked prefill over a cache: gather kernel, attention (chunk mode), then
 // the cache append of the chunk.  Buffers of the workspace (see dar_abi.cu).
 struct ChunkArgs {

@@ -26,16 +26,18 @@
 // (x = s * scale * log2(e) - m), one conversion of the pair to bf16x2 and one
 // bf16x2 exp2, whose result is the packed bf16 P the PV product reads.
 //
-// Warp roles (224 threads): warp 0 issues TMA loads, warp 6 the S products
+// Warp roles (352 threads): warp 0 issues TMA loads, warp 10 the S products
 // (and q~), warp 1 allocates TMEM and issues the PV products (each issuing
-// warp runs its loop together; one elected lane issues), warps 2-5 own one
-// query row per thread (TMEM lane = row) for the softmax and the epilogue.
-// The softmax writes P into TMEM over the S it came from, where the PV
-// products take it as their A operand; with two, later three, S buffers the
-// S products run ahead of the softmax and only wait for the PV that last read
-// a buffer.  Two CTAs share an SM (256 TMEM columns and ~110 KB of shared
-// memory each), so one CTA's softmax overlaps the other's waits.  Every wait
-// is bounded; on a timeout the CTA flags *status and exits.
+// warp runs its loop together; one elected lane issues), warps 2-9 run the
+// softmax and the epilogue, four threads per query row (TMEM lanes through
+// the 16-lane load/store shapes; a row's maximum is combined with shuffles).
+// For d_down <= 32 the softmax writes P into TMEM over the S it came from
+// (two S buffers), where the PV products take it as their A operand, so the S
+// products run a tile ahead of the softmax and only wait for the PV that last
+// read a buffer; d_down = 64 keeps one S buffer and P in columns of its own.
+// Two CTAs share an SM (256 TMEM columns each), so one CTA's softmax overlaps
+// the other's waits.  Every wait is bounded; on a timeout the CTA flags
+// *status and exits.
 #include <cuda.h>
 
 #include "dar_common.cuh"

@@ -43,6 +43,16 @@ class dar_cache(ctypes.Structure):
     ]
 
 
+class dar_latent_cache(ctypes.Structure):
+    _fields_ = [
+        ("B", ctypes.c_int32), ("Hkv", ctypes.c_int32), ("d", ctypes.c_int32), ("D", ctypes.c_int32),
+        ("d_lat", ctypes.c_int32), ("w", ctypes.c_int32),
+        ("max_pages_per_seq", ctypes.c_int32), ("num_pages", ctypes.c_int32),
+        ("win_k", ctypes.c_void_p), ("win_v", ctypes.c_void_p), ("pool_c", ctypes.c_void_p),
+        ("block_table", ctypes.c_void_p), ("seq_lens", ctypes.c_void_p), ("status", ctypes.c_void_p),
+    ]
+
+
 _lib = None
 
 
@@ -56,6 +66,7 @@ def load_library(path: str = LIB_PATH):
                            "`python -c 'import __graft_entry__ as g; g.build()'`")
     lib = ctypes.CDLL(path)
     P, I32, SZ, F = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t, ctypes.c_float
+    LP = ctypes.POINTER(dar_latent_cache)
     CP = ctypes.POINTER(dar_cache)
     sig = {
         "dar_down_project": ([ctypes.c_int, I32, I32, I32, I32, I32, P, P, P, P], ctypes.c_int),
@@ -76,6 +87,10 @@ def load_library(path: str = LIB_PATH):
         "dar_attn_backward_workspace_bytes": ([ctypes.c_int, I32, I32, I32, I32, I32], SZ),
         "dar_attn_backward": ([ctypes.c_int, I32, I32, I32, I32, I32, I32, I32] + [P] * 9 + [F] + [P] * 8 + [SZ, P],
                               ctypes.c_int),
+        "dar_latent_append": ([LP, P, P, P, I32, P, P, P], ctypes.c_int),
+        "dar_latent_absorb": ([I32, I32, I32, I32, P, P, P, P, P, P], ctypes.c_int),
+        "dar_latent_decode_workspace_bytes": ([LP, I32], SZ),
+        "dar_latent_decode": ([LP, I32, P, P, P, F, P, P, SZ, P], ctypes.c_int),
         "dar_last_error": ([], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -414,4 +429,88 @@ def dar_prefill_chunk(cache: DarCache, q, k_new, v_new, Dk, Uk, Dv, Uv, scale=0.
     _check(load_library().dar_prefill_chunk(
         cache.struct, Hq, n, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(Dk), _ptr(Uk), _ptr(Dv), _ptr(Uv),
         float(scale), _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+    return out
+
+
+# --------------------------------------------------------------------------- latent form
+
+class DarLatentCache:
+    """Caller-owned cache of the latent form (one bottleneck per token shared
+    by all heads, keys and values; full keys/values for the last ``w``
+    tokens), and its ``dar_latent_cache`` struct.  bf16."""
+
+    def __init__(self, B, Hkv, D, d_lat, w, max_pages_per_seq, num_pages=None, block_table=None, device="cuda",
+                 d=64):
+        self.B, self.Hkv, self.d, self.D, self.d_lat, self.w = B, Hkv, d, D, d_lat, w
+        self.dtype = torch.bfloat16
+        self.max_pages_per_seq = max_pages_per_seq
+        if num_pages is None:
+            num_pages = B * max_pages_per_seq
+        self.num_pages = num_pages
+        self.win_k = torch.zeros((B, Hkv, w, d), dtype=torch.bfloat16, device=device)
+        self.win_v = torch.zeros_like(self.win_k)
+        self.pool_c = torch.zeros((max(num_pages, 1), PAGE_SIZE, d_lat), dtype=torch.bfloat16, device=device)
+        if block_table is None:
+            block_table = torch.arange(B * max_pages_per_seq, dtype=torch.int32).reshape(B, max_pages_per_seq)
+        self.block_table = torch.as_tensor(block_table, dtype=torch.int32).to(device).contiguous()
+        self.seq_lens = torch.zeros(B, dtype=torch.int32, device=device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
+        self._struct = dar_latent_cache(
+            B, Hkv, d, D, d_lat, w, max_pages_per_seq, num_pages, self.win_k.data_ptr(), self.win_v.data_ptr(),
+            self.pool_c.data_ptr(), self.block_table.data_ptr(), self.seq_lens.data_ptr(), self.status.data_ptr())
+
+    @property
+    def struct(self):
+        return ctypes.byref(self._struct)
+
+    def device_status(self) -> int:
+        return int(self.status.item())
+
+
+def dar_latent_append(cache: DarLatentCache, h_new, k_new, v_new, W_down, n_per_seq=None, stream=None):
+    """Append tokens: hidden states ``h_new [B,n,D]`` (their bottleneck c = h W_down
+    is computed and cached), keys/values ``k_new, v_new [B,Hkv,n,d]``."""
+    _dev(h_new, "h_new", torch.bfloat16)
+    _dev(k_new, "k_new", torch.bfloat16)
+    _dev(v_new, "v_new", torch.bfloat16)
+    _dev(W_down, "W_down", torch.float32)
+    if n_per_seq is not None:
+        _dev(n_per_seq, "n_per_seq", torch.int32)
+    _check(load_library().dar_latent_append(cache.struct, _ptr(h_new), _ptr(k_new), _ptr(v_new), k_new.shape[2],
+                                            _ptr(n_per_seq), _ptr(W_down), _stream(stream)))
+
+
+def dar_latent_absorb(W_up, W_K, W_V, stream=None):
+    """``A_K = W_up W_K``, ``A_V = W_up W_V`` per KV head: ``W_up [d_lat,D]``,
+    ``W_K, W_V [Hkv,D,d]`` -> ``A_K [Hkv,d,d_lat]`` (transposed) and ``A_V
+    [Hkv,d_lat,d]``, fp32."""
+    for name, t in (("W_up", W_up), ("W_K", W_K), ("W_V", W_V)):
+        _dev(t, name, torch.float32)
+    Hkv, D, d = W_K.shape
+    d_lat = W_up.shape[0]
+    A_K = torch.empty((Hkv, d, d_lat), dtype=torch.float32, device=W_up.device)
+    A_V = torch.empty((Hkv, d_lat, d), dtype=torch.float32, device=W_up.device)
+    _check(load_library().dar_latent_absorb(Hkv, D, d, d_lat, _ptr(W_up), _ptr(W_K), _ptr(W_V), _ptr(A_K),
+                                            _ptr(A_V), _stream(stream)))
+    return A_K, A_V
+
+
+def latent_decode_workspace(cache: DarLatentCache, Hq: int):
+    nbytes = int(load_library().dar_latent_decode_workspace_bytes(cache.struct, Hq))
+    if nbytes == 0:
+        raise DarError(DAR_ERR_INVALID_ARG, dar_last_error() or "bad latent cache/Hq")
+    return torch.empty(nbytes, dtype=torch.uint8, device=cache.win_k.device)
+
+
+def dar_latent_decode(cache: DarLatentCache, q, A_K, A_V, workspace, scale=0.0, out=None, stream=None):
+    """One decode step of the latent form for ``q [B,Hq,d]`` (bf16)."""
+    _dev(q, "q", torch.bfloat16)
+    _dev(A_K, "A_K", torch.float32)
+    _dev(A_V, "A_V", torch.float32)
+    _dev(workspace, "workspace")
+    if out is None:
+        out = torch.empty_like(q)
+    _dev(out, "out", torch.bfloat16)
+    _check(load_library().dar_latent_decode(cache.struct, q.shape[1], _ptr(q), _ptr(A_K), _ptr(A_V), float(scale),
+                                            _ptr(out), _ptr(workspace), workspace.numel(), _stream(stream)))
     return out

@@ -162,6 +162,41 @@ def sweep_point(k: int) -> Decode:
                   "bf16", L=16384)
 
 
+@dataclasses.dataclass(frozen=True)
+class LatentDecode:
+    """A decode workload of the latent form: hidden width D, bottleneck d_lat."""
+    name: str
+    seed: int
+    B: int
+    Hq: int
+    Hkv: int
+    d: int
+    D: int
+    dl: int
+    w: int
+    L: Optional[int] = None
+    L_range: Optional[tuple] = None
+    shuffle_pages: bool = False
+    dtype: str = "bf16"
+
+
+DECODE_160M_LATENT = LatentDecode("decode-160M-latent bf16 B32 H12 L4096 d64 D768 dlat192 w128", 1021,
+                                  32, 12, 12, 64, 768, 192, 128, L=4096)
+DECODE_1B_LATENT = LatentDecode("decode-1B-latent-GQA paged bf16 B64 Hq32 Hkv8 L[1024,8192] d64 D2048 dlat256 w256",
+                                1023, 64, 32, 8, 64, 2048, 256, 256, L_range=(1024, 8192), shuffle_pages=True)
+
+
+def latent_history(cfg: LatentDecode, b: int, L: Optional[int] = None):
+    """Hidden states [L, D] and keys/values [Hkv, L, d] of every token of
+    sequence b, N(0, 1) in the storage type (one stream per sequence)."""
+    if L is None:
+        L = int(decode_lengths(cfg)[b])
+    h = normal_array(cfg.seed, S_H, (L, cfg.D), dtype=cfg.dtype, sub=b + 1)
+    k = normal_array(cfg.seed, S_K, (cfg.Hkv, L, cfg.d), dtype=cfg.dtype, sub=b + 1)
+    v = normal_array(cfg.seed, S_V, (cfg.Hkv, L, cfg.d), dtype=cfg.dtype, sub=b + 1)
+    return h, k, v
+
+
 def prefill_inputs(cfg: Prefill):
     """q [B,Hq,N,d], k, v [B,Hkv,N,d] (storage type) and the four projections."""
     s = cfg.seed

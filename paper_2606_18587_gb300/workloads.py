@@ -132,6 +132,71 @@ def append_step_bytes(cfg: I.Decode, lens) -> int:
     return cfg.Hkv * (cfg.B * per_head_new + migrating * per_head_mig)
 
 
+class LatentDecodeWorkload:
+    """A filled cache of the latent form for an :class:`inputs.LatentDecode`
+    config: every token's hidden state goes through ``dar_latent_append``
+    (which computes its bottleneck), in chunks, with per-sequence counts; the
+    absorbed maps come from ``dar_latent_absorb``."""
+
+    def __init__(self, cfg: I.LatentDecode, extra_tokens=0, chunk=1024, device="cuda", keep_history=False):
+        self.cfg = cfg
+        self.lens = I.decode_lengths(cfg)
+        cap = self.lens + extra_tokens
+        table, num_pages = I.page_assignment(cfg, cap)
+        self.cache = dar.DarLatentCache(cfg.B, cfg.Hkv, cfg.D, cfg.dl, cfg.w, table.shape[1], num_pages,
+                                        block_table=torch.from_numpy(table), device=device)
+        self.proj_host = I.latent_projections(cfg.seed, cfg.Hkv, cfg.D, cfg.dl, cfg.d)
+        self.Wdown, Wup, WK, WV = (upload(x, "f32", device) for x in self.proj_host)
+        self.A_K, self.A_V = dar.dar_latent_absorb(Wup, WK, WV)
+        hist = [I.latent_history(cfg, b, int(self.lens[b])) for b in range(cfg.B)]
+        self.history = hist if keep_history else None
+        Lmax = int(self.lens.max())
+        for t0 in range(0, Lmax, chunk):
+            n = min(chunk, Lmax - t0)
+            hc = np.zeros((cfg.B, n, cfg.D), dtype=np.uint16)
+            kc = np.zeros((cfg.B, cfg.Hkv, n, cfg.d), dtype=np.uint16)
+            vc = np.zeros_like(kc)
+            counts = np.clip(self.lens - t0, 0, n).astype(np.int32)
+            for b in range(cfg.B):
+                c = int(counts[b])
+                if c:
+                    hb, kb, vb = hist[b]
+                    hc[b, :c], kc[b, :, :c], vc[b, :, :c] = hb[t0:t0 + c], kb[:, t0:t0 + c], vb[:, t0:t0 + c]
+            dar.dar_latent_append(self.cache, upload(hc, "bf16", device), upload(kc, "bf16", device),
+                                  upload(vc, "bf16", device), self.Wdown,
+                                  n_per_seq=torch.from_numpy(counts).to(device))
+        torch.cuda.synchronize()
+        self.q_host = I.normal_array(cfg.seed, I.S_QDEC, (cfg.B, cfg.Hq, cfg.d), dtype=cfg.dtype)
+        self.q = upload(self.q_host, "bf16", device)
+        self.workspace = dar.latent_decode_workspace(self.cache, cfg.Hq)
+
+    def history_arrays(self, seqs):
+        """Zero-padded histories of the listed sequences for the oracle:
+        ``k, v [n,Hkv,Lmax,d]`` and ``h [n,Lmax,D]``."""
+        cfg = self.cfg
+        Lm = max(int(self.lens[b]) for b in seqs)
+        k = np.zeros((len(seqs), cfg.Hkv, Lm, cfg.d), dtype=np.uint16)
+        v = np.zeros_like(k)
+        h = np.zeros((len(seqs), Lm, cfg.D), dtype=np.uint16)
+        for i, b in enumerate(seqs):
+            hb, kb, vb = self.history[b]
+            h[i, :hb.shape[0]], k[i, :, :kb.shape[1]], v[i, :, :vb.shape[1]] = hb, kb, vb
+        return k, v, h
+
+    def decode(self, out=None, stream=None):
+        return dar.dar_latent_decode(self.cache, self.q, self.A_K, self.A_V, self.workspace, out=out, stream=stream)
+
+
+def latent_decode_bytes(cfg: I.LatentDecode, lens) -> int:
+    """Algorithmic bytes of one latent decode call: per sequence the window's
+    keys and values per KV head at d, the bottleneck of each distant token once
+    (d_lat, shared by every head), and the queries and outputs."""
+    e = ESIZE[cfg.dtype]
+    lens = np.asarray(lens, dtype=np.int64)
+    nwin = np.minimum(lens, cfg.w)
+    return int(np.sum(cfg.Hkv * nwin * 2 * cfg.d * e + (lens - nwin) * cfg.dl * e) + 2 * cfg.B * cfg.Hq * cfg.d * e)
+
+
 # ------------------------------------------------------------------------ prefill
 
 def prefill_pairs(N: int, w: int):
