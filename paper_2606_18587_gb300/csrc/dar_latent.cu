@@ -15,8 +15,8 @@
 //    inputs per element, rounded once to bf16) into the page of every new
 //    token; new keys/values into the ring; then the lengths.
 //  - latent_absorb: A_K, A_V (fp32 chains over D).
-//  - decode: prep (q~ = q A_K^T, bf16), main (latent splits of four pages
-//    each: TMA-staged pages, S = Q~ C^T and O += P C on mma.sync tensor
+//  - decode: prep (q~ = q A_K^T, bf16), main (latent splits of eight pages
+//    each: TMA-staged pages in a ring of two or three buffers, S = Q~ C^T and O += P C on mma.sync tensor
 //    cores, one online softmax per head; plus one CTA per KV head for the
 //    window on the CUDA cores), merge (exact log-sum-exp combination of the
 //    partial results, then o = (O_loc + O_lat A_V) / l).
@@ -34,7 +34,7 @@ namespace lat {
 using namespace sm100;
 
 constexpr int kTok = DAR_PAGE_SIZE;  // tokens per page
-constexpr int kPagesPerSplit = 4;
+constexpr int kPagesPerSplit = 8;
 constexpr int kSplitTok = kTok * kPagesPerSplit;
 constexpr int kMainThreads = 128;
 constexpr int kWinChunk = 64;  // window tokens staged at a time
@@ -152,36 +152,64 @@ __global__ void latent_absorb_kernel(const float *Wup, const float *WK, const fl
 
 // ---------------------------------------------------------------- decode: prep
 
-// q~[b][h][c] = sum_t q[b][h][t] A_K[g][t][c] (fp32, stored as bf16), one
-// warp per row, lanes over c (coalesced rows of A_K).  It starts the main
-// kernel's launch at once: that kernel stages its first pages before it waits
-// for q~.
-template <int DL>
-__global__ void __launch_bounds__(256) latent_prep_kernel(Args a)
+// q~[b][h][c] = sum_t q[b][h][t] A_K[g][t][c] (fp32, stored as bf16).  Block
+// (g, 4 rows of KV head g): A_K^g staged in shared memory by one bulk copy,
+// then one warp per row, lanes over c.  It starts the main kernel's launch at once: that
+// kernel stages its first pages before it waits for q~.
+constexpr int kRowsPerBlock = 4;  // rows (one per warp) of one KV head per block
+
+// One bulk asynchronous copy of `bytes` (a multiple of 16) from global to
+// shared memory, waited for by the whole block (bounded; on a timeout the
+// status is flagged and false returned).
+__device__ __forceinline__ bool stage_matrix(void *dst, const void *src, unsigned bytes, uint64_t *bar,
+                                             int32_t *status)
 {
+    if (threadIdx.x == 0) {
+        mbar_init(bar, 1);
+        mbar_init_fence();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        mbar_expect_tx(bar, bytes);
+        for (unsigned off = 0; off < bytes; off += 16384u)  // in copies of at most 16 KB
+            bulk_g2s(static_cast<char *>(dst) + off, static_cast<const char *>(src) + off,
+                     bytes - off < 16384u ? bytes - off : 16384u, bar);
+    }
+    const bool ok = mbar_wait(bar, 0, nullptr);
+    if (!ok && threadIdx.x == 0)
+        report(status, DAR_ERR_DEVICE);
+    return __syncthreads_and(ok) != 0;
+}
+
+template <int DL>
+__global__ void __launch_bounds__(128) latent_prep_kernel(Args a)
+{
+    extern __shared__ __align__(16) float aks[];  // [64][DL], then the barrier
     grid_dep_launch();
-    const int lane = threadIdx.x & 31;
-    const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
-    if (row >= a.B * a.Hq)
+    const int g = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (!stage_matrix(aks, a.Ak + (size_t)g * 64 * DL, 64 * DL * 4, reinterpret_cast<uint64_t *>(aks + 64 * DL),
+                      a.status))
         return;
-    const int g = (row % a.Hq) / a.G;
-    const bf16 *qr = static_cast<const bf16 *>(a.q) + (size_t)row * 64;
-    const float q0 = __bfloat162float(qr[lane]), q1 = __bfloat162float(qr[lane + 32]);
-    const float *ak = a.Ak + (size_t)g * 64 * DL + lane;
-    float s[DL / 32];
-#pragma unroll
-    for (int e = 0; e < DL / 32; ++e)
-        s[e] = 0.f;
-#pragma unroll 16
-    for (int t = 0; t < 64; ++t) {
-        const float qv = __shfl_sync(0xffffffffu, t < 32 ? q0 : q1, t & 31);
+    const int nrows = a.B * a.G;
+    for (int r = blockIdx.y * kRowsPerBlock + warp; r < min(nrows, (int)(blockIdx.y + 1) * kRowsPerBlock); r += 4) {
+        const int row = (r / a.G) * a.Hq + g * a.G + r % a.G;
+        const bf16 *qr = static_cast<const bf16 *>(a.q) + (size_t)row * 64;
+        const float q0 = __bfloat162float(qr[lane]), q1 = __bfloat162float(qr[lane + 32]);
+        float acc[DL / 32];
 #pragma unroll
         for (int e = 0; e < DL / 32; ++e)
-            s[e] = fmaf(qv, __ldg(ak + (size_t)t * DL + 32 * e), s[e]);
-    }
+            acc[e] = 0.f;
+#pragma unroll 8
+        for (int t = 0; t < 64; ++t) {
+            const float qv = __shfl_sync(0xffffffffu, t < 32 ? q0 : q1, t & 31);
 #pragma unroll
-    for (int e = 0; e < DL / 32; ++e)
-        a.qt[(size_t)row * DL + 32 * e + lane] = __float2bfloat16_rn(s[e]);
+            for (int e = 0; e < DL / 32; ++e)
+                acc[e] = fmaf(qv, aks[t * DL + 32 * e + lane], acc[e]);
+        }
+#pragma unroll
+        for (int e = 0; e < DL / 32; ++e)
+            a.qt[(size_t)row * DL + 32 * e + lane] = __float2bfloat16_rn(acc[e]);
+    }
 }
 
 // ---------------------------------------------------------------- decode: main
@@ -196,12 +224,13 @@ __device__ __forceinline__ uint32_t swz(uint32_t base, int row, int chunk)
 
 template <int DL, int MT>
 struct MainLayout {
+    static constexpr int NST = DL <= 192 ? 3 : 2;                  // page buffers (two CTAs per SM)
     static constexpr uint32_t QT = 0;                              // [DL/64][MT*16][128 B]
-    static constexpr uint32_t CB = (DL * MT * 16 * 2 + 1023) / 1024 * 1024;  // two page buffers
+    static constexpr uint32_t CB = (DL * MT * 16 * 2 + 1023) / 1024 * 1024;  // NST page buffers
     static constexpr uint32_t CSTAGE = DL / 64 * 8192;             // [DL/64][64][128 B]
-    static constexpr uint32_t P = CB + 2 * CSTAGE;                 // [MT*16][128 B]
+    static constexpr uint32_t P = CB + NST * CSTAGE;               // [MT*16][128 B]
     static constexpr uint32_t RED = P + MT * 16 * 128;             // [4][MT*16] floats
-    static constexpr uint32_t BAR = RED + 4 * MT * 16 * 4;
+    static constexpr uint32_t BAR = RED + 4 * MT * 16 * 4;        // NST full barriers, then the abort flag
     static constexpr uint32_t TOTAL = BAR + 64;
 };
 
@@ -215,7 +244,8 @@ __global__ void __launch_bounds__(kMainThreads) latent_main_kernel(const __grid_
                                                           ~uintptr_t(1023));
     const uint32_t sbase = smem_u32(sm);
     uint64_t *full = reinterpret_cast<uint64_t *>(sm + Ly::BAR);
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Ly::BAR + 16);
+    constexpr int NST = Ly::NST;
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Ly::BAR + 8 * NST);
     float *red = reinterpret_cast<float *>(sm + Ly::RED);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int b = blockIdx.y;
@@ -335,30 +365,28 @@ __global__ void __launch_bounds__(kMainThreads) latent_main_kernel(const __grid_
         return;  // the merge reads only the splits that hold tokens
     const int npg = (t1 - t0 + kTok - 1) / kTok;
     if (tid == 0) {
-        mbar_init(&full[0], 1);
-        mbar_init(&full[1], 1);
+        for (int st = 0; st < NST; ++st)
+            mbar_init(&full[st], 1);
         *abort_flag = 0;
         mbar_init_fence();
         prefetch_tensormap(&tmC);
     }
     __syncthreads();
-    auto issue = [&](int pi) {  // thread 0: page pi of the split into buffer pi % 2
+    auto issue = [&](int pi) {  // thread 0: page pi of the split into buffer pi % NST
         int pid = __ldg(a.block_table + (size_t)b * a.maxp + t0 / kTok + pi);
         if (pid < 0 || pid >= a.num_pages) {
             report(a.status, DAR_ERR_CAPACITY);
             pid = 0;
         }
-        uint64_t *bar = &full[pi & 1];
+        uint64_t *bar = &full[pi % NST];
         mbar_expect_tx(bar, kTok * DL * 2);
 #pragma unroll
         for (int cb = 0; cb < DL / 64; ++cb)
-            tma_load_2d(sm + Ly::CB + (pi & 1) * Ly::CSTAGE + cb * 8192, &tmC, cb * 64, pid * kTok, bar);
+            tma_load_2d(sm + Ly::CB + (pi % NST) * Ly::CSTAGE + cb * 8192, &tmC, cb * 64, pid * kTok, bar);
     };
-    if (tid == 0) {
-        issue(0);
-        if (npg > 1)
-            issue(1);
-    }
+    if (tid == 0)
+        for (int pi = 0; pi < NST && pi < npg; ++pi)
+            issue(pi);
     grid_dep_wait();  // q~ comes from the prep kernel
     // q~ rows (zero past Hq) into the swizzled operand tile
     for (int i = tid; i < MT * 16 * (DL / 8); i += kMainThreads) {
@@ -385,8 +413,8 @@ __global__ void __launch_bounds__(kMainThreads) latent_main_kernel(const __grid_
     bool ok = true;
 
     for (int pi = 0; pi < npg; ++pi) {
-        const int s = pi & 1;
-        if (!mbar_wait(&full[s], (pi >> 1) & 1, abort_flag))
+        const int s = pi % NST;
+        if (!mbar_wait(&full[s], (pi / NST) & 1, abort_flag))
             ok = false;
         if (__syncthreads_or(!ok)) {
             ok = false;
@@ -504,16 +532,16 @@ __global__ void __launch_bounds__(kMainThreads) latent_main_kernel(const __grid_
             }
         }
         __syncthreads();  // buffer s and P are free again
-        if (tid == 0 && pi + 2 < npg) {
+        if (tid == 0 && pi + NST < npg) {
             fence_proxy_async_smem();
-            issue(pi + 2);
+            issue(pi + NST);
         }
     }
     if (!ok) {
         // let copies still in flight land before the CTA exits
         if (tid == 0) {
-            for (int pi = 0; pi < npg && pi < 2; ++pi)
-                mbar_wait(&full[pi & 1], 0, nullptr);
+            for (int st = 0; st < NST && st < npg; ++st)
+                mbar_wait(&full[st], 0, nullptr);
             report(a.status, DAR_ERR_DEVICE);
         }
         return;
@@ -560,83 +588,88 @@ __global__ void __launch_bounds__(kMainThreads) latent_main_kernel(const __grid_
 
 // ---------------------------------------------------------------- decode: merge
 
-// One warp per (b, h): combine the window record and the sequence's latent
-// splits (log-sum-exp), lift the latent sum with A_V, divide.
+// Block (g, 4 rows of KV head g): A_V^g staged in shared memory by one bulk
+// copy (before the dependency wait: it does not come from the main kernel),
+// then one warp per row: combine the window record and the sequence's latent splits
+// (log-sum-exp, one split per lane), lift the latent sum with A_V, divide.
 template <int DL>
 __global__ void __launch_bounds__(128) latent_merge_kernel(Args a)
 {
-    __shared__ float olat[4][DL];
-    __shared__ float fs[4][32];
-    grid_dep_wait();  // the main kernel's records
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int row = blockIdx.x * 4 + warp;
-    const bool active = row < a.B * a.Hq;
-    const int b = active ? row / a.Hq : 0, h = active ? row % a.Hq : 0, g = h / a.G;
-    int L = active ? __ldg(a.seq_lens + b) : 0;
-    if (L < 0 || L > a.maxp * kTok)
-        L = 0;  // reported by the main kernel; the output is undefined then
-    const int Lg = L > a.w ? L - a.w : 0;
-    const int ns = (Lg + kSplitTok - 1) / kSplitTok;
-    const float *rw = a.rec_win + (size_t)row * 66;
-    const float *rl0 = a.rec_lat + ((size_t)b * a.nspl * a.Hq + h) * (DL + 2);  // split s at + s * Hq * (DL + 2)
-    const size_t sstride = (size_t)a.Hq * (DL + 2);
-    const float mw = L > 0 ? rw[64] : -INFINITY;
-    // the splits' maxima and sums, one split per lane (32 at a time)
-    float M = mw;
-    for (int s = lane; s < ns; s += 32)
-        M = fmaxf(M, rl0[s * sstride + DL]);
-#pragma unroll
-    for (int o = 16; o; o >>= 1)
-        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    float l = 0.f;
-    float acc[DL / 32];
-#pragma unroll
-    for (int e = 0; e < DL / 32; ++e)
-        acc[e] = 0.f;
-    for (int s0 = 0; s0 < ns; s0 += 32) {
-        float f = 0.f;
-        if (s0 + lane < ns) {
-            const float *rl = rl0 + (s0 + lane) * sstride;
-            f = ex2_approx(rl[DL] - M);
-            l += f * rl[DL + 1];
-        }
-        fs[warp][lane] = f;
-        __syncwarp();
-        const int n = min(32, ns - s0);
-#pragma unroll 4
-        for (int j = 0; j < n; ++j) {
-            const float *rl = rl0 + (s0 + j) * sstride;
-            const float fj = fs[warp][j];
-#pragma unroll
-            for (int e = 0; e < DL / 32; ++e)
-                acc[e] = fmaf(fj, rl[lane + 32 * e], acc[e]);
-        }
-        __syncwarp();
-    }
-#pragma unroll
-    for (int o = 16; o; o >>= 1)
-        l += __shfl_xor_sync(0xffffffffu, l, o);
-    const float fw = L > 0 ? ex2_approx(mw - M) : 0.f;
-    if (L > 0)
-        l += fw * rw[65];
-#pragma unroll
-    for (int e = 0; e < DL / 32; ++e)
-        olat[warp][lane + 32 * e] = acc[e];
-    __syncwarp();
-    if (!active)
+    extern __shared__ __align__(16) float msm[];
+    float *avs = msm;                  // [DL][64]
+    float *olat = avs + DL * 64;       // [4 warps][DL]
+    float *fs = olat + 4 * DL;         // [4 warps][32]
+    uint64_t *bar = reinterpret_cast<uint64_t *>(fs + 4 * 32);
+    const int g = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (!stage_matrix(avs, a.Av + (size_t)g * DL * 64, DL * 64 * 4, bar, a.status))
         return;
-    float o0 = L > 0 ? fw * rw[lane] : 0.f, o1 = L > 0 ? fw * rw[lane + 32] : 0.f;
-    const float *av = a.Av + (size_t)g * DL * 64;
+    grid_dep_wait();  // the main kernel's records
+    const int nrows = a.B * a.G;
+    const size_t sstride = (size_t)a.Hq * (DL + 2);
+    for (int r = blockIdx.y * kRowsPerBlock + warp; r < min(nrows, (int)(blockIdx.y + 1) * kRowsPerBlock); r += 4) {
+        const int b = r / a.G, h = g * a.G + r % a.G, row = b * a.Hq + h;
+        int L = __ldg(a.seq_lens + b);
+        if (L < 0 || L > a.maxp * kTok)
+            L = 0;  // reported by the main kernel; the output is undefined then
+        const int Lg = L > a.w ? L - a.w : 0;
+        const int ns = (Lg + kSplitTok - 1) / kSplitTok;
+        const float *rw = a.rec_win + (size_t)row * 66;
+        const float *rl0 = a.rec_lat + ((size_t)b * a.nspl * a.Hq + h) * (DL + 2);
+        const float mw = L > 0 ? rw[64] : -INFINITY;
+        float M = mw;
+        for (int s2 = lane; s2 < ns; s2 += 32)
+            M = fmaxf(M, rl0[s2 * sstride + DL]);
+#pragma unroll
+        for (int o = 16; o; o >>= 1)
+            M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+        float l = 0.f;
+        float acc[DL / 32];
+#pragma unroll
+        for (int e = 0; e < DL / 32; ++e)
+            acc[e] = 0.f;
+        for (int s0 = 0; s0 < ns; s0 += 32) {
+            float f = 0.f;
+            if (s0 + lane < ns) {
+                const float *rl = rl0 + (s0 + lane) * sstride;
+                f = ex2_approx(rl[DL] - M);
+                l += f * rl[DL + 1];
+            }
+            fs[warp * 32 + lane] = f;
+            __syncwarp();
+            const int n = min(32, ns - s0);
+#pragma unroll 4
+            for (int j = 0; j < n; ++j) {
+                const float *rl = rl0 + (s0 + j) * sstride;
+                const float fj = fs[warp * 32 + j];
+#pragma unroll
+                for (int e = 0; e < DL / 32; ++e)
+                    acc[e] = fmaf(fj, rl[lane + 32 * e], acc[e]);
+            }
+            __syncwarp();
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1)
+            l += __shfl_xor_sync(0xffffffffu, l, o);
+        const float fw = L > 0 ? ex2_approx(mw - M) : 0.f;
+        if (L > 0)
+            l += fw * rw[65];
+#pragma unroll
+        for (int e = 0; e < DL / 32; ++e)
+            olat[warp * DL + lane + 32 * e] = acc[e];
+        __syncwarp();
+        float o0 = L > 0 ? fw * rw[lane] : 0.f, o1 = L > 0 ? fw * rw[lane + 32] : 0.f;
 #pragma unroll 16
-    for (int c = 0; c < DL; ++c) {
-        const float x = olat[warp][c];
-        o0 = fmaf(x, __ldg(av + c * 64 + lane), o0);
-        o1 = fmaf(x, __ldg(av + c * 64 + lane + 32), o1);
+        for (int c = 0; c < DL; ++c) {
+            const float x = olat[warp * DL + c];
+            o0 = fmaf(x, avs[c * 64 + lane], o0);
+            o1 = fmaf(x, avs[c * 64 + lane + 32], o1);
+        }
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        bf16 *out = static_cast<bf16 *>(a.out) + (size_t)row * 64;
+        out[lane] = __float2bfloat16_rn(o0 * inv);
+        out[lane + 32] = __float2bfloat16_rn(o1 * inv);
+        __syncwarp();
     }
-    const float inv = l > 0.f ? 1.f / l : 0.f;
-    bf16 *out = static_cast<bf16 *>(a.out) + (size_t)row * 64;
-    out[lane] = __float2bfloat16_rn(o0 * inv);
-    out[lane + 32] = __float2bfloat16_rn(o1 * inv);
 }
 
 // ---------------------------------------------------------------- host side
@@ -666,10 +699,19 @@ static cudaError_t decode_t(const Args &a, const void *pool_c, cudaStream_t s)
     using Ly = MainLayout<DL, MT>;
     constexpr size_t win_smem = (2 * kWinChunk * kWinLd + 4 * kWinChunk + 4 * 64) * sizeof(float);
     const size_t smem = 1024 + (Ly::TOTAL > win_smem ? Ly::TOTAL : win_smem);
+    constexpr size_t prep_smem = (size_t)64 * DL * sizeof(float) + 16;
+    constexpr size_t merge_smem = ((size_t)DL * 64 + 4 * DL + 4 * 32) * sizeof(float) + 16;
     static PerDeviceOnce once;
     cudaError_t e = per_device_once(once, [&](int) {
-        return cudaFuncSetAttribute(latent_main_kernel<DL, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)smem);
+        cudaError_t e2 = cudaFuncSetAttribute(latent_main_kernel<DL, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)smem);
+        if (e2 == cudaSuccess)
+            e2 = cudaFuncSetAttribute(latent_prep_kernel<DL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)prep_smem);
+        if (e2 == cudaSuccess)
+            e2 = cudaFuncSetAttribute(latent_merge_kernel<DL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)merge_smem);
+        return e2;
     });
     if (e != cudaSuccess)
         return e;
@@ -685,10 +727,10 @@ static cudaError_t decode_t(const Args &a, const void *pool_c, cudaStream_t s)
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return cudaErrorInvalidValue;
-    const int rows = a.B * a.Hq;
     // prep starts after all earlier work on the stream; main and merge are
     // launched programmatically (each waits in-kernel for what it reads)
-    latent_prep_kernel<DL><<<(rows + 7) / 8, 256, 0, s>>>(a);
+    const dim3 rgrid(a.Hkv, (a.B * a.G + kRowsPerBlock - 1) / kRowsPerBlock);
+    latent_prep_kernel<DL><<<rgrid, 128, prep_smem, s>>>(a);
     cudaLaunchAttribute pdl[1];
     pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     pdl[0].val.programmaticStreamSerializationAllowed = 1;
@@ -702,9 +744,9 @@ static cudaError_t decode_t(const Args &a, const void *pool_c, cudaStream_t s)
     e = cudaLaunchKernelEx(&cfg, latent_main_kernel<DL, MT>, tm, a);
     if (e != cudaSuccess)
         return e;
-    cfg.gridDim = dim3((rows + 3) / 4);
+    cfg.gridDim = rgrid;
     cfg.blockDim = dim3(128);
-    cfg.dynamicSmemBytes = 0;
+    cfg.dynamicSmemBytes = merge_smem;
     e = cudaLaunchKernelEx(&cfg, latent_merge_kernel<DL>, a);
     if (e != cudaSuccess)
         return e;
