@@ -1,7 +1,7 @@
 // dar_backward.cu -- host side of the gradients of the causal DAR attention
 // forward (Sec. 2.3 training): workspace layout and the launch sequence of
 // the kernels in dar_backward.cuh (compiled per storage type in
-// dar_backward_f32.cu and dar_backward_bf16.cu).
+// dar_backward_f32.cu and, with the tensor-core kernels, dar_backward_tc.cu).
 #include "dar_backward.cuh"
 
 namespace dar {
@@ -11,7 +11,7 @@ size_t backward_workspace_bytes(dar_dtype dt, int B, int Hq, int Hkv, int N, int
     const size_t es = dt == DAR_F32 ? 4 : 2;
     const size_t qrows = (size_t)B * Hq * N, krows = (size_t)B * Hkv * N;
     return 2 * al(krows * dd * es) + 4 * al(qrows * dd * 4) + 2 * al(qrows * 4) + 2 * al(krows * dd * 4) +
-           al((size_t)bwd::kChunks * 4 * Hkv * 64 * dd * 4);
+           al((size_t)bwd::kChunks * 4 * Hkv * 64 * dd * 4) + (dt == DAR_BF16 ? 2 * al(qrows * dd * 2) : 0);
 }
 
 cudaError_t launch_backward(dar_dtype dt, const BackwardArgs &x, void *workspace, cudaStream_t s)
@@ -56,6 +56,11 @@ cudaError_t launch_backward(dar_dtype dt, const BackwardArgs &x, void *workspace
     a.dkd = reinterpret_cast<float *>(take(krows * x.dd * 4));
     a.dvd = reinterpret_cast<float *>(take(krows * x.dd * 4));
     a.part = reinterpret_cast<float *>(take((size_t)bwd::kChunks * 4 * x.Hkv * 64 * x.dd * 4));
+    a.qtb = a.dotb = nullptr;
+    if (dt == DAR_BF16) {  // bf16 copies of q~ and dO~ for the tensor-core kernels
+        a.qtb = reinterpret_cast<bf16 *>(take(qrows * x.dd * 2));
+        a.dotb = reinterpret_cast<bf16 *>(take(qrows * x.dd * 2));
+    }
     a.B = x.B;
     a.Hq = x.Hq;
     a.Hkv = x.Hkv;

@@ -19,7 +19,8 @@
 //   dUv = sum_i O^D_i^T dO_i (O^D_i = sum_global p_ij v^D_j).
 //
 // Kernels (fp32 arithmetic on the CUDA cores, both storage types):
-//  1. bwd_rows: per row, q~, dO~ and D (one warp per row).
+//  1. bwd_rows: per row, q~, dO~ and D (one warp per row, Uk and Uv staged
+//     in shared memory per KV head).
 //  2. bwd_dq: per 64-row query tile, the row log-sum-exp (first pass over the
 //     keys) and then dq, dq~ and O^D (second pass).
 //  3. bwd_dkv: per 64-key tile of a KV head, over the query heads of the
@@ -49,6 +50,7 @@ struct Args {
     float *drow, *lse;                   // [B][Hq][N]: D, log2-sum-exp2 of the scaled scores
     float *dqt, *od;                     // [B][Hq][N][DD]: dq~ (scaled), O^D
     float *dkd, *dvd;                    // [B][Hkv][N][DD]: dk^D (scaled), dv^D
+    bf16 *qtb, *dotb;                    // [B][Hq][N][DD]: q~, dO~ rounded to bf16 (tensor-core operands)
     float *part;                         // [kChunks][4][Hkv][64 * DD]
     int B, Hq, Hkv, G, N, w;
     float scale, c2;                     // scale, scale * log2(e)
@@ -56,13 +58,27 @@ struct Args {
 
 // ---------------------------------------------------------------- 1. rows
 
+// Block (g, row range): Uk^g and Uv^g staged transposed ([t][c]) in shared
+// memory; one warp per row of KV head g's query heads: D = dO . o by a warp
+// reduction, q~ = q Uk^T and dO~ = dO Uv^T with lanes over c (the row's q and
+// dO broadcast from shared memory).
 template <typename T, int DD>
 __global__ void __launch_bounds__(256) bwd_rows_kernel(Args a)
 {
-    const int lane = threadIdx.x & 31;
-    const long rows = (long)a.B * a.Hq * a.N;
-    for (long row = (long)blockIdx.x * 8 + (threadIdx.x >> 5); row < rows; row += (long)gridDim.x * 8) {
-        const int g = (int)((row / a.N) % a.Hq) / a.G;
+    __shared__ float ukt[64 * DD], uvt[64 * DD];
+    __shared__ float xs[8][2][64];
+    const int g = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < DD * 64; i += blockDim.x) {
+        const int c = i / 64, t = i % 64;
+        ukt[t * DD + c] = a.Uk[((size_t)g * DD + c) * kHeadDim + t];
+        uvt[t * DD + c] = a.Uv[((size_t)g * DD + c) * kHeadDim + t];
+    }
+    __syncthreads();
+    const long nrows = (long)a.B * a.G * a.N;  // rows of KV head g's query heads
+    for (long r = (long)blockIdx.y * 8 + warp; r < nrows; r += (long)gridDim.y * 8) {
+        const long bq = r / a.N;
+        const int i = (int)(r % a.N), b = (int)(bq / a.G), hh = (int)(bq % a.G);
+        const long row = ((long)b * a.Hq + g * a.G + hh) * a.N + i;
         const T *qr = static_cast<const T *>(a.q) + row * kHeadDim;
         const T *dr = static_cast<const T *>(a.dout) + row * kHeadDim;
         const T *orow = static_cast<const T *>(a.out) + row * kHeadDim;
@@ -74,23 +90,35 @@ __global__ void __launch_bounds__(256) bwd_rows_kernel(Args a)
             D += __shfl_xor_sync(0xffffffffu, D, o);
         if (lane == 0)
             a.drow[row] = D;
-        for (int c0 = 0; c0 < DD; c0 += 32) {
-            const int c = c0 + lane;
-            const float *uk = a.Uk + ((size_t)g * DD + (c < DD ? c : 0)) * kHeadDim;
-            const float *uv = a.Uv + ((size_t)g * DD + (c < DD ? c : 0)) * kHeadDim;
+        xs[warp][0][lane] = q0;
+        xs[warp][0][lane + 32] = q1;
+        xs[warp][1][lane] = d0;
+        xs[warp][1][lane + 32] = d1;
+        __syncwarp();
+        for (int c = lane; c < DD; c += 32) {
             float sq = 0.f, sd = 0.f;
+#pragma unroll 16
             for (int t = 0; t < kHeadDim; ++t) {
-                const float qv = __shfl_sync(0xffffffffu, t < 32 ? q0 : q1, t & 31);
-                const float dv = __shfl_sync(0xffffffffu, t < 32 ? d0 : d1, t & 31);
-                sq = fmaf(qv, uk[t], sq);
-                sd = fmaf(dv, uv[t], sd);
+                sq = fmaf(xs[warp][0][t], ukt[t * DD + c], sq);
+                sd = fmaf(xs[warp][1][t], uvt[t * DD + c], sd);
             }
-            if (c < DD) {
-                a.qt[row * DD + c] = sq;
-                a.dot[row * DD + c] = sd;
+            a.qt[row * DD + c] = sq;
+            a.dot[row * DD + c] = sd;
+            if (a.qtb) {
+                a.qtb[row * DD + c] = __float2bfloat16_rn(sq);
+                a.dotb[row * DD + c] = __float2bfloat16_rn(sd);
             }
         }
+        __syncwarp();
     }
+}
+
+// Grid of the row kernel: one column of blocks per KV head.
+inline dim3 rows_grid(const Args &a)
+{
+    const long per_g = (long)a.B * a.G * a.N;
+    const long by = (per_g + 7) / 8, cap = 2432 / a.Hkv > 0 ? 2432 / a.Hkv : 1;
+    return dim3(a.Hkv, (unsigned)(by < cap ? by : cap));
 }
 
 // Shared helpers for the two attention kernels.
@@ -543,6 +571,15 @@ __global__ void __launch_bounds__(kThreads) bwd_wsum_kernel(Args a)
 
 // ---------------------------------------------------------------- host side
 
+// The projection gradients from the per-row and per-key intermediates.
+template <typename T, int DD>
+inline cudaError_t run_weights(const Args &a, cudaStream_t s)
+{
+    bwd_wpart_kernel<T, DD><<<dim3(kChunks, a.Hkv, 4), kThreads, 0, s>>>(a);
+    bwd_wsum_kernel<DD><<<(4 * a.Hkv * 64 * DD + kThreads - 1) / kThreads, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
 template <typename T, int DD>
 inline cudaError_t run(const Args &a, cudaStream_t s)
 {
@@ -557,14 +594,11 @@ inline cudaError_t run(const Args &a, cudaStream_t s)
     });
     if (e != cudaSuccess)
         return e;
-    const long rows = (long)a.B * a.Hq * a.N;
-    bwd_rows_kernel<T, DD><<<(unsigned)min((rows + 7) / 8, 152L * 16), 256, 0, s>>>(a);
+    bwd_rows_kernel<T, DD><<<rows_grid(a), 256, 0, s>>>(a);
     const int tiles = (a.N + kRows - 1) / kRows;
     bwd_dq_kernel<T, DD><<<dim3(tiles, a.B * a.Hq), kThreads, smq, s>>>(a);
     bwd_dkv_kernel<T, DD><<<dim3(tiles, a.B * a.Hkv), kThreads, smk, s>>>(a);
-    bwd_wpart_kernel<T, DD><<<dim3(kChunks, a.Hkv, 4), kThreads, 0, s>>>(a);
-    bwd_wsum_kernel<DD><<<(4 * a.Hkv * 64 * DD + kThreads - 1) / kThreads, kThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    return run_weights<T, DD>(a, s);
 }
 
 template <typename T>
