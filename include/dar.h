@@ -297,8 +297,10 @@ dar_status dar_attn_decode_direct(const dar_cache *cache, int32_t Hq, const void
  * each overwritten (not accumulated).  The derivative is that of Eq. 1-4 with
  * the stored k^D, v^D's rounding to T not differentiated (the bottleneck
  * projections get the gradient of the unrounded product), and D_i = dout_i .
- * out_i taken from the given forward output.  fp32 arithmetic on the CUDA
- * cores for both storage types; no tensor cores.  The workspace
+ * out_i taken from the given forward output.  bf16 storage runs the score,
+ * dP and gradient contractions on the tensor cores (bf16 operands, P and dS
+ * rounded to bf16, fp32 accumulation; d_down = 8 stays on the CUDA cores);
+ * fp32 storage runs fp32 arithmetic on the CUDA cores.  The workspace
  * (dar_attn_backward_workspace_bytes, no initialisation) holds per-row and
  * per-token intermediates; outputs must not overlap inputs.  Deterministic:
  * every sum runs in a fixed order.  Shapes as dar_attn_prefill; B*Hq <= 65535.

@@ -255,26 +255,60 @@ __global__ void __launch_bounds__(kTc) bwd_dq_tc_kernel(Args a)
                     mma_bf16_16816(sg[1], qta[kk], bfr[2], bfr[3]);
                 }
             }
+            if (interior) {  // every pair of the step is valid and global: no masks, no local part
+                if (pass == 0) {
+#pragma unroll
+                    for (int r = 0; r < 2; ++r) {
+                        const float x0 = sg[0][2 * r] * a.c2, x1 = sg[0][2 * r + 1] * a.c2;
+                        const float x2 = sg[1][2 * r] * a.c2, x3 = sg[1][2 * r + 1] * a.c2;
+                        const float mn = fmaxf(m[r], fmaxf(fmaxf(x0, x1), fmaxf(x2, x3)));
+                        l[r] = l[r] * sm100::ex2_approx(m[r] - mn) + (sm100::ex2_approx(x0 - mn) + sm100::ex2_approx(x1 - mn)) +
+                               (sm100::ex2_approx(x2 - mn) + sm100::ex2_approx(x3 - mn));
+                        m[r] = mn;
+                    }
+                    continue;
+                }
+                float dpg[2][4] = {};
+#pragma unroll
+                for (int kk = 0; kk < KSD; ++kk) {
+                    uint32_t bfr[4];
+                    ldsm_x4(b_addr<LD>(stg + Ly::VD_OFF, 16 * kc, kk, lane), bfr);
+                    mma_bf16_16816(dpg[0], dota[kk], bfr[0], bfr[1]);
+                    mma_bf16_16816(dpg[1], dota[kk], bfr[2], bfr[3]);
+                }
+                float pg[2][4], dsg[2][4];
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        pg[nt][e] = sm100::ex2_approx(fmaf(sg[nt][e], a.c2, -lse[e >> 1]));
+                        dsg[nt][e] = pg[nt][e] * (dpg[nt][e] - Dr[e >> 1]);
+                    }
+                uint32_t ag[4], ap[4];
+                frag_a(ag, dsg[0], dsg[1]);
+                frag_a(ap, pg[0], pg[1]);
+#pragma unroll
+                for (int n0 = 0; n0 < DD; n0 += 16) {
+                    uint32_t bfr[4];
+                    ldsm_x4_t(bt_addr<LD>(stg + Ly::KD_OFF, 16 * kc, n0, lane), bfr);
+                    mma_bf16_16816(dqt[n0 / 8], ag, bfr[0], bfr[1]);
+                    mma_bf16_16816(dqt[n0 / 8 + 1], ag, bfr[2], bfr[3]);
+                    ldsm_x4_t(bt_addr<LD>(stg + Ly::VD_OFF, 16 * kc, n0, lane), bfr);
+                    mma_bf16_16816(od[n0 / 8], ap, bfr[0], bfr[1]);
+                    mma_bf16_16816(od[n0 / 8 + 1], ap, bfr[2], bfr[3]);
+                }
+                continue;
+            }
             float x[2][4];
             bool loc[2][4];
-            if (interior) {  // every pair of the tile is valid and global: no masks
 #pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
+            for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        loc[nt][e] = false;
-                        x[nt][e] = sg[nt][e] * a.c2;
-                    }
-            } else {
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int i = ir0 + 8 * (e >> 1), j = j0 + 16 * kc + 8 * nt + 2 * tig + (e & 1);
-                        loc[nt][e] = i - j < w;
-                        x[nt][e] = (i < N && j <= i) ? (loc[nt][e] ? sl[nt][e] : sg[nt][e]) * a.c2 : -INFINITY;
-                    }
-            }
+                for (int e = 0; e < 4; ++e) {
+                    const int i = ir0 + 8 * (e >> 1), j = j0 + 16 * kc + 8 * nt + 2 * tig + (e & 1);
+                    loc[nt][e] = i - j < w;
+                    x[nt][e] = (i < N && j <= i) ? (loc[nt][e] ? sl[nt][e] : sg[nt][e]) * a.c2 : -INFINITY;
+                }
             if (pass == 0) {
 #pragma unroll
                 for (int r = 0; r < 2; ++r) {
@@ -514,6 +548,39 @@ __global__ void __launch_bounds__(kTc) bwd_dkv_tc_kernel(Args a)
                     mma_bf16_16816(sg[1], kda[kk], bfr[2], bfr[3]);
                 }
             }
+            if (interior) {  // every pair of the step is valid and global: no masks, no local part
+                float dpg[2][4] = {};
+#pragma unroll
+                for (int kk = 0; kk < KSD; ++kk) {
+                    uint32_t bfr[4];
+                    ldsm_x4(b_addr<LD>(stg + Ly::DOT_OFF, 16 * qc, kk, lane), bfr);
+                    mma_bf16_16816(dpg[0], vda[kk], bfr[0], bfr[1]);
+                    mma_bf16_16816(dpg[1], vda[kk], bfr[2], bfr[3]);
+                }
+                float pg[2][4], dsg[2][4];
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int il = 16 * qc + 8 * nt + 2 * tig + (e & 1);
+                        pg[nt][e] = sm100::ex2_approx(fmaf(sg[nt][e], a.c2, -lse_s[il]));
+                        dsg[nt][e] = pg[nt][e] * (dpg[nt][e] - dr_s[il]);
+                    }
+                uint32_t ap[4], ad[4];
+                frag_a(ap, pg[0], pg[1]);
+                frag_a(ad, dsg[0], dsg[1]);
+#pragma unroll
+                for (int n0 = 0; n0 < DD; n0 += 16) {
+                    uint32_t bfr[4];
+                    ldsm_x4_t(bt_addr<LD>(stg + Ly::DOT_OFF, 16 * qc, n0, lane), bfr);
+                    mma_bf16_16816(dvd[n0 / 8], ap, bfr[0], bfr[1]);
+                    mma_bf16_16816(dvd[n0 / 8 + 1], ap, bfr[2], bfr[3]);
+                    ldsm_x4_t(bt_addr<LD>(stg + Ly::QT_OFF, 16 * qc, n0, lane), bfr);
+                    mma_bf16_16816(dkd[n0 / 8], ad, bfr[0], bfr[1]);
+                    mma_bf16_16816(dkd[n0 / 8 + 1], ad, bfr[2], bfr[3]);
+                }
+                continue;
+            }
             float dpl[2][4] = {}, dpg[2][4] = {};
             if (!all_global) {
 #pragma unroll
@@ -534,35 +601,22 @@ __global__ void __launch_bounds__(kTc) bwd_dkv_tc_kernel(Args a)
                 }
             }
             float pl[2][4], dsl[2][4], pg[2][4], dsg[2][4];
-            if (interior) {  // every pair of the tile is valid and global: no masks
 #pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
+            for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int il = 16 * qc + 8 * nt + 2 * tig + (e & 1);
-                        const float p = sm100::ex2_approx(fmaf(sg[nt][e], a.c2, -lse_s[il]));
-                        pg[nt][e] = p;
-                        dsg[nt][e] = p * (dpg[nt][e] - dr_s[il]);
-                        pl[nt][e] = dsl[nt][e] = 0.f;
+                for (int e = 0; e < 4; ++e) {
+                    const int j = jr0 + 8 * (e >> 1), il = 16 * qc + 8 * nt + 2 * tig + (e & 1), i = i0 + il;
+                    const bool loc = i - j < w;
+                    float p = 0.f, ds = 0.f;
+                    if (j < N && i < N && j <= i) {
+                        p = sm100::ex2_approx((loc ? sl[nt][e] : sg[nt][e]) * a.c2 - lse_s[il]);
+                        ds = p * ((loc ? dpl[nt][e] : dpg[nt][e]) - dr_s[il]);
                     }
-            } else {
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int j = jr0 + 8 * (e >> 1), il = 16 * qc + 8 * nt + 2 * tig + (e & 1), i = i0 + il;
-                        const bool loc = i - j < w;
-                        float p = 0.f, ds = 0.f;
-                        if (j < N && i < N && j <= i) {
-                            p = sm100::ex2_approx((loc ? sl[nt][e] : sg[nt][e]) * a.c2 - lse_s[il]);
-                            ds = p * ((loc ? dpl[nt][e] : dpg[nt][e]) - dr_s[il]);
-                        }
-                        pl[nt][e] = loc ? p : 0.f;
-                        dsl[nt][e] = loc ? ds : 0.f;
-                        pg[nt][e] = loc ? 0.f : p;
-                        dsg[nt][e] = loc ? 0.f : ds;
-                    }
-            }
+                    pl[nt][e] = loc ? p : 0.f;
+                    dsl[nt][e] = loc ? ds : 0.f;
+                    pg[nt][e] = loc ? 0.f : p;
+                    dsg[nt][e] = loc ? 0.f : ds;
+                }
             if (!all_global) {
                 uint32_t ap[4], ad[4];
                 frag_a(ap, pl[0], pl[1]);
