@@ -372,7 +372,7 @@ dar_status dar_latent_absorb(int32_t Hkv, int32_t D, int32_t d, int32_t d_lat, c
  * order on `stream` (q~ = q A_K^T; split-K over pages of the latent pool and
  * the window; merge and lift).  Workspace of
  * dar_latent_decode_workspace_bytes(cache, Hq) bytes, no initialisation.
- * L_b == 0 gives a zero output. */
+ * L_b == 0 gives a zero output.  B <= DAR_DECODE_MAX_BATCH. */
 size_t dar_latent_decode_workspace_bytes(const dar_latent_cache *cache, int32_t Hq);
 dar_status dar_latent_decode(const dar_latent_cache *cache, int32_t Hq, const void *q, const float *A_K,
                              const float *A_V, float scale, void *out, void *workspace,

@@ -613,6 +613,8 @@ dar_status dar_latent_decode(const dar_latent_cache *cache, int32_t Hq, const vo
         return fail(DAR_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", Hq, cache->Hkv);
     if (Hq > 32)
         return fail(DAR_ERR_UNSUPPORTED, "Hq=%d > 32", Hq);
+    if (cache->B > DAR_DECODE_MAX_BATCH)
+        return fail(DAR_ERR_UNSUPPORTED, "latent decode batch %d > %d", cache->B, DAR_DECODE_MAX_BATCH);
     if (cache->B == 0)
         return ok();
     if (!q || !A_K || !A_V || !out || !workspace)

@@ -15,11 +15,13 @@
 //    inputs per element, rounded once to bf16) into the page of every new
 //    token; new keys/values into the ring; then the lengths.
 //  - latent_absorb: A_K, A_V (fp32 chains over D).
-//  - decode: prep (q~ = q A_K^T, bf16), main (latent splits of eight pages
-//    each: TMA-staged pages in a ring of two or three buffers, S = Q~ C^T and O += P C on mma.sync tensor
-//    cores, one online softmax per head; plus one CTA per KV head for the
-//    window on the CUDA cores), merge (exact log-sum-exp combination of the
-//    partial results, then o = (O_loc + O_lat A_V) / l).
+//  - decode: prep (q~ = q A_K^T, bf16), main (a persistent kernel: work
+//    items are latent splits of four pages and windows of one KV head; a
+//    producer warp streams their 64-token tiles through a TMA ring, four
+//    consumer warps compute S = A B^T and O += P V on mma.sync tensor cores
+//    with one online softmax per head and write one partial record per item),
+//    merge (exact log-sum-exp combination of the partial records, then
+//    o = (O_loc + O_lat A_V) / l).
 #include <cuda.h>
 
 #include <mutex>
@@ -34,11 +36,8 @@ namespace lat {
 using namespace sm100;
 
 constexpr int kTok = DAR_PAGE_SIZE;  // tokens per page
-constexpr int kPagesPerSplit = 8;
+constexpr int kPagesPerSplit = 4;
 constexpr int kSplitTok = kTok * kPagesPerSplit;
-constexpr int kMainThreads = 128;
-constexpr int kWinChunk = 64;  // window tokens staged at a time
-constexpr int kWinLd = 65;
 
 struct Args {
     const void *q;  // [B][Hq][64]
@@ -215,375 +214,454 @@ __global__ void __launch_bounds__(128) latent_prep_kernel(Args a)
 // ---------------------------------------------------------------- decode: main
 
 // Shared-memory tiles are rows of 128 bytes (64 bf16) with the 16-byte chunk
-// index XOR (row % 8), the layout the 128-byte TMA swizzle writes; a d_lat-wide
-// row is DL / 64 such blocks of rows.
+// index XOR (row % 8), the layout the 128-byte TMA swizzle writes; a W-wide
+// row is W / 64 such blocks of rows.
 __device__ __forceinline__ uint32_t swz(uint32_t base, int row, int chunk)
 {
     return base + (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
+constexpr int kConsumerThreads = 128;                   // warps 0-3: tensor-core work
+constexpr int kMainThreads2 = kConsumerThreads + 32;    // warp 4: TMA producer
+
+// Persistent main kernel.  Work items, enumerated the same way by every
+// thread: first the latent splits (sequence b, up to four 64-token pages of
+// its distant part), then the windows (sequence b, KV head g: the last
+// min(L_b, w) tokens' full keys and values, in 64-token tiles).  CTA c takes
+// items c, c + gridDim.x, ...  Warp 4 streams the items' pages and tiles
+// through a ring of NST stages with TMA; warps 0-3 run each stage on the
+// tensor cores and release it.
 template <int DL, int MT>
 struct MainLayout {
-    static constexpr int NST = DL <= 192 ? 3 : 2;                  // page buffers (two CTAs per SM)
-    static constexpr uint32_t QT = 0;                              // [DL/64][MT*16][128 B]
-    static constexpr uint32_t CB = (DL * MT * 16 * 2 + 1023) / 1024 * 1024;  // NST page buffers
-    static constexpr uint32_t CSTAGE = DL / 64 * 8192;             // [DL/64][64][128 B]
-    static constexpr uint32_t P = CB + NST * CSTAGE;               // [MT*16][128 B]
-    static constexpr uint32_t RED = P + MT * 16 * 128;             // [4][MT*16] floats
-    static constexpr uint32_t BAR = RED + 4 * MT * 16 * 4;        // NST full barriers, then the abort flag
-    static constexpr uint32_t TOTAL = BAR + 64;
+    static constexpr uint32_t CST = DL >= 128 ? DL / 64 * 8192 : 16384;  // a latent page, or a window K + V tile
+    static constexpr int NST = DL <= 128 ? 6 : DL == 192 ? 4 : 2;
+    static constexpr uint32_t QA = 0;                                     // [DL/64][MT*16][128 B] A operand
+    static constexpr uint32_t STG = (DL / 64 * MT * 16 * 128 + 1023) / 1024 * 1024;
+    static constexpr uint32_t P = STG + NST * CST;                        // [MT*16][128 B]
+    static constexpr uint32_t RED = P + MT * 16 * 128;                    // [4][MT*16] floats
+    static constexpr uint32_t PREF = RED + 4 * MT * 16 * 4;               // [B + 1] ints (B <= 1024)
+    static constexpr uint32_t BAR = PREF + (DAR_DECODE_MAX_BATCH + 1) * 4 + 4;
+    static constexpr uint32_t TOTAL = (BAR + 16 * NST + 16 + 15) / 16 * 16;
 };
 
+struct Item {
+    bool latent;
+    int b, part;  // latent: split index; window: KV head
+    int npg;      // pages / tiles
+};
+
+template <int MT>
+__device__ __forceinline__ void consumer_sync()
+{
+    asm volatile("bar.sync 1, %0;" ::"n"(kConsumerThreads) : "memory");
+}
+
+// One stage on the tensor cores: S = A B^T over W-wide rows (A: the item's
+// q~ / q rows, MTT m-tiles; B: the stage's key-side tile), masks past ntok,
+// one online-softmax step per row (maxima exchanged through `red`), P into
+// shared memory, O += P V (V: the stage's value-side tile, W-wide rows).
+template <int W, int MTT, int MTR>
+__device__ __forceinline__ void run_stage(uint32_t qa, uint32_t ktile, uint32_t vtile, unsigned char *sm_p,
+                                          uint32_t pbase, float *red, int ntok, float c2, float (&o)[MTT][W / 32][4],
+                                          float (&mrun)[MTT][2], float (&lpart)[MTT][2], int warp, int lane)
+{
+    constexpr int NT = W / 32;
+    const int grp = lane >> 2, tig = lane & 3;
+    float sc[MTT][2][4];
+#pragma unroll
+    for (int mt = 0; mt < MTT; ++mt)
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt)
+            sc[mt][nt][0] = sc[mt][nt][1] = sc[mt][nt][2] = sc[mt][nt][3] = 0.f;
+    {
+        const int tok = 16 * warp + (lane & 7) + ((lane >> 4) << 3);
+        const int khalf = (lane >> 3) & 1;
+#pragma unroll
+        for (int kk = 0; kk < W / 16; ++kk) {
+            const int ch = 2 * kk + khalf;
+            uint32_t bfr[4];
+            ldsm_x4(swz(ktile + (ch / 8) * 8192, tok, ch % 8), bfr);
+#pragma unroll
+            for (int mt = 0; mt < MTT; ++mt) {
+                const int row = mt * 16 + (lane & 15), ach = 2 * kk + (lane >> 4);
+                uint32_t afr[4];
+                ldsm_x4(swz(qa + (ach / 8) * (MTR * 16 * 128), row, ach % 8), afr);
+                mma_bf16_16816(sc[mt][0], afr, bfr[0], bfr[1]);
+                mma_bf16_16816(sc[mt][1], afr, bfr[2], bfr[3]);
+            }
+        }
+    }
+#pragma unroll
+    for (int mt = 0; mt < MTT; ++mt) {
+        float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int col = 16 * warp + 8 * nt + 2 * tig + e;
+                if (col >= ntok)
+                    sc[mt][nt][e] = sc[mt][nt][2 + e] = -INFINITY;
+                mx0 = fmaxf(mx0, sc[mt][nt][e]);
+                mx1 = fmaxf(mx1, sc[mt][nt][2 + e]);
+            }
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        if (tig == 0) {
+            red[warp * MTT * 16 + mt * 16 + grp] = mx0;
+            red[warp * MTT * 16 + mt * 16 + grp + 8] = mx1;
+        }
+    }
+    consumer_sync<MTT>();
+#pragma unroll
+    for (int mt = 0; mt < MTT; ++mt)
+#pragma unroll
+        for (int hr = 0; hr < 2; ++hr) {
+            const int row = mt * 16 + grp + 8 * hr;
+            float tmax = red[row];
+#pragma unroll
+            for (int w2 = 1; w2 < 4; ++w2)
+                tmax = fmaxf(tmax, red[w2 * MTT * 16 + row]);
+            const float mnew = fmaxf(mrun[mt][hr], tmax * c2);
+            const float alpha = mrun[mt][hr] == -INFINITY ? 0.f : ex2_approx(mrun[mt][hr] - mnew);
+            mrun[mt][hr] = mnew;
+            lpart[mt][hr] *= alpha;
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                o[mt][nt][2 * hr] *= alpha;
+                o[mt][nt][2 * hr + 1] *= alpha;
+            }
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                const float x0 = sc[mt][nt][2 * hr], x1 = sc[mt][nt][2 * hr + 1];
+                const float p0 = x0 == -INFINITY ? 0.f : ex2_approx(fmaf(x0, c2, -mnew));
+                const float p1 = x1 == -INFINITY ? 0.f : ex2_approx(fmaf(x1, c2, -mnew));
+                const uint32_t pk = cvt_bf16x2(p0, p1);
+                lpart[mt][hr] += bf16lo(pk) + bf16hi(pk);  // the weights the PV product uses
+                const int col = 16 * warp + 8 * nt + 2 * tig;
+                *reinterpret_cast<uint32_t *>(sm_p + row * 128 + (((col >> 3) ^ (row & 7)) << 4) + 4 * tig) = pk;
+            }
+        }
+    consumer_sync<MTT>();
+#pragma unroll
+    for (int kk = 0; kk < kTok / 16; ++kk) {
+        uint32_t afr[MTT][4];
+#pragma unroll
+        for (int mt = 0; mt < MTT; ++mt)
+            ldsm_x4(swz(pbase, mt * 16 + (lane & 15), 2 * kk + (lane >> 4)), afr[mt]);
+        const int krow = 16 * kk + (lane & 7) + (((lane >> 3) & 1) << 3);
+#pragma unroll
+        for (int np = 0; np < NT / 2; ++np) {
+            const int n0 = warp * (W / 4) + 16 * np + ((lane >> 4) << 3);
+            uint32_t bfr[4];
+            ldsm_x4_t(swz(vtile + (n0 / 64) * 8192, krow, (n0 % 64) / 8), bfr);
+#pragma unroll
+            for (int mt = 0; mt < MTT; ++mt) {
+                mma_bf16_16816(o[mt][2 * np], afr[mt], bfr[0], bfr[1]);
+                mma_bf16_16816(o[mt][2 * np + 1], afr[mt], bfr[2], bfr[3]);
+            }
+        }
+    }
+}
+
 template <int DL, int MT>
-__global__ void __launch_bounds__(kMainThreads) latent_main_kernel(const __grid_constant__ CUtensorMap tmC, Args a)
+__global__ void __launch_bounds__(kMainThreads2) latent_main_kernel(const __grid_constant__ CUtensorMap tmC,
+                                                                    const __grid_constant__ CUtensorMap tmK,
+                                                                    const __grid_constant__ CUtensorMap tmV, Args a)
 {
     using Ly = MainLayout<DL, MT>;
-    constexpr int NT = DL / 32;  // n-tiles of 8 columns per warp in O
+    constexpr int NST = Ly::NST;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                           ~uintptr_t(1023));
     const uint32_t sbase = smem_u32(sm);
     uint64_t *full = reinterpret_cast<uint64_t *>(sm + Ly::BAR);
-    constexpr int NST = Ly::NST;
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Ly::BAR + 8 * NST);
+    uint64_t *empty = full + NST;
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(empty + NST);
     float *red = reinterpret_cast<float *>(sm + Ly::RED);
+    int *pref = reinterpret_cast<int *>(sm + Ly::PREF);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int b = blockIdx.y;
-    const int L = __ldg(a.seq_lens + b);
     grid_dep_launch();  // the merge kernel may launch; it waits for this grid to finish
 
-    if ((int)blockIdx.x >= a.nspl) {
-        // (reads q, the ring and the lengths, which the work before the prep
-        // kernel wrote: this CTA needs nothing from the prep kernel)
-        // ------------------------------------------------ window CTA: KV head g
-        const int g = blockIdx.x - a.nspl;
-        float *Ks = reinterpret_cast<float *>(sm);      // [kWinChunk][65]
-        float *Vs = Ks + kWinChunk * kWinLd;            // [kWinChunk][65]
-        float *Pw = Vs + kWinChunk * kWinLd;            // [4 warps][kWinChunk]
-        float *Qs = Pw + 4 * kWinChunk;                 // [4 warps][64]
-        if (L < 0 || L > a.maxp * kTok) {
-            if (tid == 0)
-                report(a.status, DAR_ERR_CAPACITY);
-            return;
-        }
-        const int nwin = min(L, a.w), p0 = L - nwin;
-        for (int hh0 = 0; hh0 < a.G; hh0 += 4) {
-            const int hh = hh0 + warp, h = g * a.G + hh;
-            const bool active = hh < a.G;
-            float m = -INFINITY, l = 0.f, acc0 = 0.f, acc1 = 0.f;
-            if (active) {
-                const bf16 *qr = static_cast<const bf16 *>(a.q) + ((size_t)b * a.Hq + h) * 64;
-                Qs[warp * 64 + lane] = __bfloat162float(qr[lane]) * a.c2;
-                Qs[warp * 64 + lane + 32] = __bfloat162float(qr[lane + 32]) * a.c2;
-            }
-            for (int c0 = 0; c0 < nwin; c0 += kWinChunk) {
-                const int nc = min(kWinChunk, nwin - c0);
-                __syncthreads();
-                for (int i = tid; i < nc * 8; i += kMainThreads) {  // 16-byte chunks
-                    const int j = i / 8, ch = i % 8;
-                    const int p = p0 + c0 + j;
-                    const size_t row = ((size_t)b * a.Hkv + g) * a.w + p % a.w;
-                    const uint4 kv = reinterpret_cast<const uint4 *>(a.win_k)[row * 8 + ch];
-                    const uint4 vv = reinterpret_cast<const uint4 *>(a.win_v)[row * 8 + ch];
-                    float kf[8], vf[8];
-                    unpack(kv, kf, bf16());
-                    unpack(vv, vf, bf16());
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        Ks[j * kWinLd + ch * 8 + e] = kf[e];
-                        Vs[j * kWinLd + ch * 8 + e] = vf[e];
-                    }
-                }
-                __syncthreads();
-                if (!active)
-                    continue;
-                float s[kWinChunk / 32];
-                float mx = -INFINITY;
-#pragma unroll
-                for (int u = 0; u < kWinChunk / 32; ++u) {
-                    const int j = lane + 32 * u;
-                    float acc = -INFINITY;
-                    if (j < nc) {
-                        acc = 0.f;
-#pragma unroll 16
-                        for (int t = 0; t < 64; ++t)
-                            acc = fmaf(Qs[warp * 64 + t], Ks[j * kWinLd + t], acc);
-                    }
-                    s[u] = acc;
-                    mx = fmaxf(mx, acc);
-                }
-#pragma unroll
-                for (int o = 16; o; o >>= 1)
-                    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-                const float mnew = fmaxf(m, mx);
-                const float alpha = m == -INFINITY ? 0.f : ex2_approx(m - mnew);
-                float ps = 0.f;
-#pragma unroll
-                for (int u = 0; u < kWinChunk / 32; ++u) {
-                    const float p = s[u] == -INFINITY ? 0.f : ex2_approx(s[u] - mnew);
-                    Pw[warp * kWinChunk + lane + 32 * u] = p;
-                    ps += p;
-                }
-#pragma unroll
-                for (int o = 16; o; o >>= 1)
-                    ps += __shfl_xor_sync(0xffffffffu, ps, o);
-                l = l * alpha + ps;
-                m = mnew;
-                acc0 *= alpha;
-                acc1 *= alpha;
-                __syncwarp();
-                for (int j = 0; j < nc; ++j) {
-                    const float p = Pw[warp * kWinChunk + j];
-                    acc0 = fmaf(p, Vs[j * kWinLd + lane], acc0);
-                    acc1 = fmaf(p, Vs[j * kWinLd + lane + 32], acc1);
-                }
-                __syncwarp();
-            }
-            if (active) {
-                float *rec = a.rec_win + ((size_t)b * a.Hq + h) * 66;
-                rec[lane] = acc0;
-                rec[lane + 32] = acc1;
-                if (lane == 0) {
-                    rec[64] = m;
-                    rec[65] = l;
-                }
-            }
-        }
-        return;
-    }
-
-    // ---------------------------------------------------- latent CTA: 4 pages
-    const int split = blockIdx.x;
-    const int Lg = L > a.w ? L - a.w : 0;
-    if (L > a.maxp * kTok) {
-        if (tid == 0 && split == 0)
+    // lengths -> latent splits per sequence, prefix sums (every CTA, the same)
+    const int B = a.B, cap = a.maxp * kTok;
+    auto len_of = [&](int b) {
+        const int L = __ldg(a.seq_lens + b);
+        return (L < 0 || L > cap) ? 0 : L;  // reported below; such a sequence gets no items
+    };
+    for (int b = tid; b < B; b += blockDim.x) {
+        const int L = __ldg(a.seq_lens + b);
+        if ((L < 0 || L > cap) && blockIdx.x == 0)
             report(a.status, DAR_ERR_CAPACITY);
-        return;
+        const int Lg = len_of(b) > a.w ? len_of(b) - a.w : 0;
+        pref[b + 1] = (Lg + kSplitTok - 1) / kSplitTok;
     }
-    const int t0 = split * kSplitTok, t1 = min(Lg, t0 + kSplitTok);
-    if (t0 >= t1)
-        return;  // the merge reads only the splits that hold tokens
-    const int npg = (t1 - t0 + kTok - 1) / kTok;
+    __syncthreads();
+    if (warp == 0) {
+        int run = 0;
+        for (int c0 = 0; c0 < B; c0 += 32) {
+            int v = c0 + lane < B ? pref[c0 + lane + 1] : 0;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int u = __shfl_up_sync(0xffffffffu, v, o);
+                if (lane >= o)
+                    v += u;
+            }
+            if (c0 + lane < B)
+                pref[c0 + lane + 1] = run + v;
+            run += __shfl_sync(0xffffffffu, v, 31);
+        }
+        if (lane == 0)
+            pref[0] = 0;
+    }
     if (tid == 0) {
-        for (int st = 0; st < NST; ++st)
+        for (int st = 0; st < NST; ++st) {
             mbar_init(&full[st], 1);
+            mbar_init(&empty[st], 4);  // one arrival per consumer warp
+        }
         *abort_flag = 0;
         mbar_init_fence();
-        prefetch_tensormap(&tmC);
     }
     __syncthreads();
-    auto issue = [&](int pi) {  // thread 0: page pi of the split into buffer pi % NST
-        int pid = __ldg(a.block_table + (size_t)b * a.maxp + t0 / kTok + pi);
-        if (pid < 0 || pid >= a.num_pages) {
-            report(a.status, DAR_ERR_CAPACITY);
-            pid = 0;
+    const int n_lat = pref[B], n_items = n_lat + B * a.Hkv;
+    auto item_of = [&](int k) {
+        Item it;
+        if (k < n_lat) {
+            int lo = 0, hi = B - 1;  // the last b with pref[b] <= k
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (pref[mid] <= k)
+                    lo = mid;
+                else
+                    hi = mid - 1;
+            }
+            it.latent = true;
+            it.b = lo;
+            it.part = k - pref[lo];
+            const int L = len_of(lo), Lg = L > a.w ? L - a.w : 0;
+            const int t0 = it.part * kSplitTok, t1 = min(Lg, t0 + kSplitTok);
+            it.npg = (t1 - t0 + kTok - 1) / kTok;
+        } else {
+            const int r = k - n_lat;
+            it.latent = false;
+            it.b = r / a.Hkv;
+            it.part = r % a.Hkv;
+            const int nwin = min(len_of(it.b), a.w);
+            it.npg = (nwin + kTok - 1) / kTok;
         }
-        uint64_t *bar = &full[pi % NST];
-        mbar_expect_tx(bar, kTok * DL * 2);
-#pragma unroll
-        for (int cb = 0; cb < DL / 64; ++cb)
-            tma_load_2d(sm + Ly::CB + (pi % NST) * Ly::CSTAGE + cb * 8192, &tmC, cb * 64, pid * kTok, bar);
+        return it;
     };
-    if (tid == 0)
-        for (int pi = 0; pi < NST && pi < npg; ++pi)
-            issue(pi);
-    grid_dep_wait();  // q~ comes from the prep kernel
-    // q~ rows (zero past Hq) into the swizzled operand tile
-    for (int i = tid; i < MT * 16 * (DL / 8); i += kMainThreads) {
-        const int r = i / (DL / 8), ch = i % (DL / 8);
-        uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if (r < a.Hq)
-            v = *reinterpret_cast<const uint4 *>(a.qt + ((size_t)b * a.Hq + r) * DL + ch * 8);
-        *reinterpret_cast<uint4 *>(sm + Ly::QT + (ch / 8) * (MT * 16 * 128) + r * 128 +
-                                   (((ch % 8) ^ (r & 7)) << 4)) = v;
-    }
-    __syncthreads();
 
-    float o[MT][NT][4];
+    if (warp == 4) {
+        // ------------------------------------------------ producer
+        if (lane == 0) {
+            prefetch_tensormap(&tmC);
+            prefetch_tensormap(&tmK);
+            prefetch_tensormap(&tmV);
+            int gp = 0;
+            for (int k = blockIdx.x; k < n_items; k += gridDim.x) {
+                const Item it = item_of(k);
+                for (int p = 0; p < it.npg; ++p, ++gp) {
+                    const int st = gp % NST;
+                    if (gp >= NST && !mbar_wait(&empty[st], ((gp / NST) - 1) & 1, abort_flag))
+                        goto done;
+                    unsigned char *dst = sm + Ly::STG + st * Ly::CST;
+                    if (it.latent) {
+                        int pid = __ldg(a.block_table + (size_t)it.b * a.maxp + it.part * kPagesPerSplit + p);
+                        if (pid < 0 || pid >= a.num_pages) {
+                            report(a.status, DAR_ERR_CAPACITY);
+                            pid = 0;
+                        }
+                        mbar_expect_tx(&full[st], kTok * DL * 2);
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
-            o[mt][nt][0] = o[mt][nt][1] = o[mt][nt][2] = o[mt][nt][3] = 0.f;
-    float mrun[MT][2], lpart[MT][2];
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
-        mrun[mt][0] = mrun[mt][1] = -INFINITY, lpart[mt][0] = lpart[mt][1] = 0.f;
-    const int grp = lane >> 2, tig = lane & 3;
-    bool ok = true;
-
-    for (int pi = 0; pi < npg; ++pi) {
-        const int s = pi % NST;
-        if (!mbar_wait(&full[s], (pi / NST) & 1, abort_flag))
-            ok = false;
-        if (__syncthreads_or(!ok)) {
-            ok = false;
-            break;
-        }
-        const uint32_t cbuf = sbase + Ly::CB + s * Ly::CSTAGE;
-        const int ntok = min(kTok, t1 - (t0 + pi * kTok));
-        if (ntok < kTok) {  // rows past the last distant token: zero (their P is 0; 0 * NaN must not arise)
-            for (int i = tid; i < (kTok - ntok) * (DL / 8); i += kMainThreads) {
-                const int r = ntok + i / (DL / 8), ch = i % (DL / 8);
-                *reinterpret_cast<uint4 *>(sm + Ly::CB + s * Ly::CSTAGE + (ch / 8) * 8192 + r * 128 +
-                                           (((ch % 8) ^ (r & 7)) << 4)) = make_uint4(0u, 0u, 0u, 0u);
-            }
-            __syncthreads();
-        }
-        // S = Q~ C^T: this warp's 16 tokens (two n-tiles) for every head row
-        float sc[MT][2][4];
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-                sc[mt][nt][0] = sc[mt][nt][1] = sc[mt][nt][2] = sc[mt][nt][3] = 0.f;
-        {
-            const int tok = 16 * warp + (lane & 7) + ((lane >> 4) << 3);
-            const int khalf = (lane >> 3) & 1;
-#pragma unroll
-            for (int kk = 0; kk < DL / 16; ++kk) {
-                const int ch = 2 * kk + khalf;  // 16-byte chunk along d_lat
-                uint32_t bfr[4];
-                ldsm_x4(swz(cbuf + (ch / 8) * 8192, tok, ch % 8), bfr);
-#pragma unroll
-                for (int mt = 0; mt < MT; ++mt) {
-                    const int row = mt * 16 + (lane & 15), ach = 2 * kk + (lane >> 4);
-                    uint32_t afr[4];
-                    ldsm_x4(swz(sbase + Ly::QT + (ach / 8) * (MT * 16 * 128), row, ach % 8), afr);
-                    mma_bf16_16816(sc[mt][0], afr, bfr[0], bfr[1]);
-                    mma_bf16_16816(sc[mt][1], afr, bfr[2], bfr[3]);
+                        for (int cb = 0; cb < DL / 64; ++cb)
+                            tma_load_2d(dst + cb * 8192, &tmC, cb * 64, pid * kTok, &full[st]);
+                    } else {
+                        const int row = (it.b * a.Hkv + it.part) * a.w + p * kTok;
+                        mbar_expect_tx(&full[st], 2 * 8192);
+                        tma_load_2d(dst, &tmK, 0, row, &full[st]);
+                        tma_load_2d(dst + 8192, &tmV, 0, row, &full[st]);
+                    }
                 }
             }
-        }
-        // masks and per-warp row maxima
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int col = 16 * warp + 8 * nt + 2 * tig + e;
-                    if (col >= ntok)
-                        sc[mt][nt][e] = sc[mt][nt][2 + e] = -INFINITY;
-                    mx0 = fmaxf(mx0, sc[mt][nt][e]);
-                    mx1 = fmaxf(mx1, sc[mt][nt][2 + e]);
-                }
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-            if (tig == 0) {
-                red[warp * MT * 16 + mt * 16 + grp] = mx0;
-                red[warp * MT * 16 + mt * 16 + grp + 8] = mx1;
-            }
-        }
-        __syncthreads();
-        // running maxima (log2 units), P = 2^(s c2 - m) into shared memory, rescale O
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-            for (int hr = 0; hr < 2; ++hr) {
-                const int row = mt * 16 + grp + 8 * hr;
-                float tmax = red[row];
-#pragma unroll
-                for (int w2 = 1; w2 < 4; ++w2)
-                    tmax = fmaxf(tmax, red[w2 * MT * 16 + row]);
-                const float mnew = fmaxf(mrun[mt][hr], tmax * a.c2);
-                const float alpha = mrun[mt][hr] == -INFINITY ? 0.f : ex2_approx(mrun[mt][hr] - mnew);
-                mrun[mt][hr] = mnew;
-                lpart[mt][hr] *= alpha;
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt) {
-                    o[mt][nt][2 * hr] *= alpha;
-                    o[mt][nt][2 * hr + 1] *= alpha;
-                }
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt) {
-                    const float x0 = sc[mt][nt][2 * hr], x1 = sc[mt][nt][2 * hr + 1];
-                    const float p0 = x0 == -INFINITY ? 0.f : ex2_approx(fmaf(x0, a.c2, -mnew));
-                    const float p1 = x1 == -INFINITY ? 0.f : ex2_approx(fmaf(x1, a.c2, -mnew));
-                    const uint32_t pk = cvt_bf16x2(p0, p1);
-                    lpart[mt][hr] += bf16lo(pk) + bf16hi(pk);  // the weights the PV product uses
-                    const int col = 16 * warp + 8 * nt + 2 * tig;
-                    *reinterpret_cast<uint32_t *>(sm + Ly::P + row * 128 + (((col >> 3) ^ (row & 7)) << 4) +
-                                                  4 * tig) = pk;
-                }
-            }
-        __syncthreads();
-        // O += P C: this warp's DL/4 columns, K = the page's 64 tokens
-#pragma unroll
-        for (int kk = 0; kk < kTok / 16; ++kk) {
-            uint32_t afr[MT][4];
-#pragma unroll
-            for (int mt = 0; mt < MT; ++mt)
-                ldsm_x4(swz(sbase + Ly::P, mt * 16 + (lane & 15), 2 * kk + (lane >> 4)), afr[mt]);
-            const int krow = 16 * kk + (lane & 7) + (((lane >> 3) & 1) << 3);
-#pragma unroll
-            for (int np = 0; np < NT / 2; ++np) {
-                const int n0 = warp * (DL / 4) + 16 * np + ((lane >> 4) << 3);  // column of this lane's matrix
-                uint32_t bfr[4];
-                ldsm_x4_t(swz(cbuf + (n0 / 64) * 8192, krow, (n0 % 64) / 8), bfr);
-#pragma unroll
-                for (int mt = 0; mt < MT; ++mt) {
-                    mma_bf16_16816(o[mt][2 * np], afr[mt], bfr[0], bfr[1]);
-                    mma_bf16_16816(o[mt][2 * np + 1], afr[mt], bfr[2], bfr[3]);
-                }
-            }
-        }
-        __syncthreads();  // buffer s and P are free again
-        if (tid == 0 && pi + NST < npg) {
-            fence_proxy_async_smem();
-            issue(pi + NST);
-        }
-    }
-    if (!ok) {
-        // let copies still in flight land before the CTA exits
-        if (tid == 0) {
-            for (int st = 0; st < NST && st < npg; ++st)
-                mbar_wait(&full[st], 0, nullptr);
-            report(a.status, DAR_ERR_DEVICE);
+        done:;
         }
         return;
     }
 
-    // row sums: across the quad, then across the four warps
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            float ls = lpart[mt][hr];
-            ls += __shfl_xor_sync(0xffffffffu, ls, 1);
-            ls += __shfl_xor_sync(0xffffffffu, ls, 2);
-            lpart[mt][hr] = ls;
-        }
-    __syncthreads();
-    if (tig == 0)
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            red[warp * MT * 16 + mt * 16 + grp] = lpart[mt][0];
-            red[warp * MT * 16 + mt * 16 + grp + 8] = lpart[mt][1];
-        }
-    __syncthreads();
-    const size_t rbase = ((size_t)b * a.nspl + split) * a.Hq;
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-        for (int hr = 0; hr < 2; ++hr) {
-            const int row = mt * 16 + grp + 8 * hr;
-            if (row >= a.Hq)
-                continue;
-            float *rec = a.rec_lat + (rbase + row) * (DL + 2);
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const int col = warp * (DL / 4) + 8 * nt + 2 * tig;
-                *reinterpret_cast<float2 *>(rec + col) = make_float2(o[mt][nt][2 * hr], o[mt][nt][2 * hr + 1]);
+    // ---------------------------------------------------- consumers (warps 0-3)
+    grid_dep_wait();  // q~ comes from the prep kernel
+    const int grp = lane >> 2, tig = lane & 3;
+    int gp = 0;
+    bool ok = true;
+    for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+        const Item it = item_of(k);
+        if (it.npg == 0)
+            continue;
+        if (it.latent) {
+            // q~ rows of every head (zero past Hq) into the A-operand tile
+            for (int i = tid; i < MT * 16 * (DL / 8); i += kConsumerThreads) {
+                const int r = i / (DL / 8), ch = i % (DL / 8);
+                uint4 v = make_uint4(0u, 0u, 0u, 0u);
+                if (r < a.Hq)
+                    v = *reinterpret_cast<const uint4 *>(a.qt + ((size_t)it.b * a.Hq + r) * DL + ch * 8);
+                *reinterpret_cast<uint4 *>(sm + Ly::QA + (ch / 8) * (MT * 16 * 128) + r * 128 +
+                                           (((ch % 8) ^ (r & 7)) << 4)) = v;
             }
-            if (warp == 0 && tig == 0) {
-                rec[DL] = mrun[mt][hr];
-                rec[DL + 1] = red[row] + red[MT * 16 + row] + red[2 * MT * 16 + row] + red[3 * MT * 16 + row];
+        } else {
+            // q rows of KV head g's query heads (zero past G) into a 64-wide A tile
+            for (int i = tid; i < 16 * 8; i += kConsumerThreads) {
+                const int r = i / 8, ch = i % 8;
+                uint4 v = make_uint4(0u, 0u, 0u, 0u);
+                if (r < a.G)
+                    v = *reinterpret_cast<const uint4 *>(static_cast<const bf16 *>(a.q) +
+                                                         ((size_t)it.b * a.Hq + it.part * a.G + r) * 64 + ch * 8);
+                *reinterpret_cast<uint4 *>(sm + Ly::QA + r * 128 + ((ch ^ (r & 7)) << 4)) = v;
             }
         }
+        consumer_sync<MT>();
+        const int L = len_of(it.b), Lg = L > a.w ? L - a.w : 0, nwin = min(L, a.w);
+        // Wait for a stage, zero its rows past the item's last token (their P is
+        // 0; 0 * NaN must not arise), then one barrier so every consumer thread
+        // takes the same decision if any wait gave up (the flag is set first).
+        auto stage_wait = [&](int st, int ntok, int rows_w) -> bool {
+            const bool got = mbar_wait(&full[st], (gp / NST) & 1, abort_flag);
+            if (got && ntok < kTok) {
+                unsigned char *t = sm + Ly::STG + st * Ly::CST;
+                for (int i = tid; i < (kTok - ntok) * (rows_w / 8); i += kConsumerThreads) {
+                    const int r = ntok + i / (rows_w / 8), ch = i % (rows_w / 8);
+                    *reinterpret_cast<uint4 *>(t + (ch / 8) * 8192 + r * 128 + (((ch % 8) ^ (r & 7)) << 4)) =
+                        make_uint4(0u, 0u, 0u, 0u);
+                }
+                fence_proxy_async_smem();  // these writes precede the stage's next TMA fill
+            }
+            consumer_sync<MT>();
+            return *abort_flag == 0;
+        };
+        auto release = [&](int st) {
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&empty[st]);
+        };
+        if (it.latent) {
+            float o[MT][DL / 32][4];
+            float mrun[MT][2], lpart[MT][2];
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+                for (int nt = 0; nt < DL / 32; ++nt)
+                    o[mt][nt][0] = o[mt][nt][1] = o[mt][nt][2] = o[mt][nt][3] = 0.f;
+                mrun[mt][0] = mrun[mt][1] = -INFINITY;
+                lpart[mt][0] = lpart[mt][1] = 0.f;
+            }
+            const int t0 = it.part * kSplitTok, t1 = min(Lg, t0 + kSplitTok);
+            for (int p = 0; p < it.npg; ++p, ++gp) {
+                const int st = gp % NST, ntok = min(kTok, t1 - (t0 + p * kTok));
+                if (!stage_wait(st, ntok, DL)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t t = sbase + Ly::STG + st * Ly::CST;
+                run_stage<DL, MT, MT>(sbase + Ly::QA, t, t, sm + Ly::P, sbase + Ly::P, red, ntok, a.c2, o, mrun,
+                                      lpart, warp, lane);
+                release(st);
+            }
+            if (!ok)
+                break;
+            // record (O_lat, m, l) of every head: row sums across the quad, then the warps
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+                for (int hr = 0; hr < 2; ++hr) {
+                    float ls = lpart[mt][hr];
+                    ls += __shfl_xor_sync(0xffffffffu, ls, 1);
+                    ls += __shfl_xor_sync(0xffffffffu, ls, 2);
+                    lpart[mt][hr] = ls;
+                }
+            consumer_sync<MT>();
+            if (tig == 0)
+#pragma unroll
+                for (int mt = 0; mt < MT; ++mt) {
+                    red[warp * MT * 16 + mt * 16 + grp] = lpart[mt][0];
+                    red[warp * MT * 16 + mt * 16 + grp + 8] = lpart[mt][1];
+                }
+            consumer_sync<MT>();
+            const size_t rbase = ((size_t)it.b * a.nspl + it.part) * a.Hq;
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+                for (int hr = 0; hr < 2; ++hr) {
+                    const int row = mt * 16 + grp + 8 * hr;
+                    if (row >= a.Hq)
+                        continue;
+                    float *rec = a.rec_lat + (rbase + row) * (DL + 2);
+#pragma unroll
+                    for (int nt = 0; nt < DL / 32; ++nt) {
+                        const int col = warp * (DL / 4) + 8 * nt + 2 * tig;
+                        *reinterpret_cast<float2 *>(rec + col) =
+                            make_float2(o[mt][nt][2 * hr], o[mt][nt][2 * hr + 1]);
+                    }
+                    if (warp == 0 && tig == 0) {
+                        rec[DL] = mrun[mt][hr];
+                        rec[DL + 1] =
+                            red[row] + red[MT * 16 + row] + red[2 * MT * 16 + row] + red[3 * MT * 16 + row];
+                    }
+                }
+        } else {
+            float o[1][2][4];
+            float mrun[1][2] = {{-INFINITY, -INFINITY}}, lpart[1][2] = {{0.f, 0.f}};
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+                o[0][nt][0] = o[0][nt][1] = o[0][nt][2] = o[0][nt][3] = 0.f;
+            for (int p = 0; p < it.npg; ++p, ++gp) {
+                const int st = gp % NST, ntok = min(kTok, nwin - p * kTok);
+                // zero both tiles' rows past the window (K block at +0, V block at +8192)
+                if (!stage_wait(st, ntok, 128)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t t = sbase + Ly::STG + st * Ly::CST;
+                run_stage<64, 1, 1>(sbase + Ly::QA, t, t + 8192, sm + Ly::P, sbase + Ly::P, red, ntok, a.c2, o, mrun,
+                                    lpart, warp, lane);
+                release(st);
+            }
+            if (!ok)
+                break;
+#pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+                float ls = lpart[0][hr];
+                ls += __shfl_xor_sync(0xffffffffu, ls, 1);
+                ls += __shfl_xor_sync(0xffffffffu, ls, 2);
+                lpart[0][hr] = ls;
+            }
+            consumer_sync<MT>();
+            if (tig == 0) {
+                red[warp * 16 + grp] = lpart[0][0];
+                red[warp * 16 + grp + 8] = lpart[0][1];
+            }
+            consumer_sync<MT>();
+#pragma unroll
+            for (int hr = 0; hr < 2; ++hr) {
+                const int row = grp + 8 * hr;
+                if (row >= a.G)
+                    continue;
+                float *rec = a.rec_win + ((size_t)it.b * a.Hq + it.part * a.G + row) * 66;
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt) {
+                    const int col = warp * 16 + 8 * nt + 2 * tig;
+                    *reinterpret_cast<float2 *>(rec + col) = make_float2(o[0][nt][2 * hr], o[0][nt][2 * hr + 1]);
+                }
+                if (warp == 0 && tig == 0) {
+                    rec[64] = mrun[0][hr];
+                    rec[65] = red[row] + red[16 + row] + red[32 + row] + red[48 + row];
+                }
+            }
+        }
+        consumer_sync<MT>();  // the A tile and `red` are reused by the next item
+    }
+    if (!ok && tid == 0)
+        report(a.status, DAR_ERR_DEVICE);
 }
 
 // ---------------------------------------------------------------- decode: merge
@@ -693,39 +771,53 @@ static EncodeTiledFn encode_fn()
     return fn;
 }
 
-template <int DL, int MT>
-static cudaError_t decode_t(const Args &a, const void *pool_c, cudaStream_t s)
+static bool encode_2d(CUtensorMap *tm, const void *base, unsigned long long rows, int cols)
 {
-    using Ly = MainLayout<DL, MT>;
-    constexpr size_t win_smem = (2 * kWinChunk * kWinLd + 4 * kWinChunk + 4 * 64) * sizeof(float);
-    const size_t smem = 1024 + (Ly::TOTAL > win_smem ? Ly::TOTAL : win_smem);
-    constexpr size_t prep_smem = (size_t)64 * DL * sizeof(float) + 16;
-    constexpr size_t merge_smem = ((size_t)DL * 64 + 4 * DL + 4 * 32) * sizeof(float) + 16;
-    static PerDeviceOnce once;
-    cudaError_t e = per_device_once(once, [&](int) {
-        cudaError_t e2 = cudaFuncSetAttribute(latent_main_kernel<DL, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              (int)smem);
-        if (e2 == cudaSuccess)
-            e2 = cudaFuncSetAttribute(latent_prep_kernel<DL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)prep_smem);
-        if (e2 == cudaSuccess)
-            e2 = cudaFuncSetAttribute(latent_merge_kernel<DL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)merge_smem);
-        return e2;
-    });
-    if (e != cudaSuccess)
-        return e;
     EncodeTiledFn enc = encode_fn();
     if (!enc)
-        return cudaErrorNotSupported;
-    CUtensorMap tm;
-    const cuuint64_t dims[2] = {(cuuint64_t)DL, (cuuint64_t)a.num_pages * kTok};
-    const cuuint64_t strides[1] = {(cuuint64_t)DL * 2};
+        return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
     const cuuint32_t box[2] = {64, (cuuint32_t)kTok};
     const cuuint32_t estr[2] = {1, 1};
-    if (enc(&tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(pool_c), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int DL, int MT>
+static cudaError_t decode_t(const Args &a, const void *pool_c, const void *win_k, const void *win_v, cudaStream_t s)
+{
+    using Ly = MainLayout<DL, MT>;
+    const size_t smem = 1024 + Ly::TOTAL;
+    constexpr size_t prep_smem = (size_t)64 * DL * sizeof(float) + 16;
+    constexpr size_t merge_smem = ((size_t)DL * 64 + 4 * DL + 4 * 32) * sizeof(float) + 16;
+    static PerDeviceOnce once;  // records the SM count
+    int sms = 0;
+    cudaError_t e = per_device_once(
+        once,
+        [&](int dev) {
+            cudaError_t e2 = cudaFuncSetAttribute(latent_main_kernel<DL, MT>,
+                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (e2 == cudaSuccess)
+                e2 = cudaFuncSetAttribute(latent_prep_kernel<DL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)prep_smem);
+            if (e2 == cudaSuccess)
+                e2 = cudaFuncSetAttribute(latent_merge_kernel<DL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)merge_smem);
+            int n = 0;
+            if (e2 == cudaSuccess)
+                e2 = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+            once.value[dev] = n;
+            return e2;
+        },
+        &sms);
+    if (e != cudaSuccess)
+        return e;
+    CUtensorMap tm[3];
+    if (!encode_2d(&tm[0], pool_c, (unsigned long long)a.num_pages * kTok, DL) ||
+        !encode_2d(&tm[1], win_k, (unsigned long long)a.B * a.Hkv * a.w, 64) ||
+        !encode_2d(&tm[2], win_v, (unsigned long long)a.B * a.Hkv * a.w, 64))
         return cudaErrorInvalidValue;
     // prep starts after all earlier work on the stream; main and merge are
     // launched programmatically (each waits in-kernel for what it reads)
@@ -738,10 +830,10 @@ static cudaError_t decode_t(const Args &a, const void *pool_c, cudaStream_t s)
     cfg.stream = s;
     cfg.attrs = pdl;
     cfg.numAttrs = 1;
-    cfg.gridDim = dim3(a.nspl + a.Hkv, a.B);
-    cfg.blockDim = dim3(kMainThreads);
+    cfg.gridDim = dim3(2 * (sms > 0 ? sms : 1));  // persistent: two CTAs per SM
+    cfg.blockDim = dim3(kMainThreads2);
     cfg.dynamicSmemBytes = smem;
-    e = cudaLaunchKernelEx(&cfg, latent_main_kernel<DL, MT>, tm, a);
+    e = cudaLaunchKernelEx(&cfg, latent_main_kernel<DL, MT>, tm[0], tm[1], tm[2], a);
     if (e != cudaSuccess)
         return e;
     cfg.gridDim = rgrid;
@@ -754,9 +846,9 @@ static cudaError_t decode_t(const Args &a, const void *pool_c, cudaStream_t s)
 }
 
 template <int DL>
-static cudaError_t decode_dl(const Args &a, const void *pool_c, cudaStream_t s)
+static cudaError_t decode_dl(const Args &a, const void *pool_c, const void *win_k, const void *win_v, cudaStream_t s)
 {
-    return a.Hq <= 16 ? decode_t<DL, 1>(a, pool_c, s) : decode_t<DL, 2>(a, pool_c, s);
+    return a.Hq <= 16 ? decode_t<DL, 1>(a, pool_c, win_k, win_v, s) : decode_t<DL, 2>(a, pool_c, win_k, win_v, s);
 }
 
 }  // namespace lat
@@ -799,10 +891,10 @@ cudaError_t launch_latent_decode(const LatentDecodeArgs &x, void *workspace, cud
     p += al((size_t)x.B * a.nspl * x.Hq * (x.DL + 2) * 4);
     a.rec_win = reinterpret_cast<float *>(p);
     switch (x.DL) {
-    case 64: return lat::decode_dl<64>(a, x.pool_c, s);
-    case 128: return lat::decode_dl<128>(a, x.pool_c, s);
-    case 192: return lat::decode_dl<192>(a, x.pool_c, s);
-    case 256: return lat::decode_dl<256>(a, x.pool_c, s);
+    case 64: return lat::decode_dl<64>(a, x.pool_c, x.win_k, x.win_v, s);
+    case 128: return lat::decode_dl<128>(a, x.pool_c, x.win_k, x.win_v, s);
+    case 192: return lat::decode_dl<192>(a, x.pool_c, x.win_k, x.win_v, s);
+    case 256: return lat::decode_dl<256>(a, x.pool_c, x.win_k, x.win_v, s);
     default: return cudaErrorInvalidValue;
     }
 }
