@@ -47,7 +47,7 @@ struct Args {
     int32_t *status;
     const float *Ak, *Av;  // [Hkv][64][DL] (transposed), [Hkv][DL][64]
     bf16 *qt;              // [B][Hq][DL]
-    float *rec_lat;        // [B][nspl][Hq][DL + 2]
+    float *rec_lat;        // [B][Hq][nspl][DL + 2]
     float *rec_win;        // [B][Hq][66]
     int B, Hq, Hkv, G, w, maxp, num_pages, nspl;
     float c2;  // scale * log2(e)
@@ -587,7 +587,6 @@ __global__ void __launch_bounds__(kMainThreads2) latent_main_kernel(const __grid
                     red[warp * MT * 16 + mt * 16 + grp + 8] = lpart[mt][1];
                 }
             consumer_sync<MT>();
-            const size_t rbase = ((size_t)it.b * a.nspl + it.part) * a.Hq;
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
@@ -595,7 +594,8 @@ __global__ void __launch_bounds__(kMainThreads2) latent_main_kernel(const __grid
                     const int row = mt * 16 + grp + 8 * hr;
                     if (row >= a.Hq)
                         continue;
-                    float *rec = a.rec_lat + (rbase + row) * (DL + 2);
+                    // records of one (b, h) are consecutive over the splits
+                    float *rec = a.rec_lat + (((size_t)it.b * a.Hq + row) * a.nspl + it.part) * (DL + 2);
 #pragma unroll
                     for (int nt = 0; nt < DL / 32; ++nt) {
                         const int col = warp * (DL / 4) + 8 * nt + 2 * tig;
@@ -683,7 +683,6 @@ __global__ void __launch_bounds__(128) latent_merge_kernel(Args a)
         return;
     grid_dep_wait();  // the main kernel's records
     const int nrows = a.B * a.G;
-    const size_t sstride = (size_t)a.Hq * (DL + 2);
     for (int r = blockIdx.y * kRowsPerBlock + warp; r < min(nrows, (int)(blockIdx.y + 1) * kRowsPerBlock); r += 4) {
         const int b = r / a.G, h = g * a.G + r % a.G, row = b * a.Hq + h;
         int L = __ldg(a.seq_lens + b);
@@ -692,11 +691,14 @@ __global__ void __launch_bounds__(128) latent_merge_kernel(Args a)
         const int Lg = L > a.w ? L - a.w : 0;
         const int ns = (Lg + kSplitTok - 1) / kSplitTok;
         const float *rw = a.rec_win + (size_t)row * 66;
-        const float *rl0 = a.rec_lat + ((size_t)b * a.nspl * a.Hq + h) * (DL + 2);
+        const float *rl0 = a.rec_lat + (size_t)row * a.nspl * (DL + 2);  // this row's splits, consecutive
         const float mw = L > 0 ? rw[64] : -INFINITY;
+        // the splits' maxima and sums, one split per lane (32 at a time); the
+        // weighted sum of their O in batches of 8 splits with every load issued
+        // before it is used
         float M = mw;
         for (int s2 = lane; s2 < ns; s2 += 32)
-            M = fmaxf(M, rl0[s2 * sstride + DL]);
+            M = fmaxf(M, rl0[s2 * (DL + 2) + DL]);
 #pragma unroll
         for (int o = 16; o; o >>= 1)
             M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
@@ -708,20 +710,27 @@ __global__ void __launch_bounds__(128) latent_merge_kernel(Args a)
         for (int s0 = 0; s0 < ns; s0 += 32) {
             float f = 0.f;
             if (s0 + lane < ns) {
-                const float *rl = rl0 + (s0 + lane) * sstride;
+                const float *rl = rl0 + (s0 + lane) * (DL + 2);
                 f = ex2_approx(rl[DL] - M);
                 l += f * rl[DL + 1];
             }
             fs[warp * 32 + lane] = f;
             __syncwarp();
             const int n = min(32, ns - s0);
-#pragma unroll 4
-            for (int j = 0; j < n; ++j) {
-                const float *rl = rl0 + (s0 + j) * sstride;
-                const float fj = fs[warp * 32 + j];
+            for (int j0 = 0; j0 < n; j0 += 8) {
+                float x[8][DL / 32];
 #pragma unroll
-                for (int e = 0; e < DL / 32; ++e)
-                    acc[e] = fmaf(fj, rl[lane + 32 * e], acc[e]);
+                for (int j = 0; j < 8; ++j)
+#pragma unroll
+                    for (int e = 0; e < DL / 32; ++e)
+                        x[j][e] = j0 + j < n ? rl0[(s0 + j0 + j) * (DL + 2) + lane + 32 * e] : 0.f;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const float fj = j0 + j < n ? fs[warp * 32 + j0 + j] : 0.f;
+#pragma unroll
+                    for (int e = 0; e < DL / 32; ++e)
+                        acc[e] = fmaf(fj, x[j][e], acc[e]);
+                }
             }
             __syncwarp();
         }
