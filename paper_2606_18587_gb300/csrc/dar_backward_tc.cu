@@ -126,7 +126,7 @@ struct DqLayout {
 };
 
 template <int DD>
-__global__ void __launch_bounds__(kTc) bwd_dq_tc_kernel(Args a)
+__global__ void __launch_bounds__(kTc, DD <= 32 ? 3 : 1) bwd_dq_tc_kernel(Args a)
 {
     using Ly = DqLayout<DD>;
     constexpr int LD = Ly::LD, KSD = DD / 16, NTD = DD / 8;
@@ -177,12 +177,10 @@ __global__ void __launch_bounds__(kTc) bwd_dq_tc_kernel(Args a)
     cp_wait<1>();  // the query-side rows (the first key stage may still be in flight)
     __syncthreads();
 
-    uint32_t qa[4][4], doa[4][4], qta[KSD][4], dota[KSD][4];
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-        ldsm_x4(a_addr<kLdW>(sb + Ly::Q, wr0, kk, lane), qa[kk]);
-        ldsm_x4(a_addr<kLdW>(sb + Ly::DO, wr0, kk, lane), doa[kk]);
-    }
+    // A fragments: the d_down-wide rows stay in registers (every global step
+    // uses them); the 64-wide q and dO rows are read from shared memory by the
+    // (rarer) steps with local pairs, which keeps registers for occupancy
+    uint32_t qta[KSD][4], dota[KSD][4];
 #pragma unroll
     for (int kk = 0; kk < KSD; ++kk) {
         ldsm_x4(a_addr<LD>(sb + Ly::QT, wr0, kk, lane), qta[kk]);
@@ -240,10 +238,11 @@ __global__ void __launch_bounds__(kTc) bwd_dq_tc_kernel(Args a)
             if (!all_global) {
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
-                    uint32_t bfr[4];
+                    uint32_t bfr[4], afr[4];
+                    ldsm_x4(a_addr<kLdW>(sb + Ly::Q, wr0, kk, lane), afr);
                     ldsm_x4(b_addr<kLdW>(stg + Ly::K_OFF, 16 * kc, kk, lane), bfr);
-                    mma_bf16_16816(sl[0], qa[kk], bfr[0], bfr[1]);
-                    mma_bf16_16816(sl[1], qa[kk], bfr[2], bfr[3]);
+                    mma_bf16_16816(sl[0], afr, bfr[0], bfr[1]);
+                    mma_bf16_16816(sl[1], afr, bfr[2], bfr[3]);
                 }
             }
             if (!all_local) {
@@ -331,10 +330,11 @@ __global__ void __launch_bounds__(kTc) bwd_dq_tc_kernel(Args a)
             if (!all_global) {
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
-                    uint32_t bfr[4];
+                    uint32_t bfr[4], afr[4];
+                    ldsm_x4(a_addr<kLdW>(sb + Ly::DO, wr0, kk, lane), afr);
                     ldsm_x4(b_addr<kLdW>(stg + Ly::V_OFF, 16 * kc, kk, lane), bfr);
-                    mma_bf16_16816(dpl[0], doa[kk], bfr[0], bfr[1]);
-                    mma_bf16_16816(dpl[1], doa[kk], bfr[2], bfr[3]);
+                    mma_bf16_16816(dpl[0], afr, bfr[0], bfr[1]);
+                    mma_bf16_16816(dpl[1], afr, bfr[2], bfr[3]);
                 }
             }
             if (!all_local) {
@@ -442,7 +442,7 @@ struct DkvLayout {
 };
 
 template <int DD>
-__global__ void __launch_bounds__(kTc) bwd_dkv_tc_kernel(Args a)
+__global__ void __launch_bounds__(kTc, DD <= 32 ? 3 : 1) bwd_dkv_tc_kernel(Args a)
 {
     using Ly = DkvLayout<DD>;
     constexpr int LD = Ly::LD, KSD = DD / 16, NTD = DD / 8;
@@ -490,12 +490,9 @@ __global__ void __launch_bounds__(kTc) bwd_dkv_tc_kernel(Args a)
     cp_wait<1>();  // the key-side rows
     __syncthreads();
 
-    uint32_t ka[4][4], va[4][4], kda[KSD][4], vda[KSD][4];
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-        ldsm_x4(a_addr<kLdW>(sb + Ly::K, wk0, kk, lane), ka[kk]);
-        ldsm_x4(a_addr<kLdW>(sb + Ly::V, wk0, kk, lane), va[kk]);
-    }
+    // A fragments: the d_down-wide key rows stay in registers; the 64-wide k
+    // and v rows are read from shared memory by the steps with local pairs
+    uint32_t kda[KSD][4], vda[KSD][4];
 #pragma unroll
     for (int kk = 0; kk < KSD; ++kk) {
         ldsm_x4(a_addr<LD>(sb + Ly::KD, wk0, kk, lane), kda[kk]);
@@ -533,10 +530,11 @@ __global__ void __launch_bounds__(kTc) bwd_dkv_tc_kernel(Args a)
             if (!all_global) {
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
-                    uint32_t bfr[4];
+                    uint32_t bfr[4], afr[4];
+                    ldsm_x4(a_addr<kLdW>(sb + Ly::K, wk0, kk, lane), afr);
                     ldsm_x4(b_addr<kLdW>(stg + Ly::Q_OFF, 16 * qc, kk, lane), bfr);
-                    mma_bf16_16816(sl[0], ka[kk], bfr[0], bfr[1]);
-                    mma_bf16_16816(sl[1], ka[kk], bfr[2], bfr[3]);
+                    mma_bf16_16816(sl[0], afr, bfr[0], bfr[1]);
+                    mma_bf16_16816(sl[1], afr, bfr[2], bfr[3]);
                 }
             }
             if (!all_local) {
@@ -585,10 +583,11 @@ __global__ void __launch_bounds__(kTc) bwd_dkv_tc_kernel(Args a)
             if (!all_global) {
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
-                    uint32_t bfr[4];
+                    uint32_t bfr[4], afr[4];
+                    ldsm_x4(a_addr<kLdW>(sb + Ly::V, wk0, kk, lane), afr);
                     ldsm_x4(b_addr<kLdW>(stg + Ly::DO_OFF, 16 * qc, kk, lane), bfr);
-                    mma_bf16_16816(dpl[0], va[kk], bfr[0], bfr[1]);
-                    mma_bf16_16816(dpl[1], va[kk], bfr[2], bfr[3]);
+                    mma_bf16_16816(dpl[0], afr, bfr[0], bfr[1]);
+                    mma_bf16_16816(dpl[1], afr, bfr[2], bfr[3]);
                 }
             }
             if (!all_local) {
