@@ -18,7 +18,9 @@
 //   dUk = sum_i dq~_i^T q_i (dq~_i = scale sum_global dS_ij k^D_j),
 //   dUv = sum_i O^D_i^T dO_i (O^D_i = sum_global p_ij v^D_j).
 //
-// Kernels (fp32 arithmetic on the CUDA cores, both storage types):
+// Kernels (fp32 arithmetic on the CUDA cores; used for fp32 storage and for
+// bf16 with d_down = 8 -- other bf16 shapes run steps 2 and 3 on the tensor
+// cores, dar_backward_tc.cu, and share steps 1 and 4):
 //  1. bwd_rows: per row, q~, dO~ and D (one warp per row, Uk and Uv staged
 //     in shared memory per KV head).
 //  2. bwd_dq: per 64-row query tile, the row log-sum-exp (first pass over the
