@@ -193,3 +193,48 @@ def test_direct_and_backward_reject_bad_arguments(lib):
     n = L.dar_attn_backward_workspace_bytes(lib.DAR_BF16, 1, 4, 2, 16, 16)
     assert n > 0 and n % 256 == 0
     assert L.dar_attn_backward_workspace_bytes(lib.DAR_BF16, 1, 3, 2, 16, 16) == 0
+
+
+def _latent(lib, **kw):
+    c = dict(B=2, Hkv=2, d=64, D=128, d_lat=64, w=8, max_pages_per_seq=4, num_pages=8, win_k=256, win_v=512,
+             pool_c=768, block_table=1024, seq_lens=1280, status=1536)
+    c.update(kw)
+    return lib.dar_latent_cache(*[c[f] for f, _ in lib.dar_latent_cache._fields_])
+
+
+def test_latent_entry_points_reject_bad_arguments(lib):
+    """The latent form's entry points refuse bad shapes and pointers on the
+    host, with the documented codes, and launch nothing."""
+    L = lib.load_library()
+    P = 4096
+    c = _latent(lib)
+    ws = L.dar_latent_decode_workspace_bytes(ctypes.byref(c), 4)
+    assert ws > 0 and ws % 256 == 0
+    assert L.dar_latent_decode_workspace_bytes(ctypes.byref(c), 3) == 0          # Hq not a multiple of Hkv
+    assert L.dar_latent_decode_workspace_bytes(ctypes.byref(c), 34) == 0         # more than 32 query heads
+
+    def dec(cache=c, Hq=4, q=P, wsb=1 << 30):
+        return L.dar_latent_decode(ctypes.byref(cache), Hq, q, P, P, 0.0, P, P, wsb, None)
+    assert dec(cache=_latent(lib, d_lat=96)) == 2     # d_lat not built
+    assert dec(cache=_latent(lib, d=32)) == 2         # head dimension not built
+    assert dec(cache=_latent(lib, B=1025)) == 2       # beyond the decode's batch limit
+    assert dec(Hq=64) == 2                            # more than 32 query heads
+    assert dec(Hq=3) == 1
+    assert dec(q=0) == 1
+    assert dec(q=P + 4) == 1                          # misaligned
+    assert dec(wsb=16) == 3                           # workspace too small
+    assert "workspace" in L.dar_last_error().decode()
+    assert dec(cache=_latent(lib, B=0)) == 0          # nothing to do
+
+    def app(cache=c, h=P, n=4, W=P):
+        return L.dar_latent_append(ctypes.byref(cache), h, P, P, n, None, W, None)
+    assert app(h=0) == 1
+    assert app(n=-1) == 1
+    assert app(W=P + 8) == 1
+    assert app(cache=_latent(lib, D=8193)) == 2       # hidden width beyond the staging limit
+    assert app(cache=_latent(lib, w=0)) == 1
+    assert app(n=0) == 0
+
+    assert L.dar_latent_absorb(2, 128, 32, 64, P, P, P, P, P, None) == 2   # d != 64
+    assert L.dar_latent_absorb(0, 128, 64, 64, P, P, P, P, P, None) == 1   # no KV head
+    assert L.dar_latent_absorb(2, 128, 64, 64, P, None, P, P, P, None) == 1
