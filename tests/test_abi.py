@@ -238,3 +238,32 @@ def test_latent_entry_points_reject_bad_arguments(lib):
     assert L.dar_latent_absorb(2, 128, 32, 64, P, P, P, P, P, None) == 2   # d != 64
     assert L.dar_latent_absorb(0, 128, 64, 64, P, P, P, P, P, None) == 1   # no KV head
     assert L.dar_latent_absorb(2, 128, 64, 64, P, None, P, P, P, None) == 1
+
+
+def test_chunk_and_down_project_reject_bad_arguments(lib):
+    """dar_prefill_chunk (bf16, d_down >= 16) and dar_down_project refuse bad
+    arguments on the host with the documented codes."""
+    L = lib.load_library()
+    P = 4096
+    c = _cache(lib)
+    n_ws = L.dar_prefill_chunk_workspace_bytes(ctypes.byref(c), 100)
+    assert n_ws > 0 and n_ws % 256 == 0
+
+    def chunk(cache=c, Hq=4, n=100, q=P, wsb=1 << 30):
+        return L.dar_prefill_chunk(ctypes.byref(cache), Hq, n, q, P, P, P, P, P, P, 0.0, P, P, wsb, None)
+    assert chunk(cache=_cache(lib, dtype=lib.DAR_F32)) == 2   # bf16 caches only
+    assert chunk(cache=_cache(lib, d_down=8)) == 2            # d_down >= 16
+    assert chunk(Hq=3) == 1
+    assert chunk(n=-2) == 1
+    assert chunk(q=P + 2) == 1
+    assert chunk(wsb=16) == 3
+    assert chunk(n=0) == 0
+
+    def dp(B=1, n=10, d=64, dd=16, x=P, W=P, out=P):
+        return L.dar_down_project(lib.DAR_BF16, B, 2, n, d, dd, x, W, out, None)
+    assert dp(d=32) == 2
+    assert dp(dd=12) == 2
+    assert dp(n=-1) == 1
+    assert dp(x=0) == 1
+    assert dp(out=P + 2) == 1
+    assert dp(n=0) == 0
