@@ -699,7 +699,9 @@ def run_ours(args, world, rank, local):
         prefill = prefill_section(args, torch, dar, W, I, dev, stream, tc_peak, peak_src, local)
 
     extra = None
-    if args.only == "all" and not args.no_sweep:
+    # the other workloads and the NEXT rows are measured on single-GPU runs
+    # (a multi-GPU run reports the replicated step only, to stay short)
+    if args.only == "all" and not args.no_sweep and world == 1:
         del wls, outs, saved, restore, steps_graph
         torch.cuda.empty_cache()
         gqa = decode_only_point(torch, dar, I, W, I.DECODE_1B_GQA, K, l2, dev, stream, hbm_peak)
